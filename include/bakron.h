@@ -1,0 +1,141 @@
+/*
+ * bakron.h -- C ABI of the GB300 BaKron solver (libbakron.so).
+ *
+ * BaKron ("Babai quantization for Kronecker-factored Hessians") rounds an
+ * m x n weight matrix W onto a quantisation alphabet by Babai nearest-plane /
+ * GPTQ error feedback under the Hessian H = A (x) B, with A (n x n) the
+ * input-side and B (m x m) the output-side SPD Kronecker factor (paper,
+ * Sec. 3, Alg. 2-5).  The factors enter through their unit-lower forms
+ * L^A = Cholesky(A^-1), L^B = Cholesky(B^-1) with columns scaled to a unit
+ * diagonal (Alg. 1/2, first two lines), and entry (i, j) is rounded at
+ *
+ *     X_ij = W_ij + sum_{(p,q) < (i,j)} L^B_ip E_pq L^A_jq,   E = V - X,
+ *
+ * the order-free definition of the equivalence proof (Appendix, Eq.
+ * canonical-antidiagonal).  All anti-diagonals i + j = k are independent, so
+ * the solve takes m + n - 1 dependent rounding steps, and the bulk error
+ * propagation follows Alg. 5 (recursive halving of the anti-diagonal range),
+ * O(mn(m+n)) work in total (Appendix, complexity of BaKron).
+ *
+ * Conventions for every entry point:
+ *  - Matrices are row-major.  Pointers marked "device" are CUDA device memory
+ *    owned by the caller; the library never allocates, frees or retains them,
+ *    and keeps no state between calls other than read-only constant tables.
+ *  - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is
+ *    enqueued asynchronously on it unless stated otherwise.
+ *  - Arguments are validated on the host before anything is enqueued; an
+ *    invalid argument returns BAKRON_ERR_INVALID_ARG and enqueues nothing.
+ *  - Errors found on the device (a non-positive Cholesky pivot, a non-finite
+ *    value) are recorded in a status word inside the workspace; entry points
+ *    that synchronise return it, and bakron_read_status() returns it later.
+ *    No kernel traps or aborts.
+ *  - Only the lower triangles of A and B are read.
+ */
+#ifndef BAKRON_H_
+#define BAKRON_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  BAKRON_OK = 0,
+  BAKRON_ERR_INVALID_ARG = 1,   /* bad pointer, size, bits, group, dtype      */
+  BAKRON_ERR_NOT_SPD = 2,       /* damped A or B not positive definite        */
+  BAKRON_ERR_CUDA = 3,          /* a CUDA runtime call failed                 */
+  BAKRON_ERR_TIMEOUT = 4,       /* a bounded device wait ran out              */
+  BAKRON_ERR_WORKSPACE = 5,     /* workspace smaller than required            */
+  BAKRON_ERR_NONFINITE = 6      /* NaN/Inf met while rounding                 */
+} bakron_status;
+
+typedef enum { BAKRON_F32 = 0, BAKRON_BF16 = 1 } bakron_dtype;
+
+/* Bytes of the opaque factor buffer for an m x n problem (L^A, L^B and the
+ * RevCholesky diagonals, padded to the kernels' tile size). */
+size_t bakron_factors_bytes(int m, int n);
+
+/* Bytes of scratch a call to bakron_prepare or bakron_solve needs for an
+ * m x n problem (the larger of the two; one buffer serves both). */
+size_t bakron_workspace_bytes(int m, int n);
+
+/*
+ * bakron_prepare -- damp A and B and build their unit-lower factors.
+ * Paper: Alg. 2 first two lines; damping as in Sec. 4 and Appendix
+ * "Experiments" (H + damp * mean(diag H) * I).  Computed as
+ * L = RevCholesky(H_d)^-1 diag(RevCholesky(H_d)), which equals the
+ * normalised Cholesky(H_d^-1) without forming the inverse.
+ *   A        device, n x n fp32, input-side Gram (lower triangle read)
+ *   B        device, m x m fp32, output-side Gram (lower triangle read)
+ *   damp     >= 0, relative diagonal damping
+ *   factors  device, bakron_factors_bytes(m, n) bytes, written
+ *   workspace device, >= bakron_workspace_bytes(m, n) bytes, scratch
+ * Synchronises `stream` at the end and returns BAKRON_ERR_NOT_SPD if a pivot
+ * of the damped A or B was not positive (factors are then undefined).
+ */
+int bakron_prepare(const float* A, const float* B, int m, int n, float damp,
+                   void* factors, void* workspace, size_t workspace_bytes,
+                   void* stream);
+
+/*
+ * bakron_set_factors -- fill a factor buffer from given unit-lower factors.
+ *   LA  device, n x n fp32 row-major; strictly-lower part read, diagonal = 1
+ *   LB  device, m x m fp32 row-major; likewise
+ *   rA, rB  device, length n and m, the RevCholesky diagonals (may be NULL;
+ *           they are only stored for the caller)
+ * Asynchronous.
+ */
+int bakron_set_factors(const float* LA, const float* LB, const float* rA,
+                       const float* rB, int m, int n, void* factors,
+                       void* stream);
+
+/*
+ * bakron_get_factors -- copy the unit-lower factors and RevCholesky
+ * diagonals out of a factor buffer (device destinations; any may be NULL).
+ * Asynchronous.
+ */
+int bakron_get_factors(const void* factors, int m, int n, float* LA,
+                       float* LB, float* rA, float* rB, void* stream);
+
+/*
+ * bakron_solve -- BaKron rounding of W (paper, Alg. 5; result defined by the
+ * equivalence proof's canonical recursion).
+ *   W        device, m rows of n values, row stride ldw elements (>= n),
+ *            dtype BAKRON_F32 or BAKRON_BF16 (bf16 is widened exactly)
+ *   factors  device, from bakron_prepare or bakron_set_factors
+ *   bits     1..8: the alphabet is {0, ..., 2^bits - 1}
+ *   group_size 0 for one grid per row, else a divisor of n: one grid per
+ *            (row, group of group_size columns)
+ *   codes    device, m x n uint8, written (row stride n)
+ *   scales, zeros  device, m x G fp32 (G = 1 or n / group_size), written:
+ *            the grid of each row/group, from the ORIGINAL W: xmin =
+ *            min(0, min w), xmax = max(0, max w) ([-1, 1] if both are 0),
+ *            s = (xmax - xmin) / (2^bits - 1), z = rint(-xmin / s), all in
+ *            fp32; value of code c is s * (c - z)
+ *   prerounding device, m x n fp32 (row stride n), or NULL: the value each
+ *            entry was rounded at (the paper's in-place workspace)
+ *   workspace device, >= bakron_workspace_bytes(m, n) bytes, scratch
+ *   sync     nonzero: synchronise `stream` and return the device status;
+ *            zero: fully asynchronous (use bakron_read_status afterwards)
+ * Codes are c = clamp(rint(x / s) + z, 0, 2^bits - 1), round half to even.
+ */
+int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw,
+                 const void* factors, int bits, int group_size,
+                 uint8_t* codes, float* scales, float* zeros,
+                 float* prerounding, void* workspace, size_t workspace_bytes,
+                 int sync, void* stream);
+
+/* Synchronise `stream`, return and clear the device status word kept in
+ * `workspace` by the last prepare/solve that used it. */
+int bakron_read_status(void* workspace, void* stream);
+
+/* Static description of a status code. */
+const char* bakron_strerror(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BAKRON_H_ */

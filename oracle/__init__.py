@@ -10,4 +10,5 @@ from .bakron_oracle import (Factors, Grid, Result, bakron, bakron_antidiagonal, 
                             error_bound, gptq_rows, integer_grid, midpoint_distance,
                             objective, objective_from_errors, prepare, quant_grid,
                             quantize, rev_cholesky, rtn, teacher_forced,
-                            unit_lower_factor, unit_lower_factor_via_rev)
+                            unit_lower_factor, unit_lower_factor_via_rev,
+                            certificate_rows, grid_rows)

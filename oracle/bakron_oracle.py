@@ -457,3 +457,32 @@ def babai_step_by_enumeration(x, s, z, qmax):
         even = [i for i in idx if (int(cands[i] - z) % 2) == 0]
         return int(cands[even[0]] if even else cands[idx[0]])
     return int(cands[idx[0]])
+
+
+def certificate_rows(W_rows, codes_rows, D_rows_above, grid_rows, RA, RB_rows, rows):
+    """The certificate on a subset of rows, from RevCholesky factors.
+
+    With L^-1 = diag(R)^-1 R (R = RevCholesky), E = diag(R_B)^-1 R_B (V - W)
+    R_A^T diag(R_A)^-1.  For a set of rows P, (R_B (V - W))[P] needs R_B[P, :]
+    and (V - W) on rows 0..max(P) only, so large problems are checked on
+    sampled row blocks without the full m x m solve.
+      W_rows, codes_rows : W and codes on rows P (|P| x n)
+      D_rows_above       : (V - W) on rows 0..max(P) (as needed by R_B[P, :])
+      grid_rows          : Grid restricted to rows P
+      RA                 : RevCholesky(A_d), n x n
+      RB_rows            : R_B[P, 0:max(P)+1]
+      rows               : the row indices P
+    Returns (X on P, mismatch mask, midpoint distance) like ``certificate``."""
+    n = W_rows.shape[1]
+    S, Z = grid_rows.expand(n)
+    rbd = np.array([RB_rows[k, r] for k, r in enumerate(rows)], dtype=F64)
+    Y = (RB_rows @ D_rows_above) / rbd[:, None]            # diag(R_B)^-1 R_B (V - W), rows P
+    E = (Y @ RA.T) / np.diag(RA)[None, :]
+    V = S * (np.asarray(codes_rows, F64) - Z)
+    X = V - E
+    c, _ = quantize(X, S, Z, grid_rows.qmax)
+    return X, c != codes_rows, midpoint_distance(X, S)
+
+
+def grid_rows(grid: Grid, rows) -> Grid:
+    return Grid(grid.s[rows], grid.z[rows], grid.qmax, grid.group)

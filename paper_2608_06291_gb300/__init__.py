@@ -1,0 +1,10 @@
+"""GB300-native BaKron solver: two-sided Babai/GPTQ rounding under A (x) B.
+
+The compute path is libbakron.so (hand-written sm_103a CUDA kernels behind the
+C ABI in include/bakron.h); this package is its build script and a thin
+ctypes binding with the same entry-point names.
+"""
+from .bakron import (BakronError, Factors, alloc_workspace, bakron_get_factors,  # noqa: F401
+                     bakron_prepare, bakron_read_status, bakron_set_factors, bakron_solve,
+                     dequantize, factors_bytes, lib, library_path, strerror, workspace_bytes)
+from .buildlib import build  # noqa: F401

@@ -1,0 +1,186 @@
+"""Thin ctypes binding of libbakron.so (include/bakron.h), same names as the C ABI.
+
+Only argument marshalling lives here: every step of the solve runs in the
+library's CUDA kernels.  torch supplies device memory and the current stream.
+If the library is missing this module raises; there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import buildlib as _build
+
+OK, ERR_INVALID_ARG, ERR_NOT_SPD, ERR_CUDA, ERR_TIMEOUT, ERR_WORKSPACE, ERR_NONFINITE = range(7)
+F32, BF16 = 0, 1
+
+_lib = None
+
+
+class BakronError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {strerror(status)} (status {status})")
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib() -> ctypes.CDLL:
+    """Load libbakron.so (built by ``build()``); raise if it is absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with "
+                           "paper_2608_06291_gb300.build.build() (no CPU fallback exists)")
+    L = ctypes.CDLL(path)
+    vp, i32, i64, sz, f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_size_t, ctypes.c_float
+    L.bakron_factors_bytes.argtypes = [i32, i32]
+    L.bakron_factors_bytes.restype = sz
+    L.bakron_workspace_bytes.argtypes = [i32, i32]
+    L.bakron_workspace_bytes.restype = sz
+    L.bakron_prepare.argtypes = [vp, vp, i32, i32, f32, vp, vp, sz, vp]
+    L.bakron_prepare.restype = i32
+    L.bakron_set_factors.argtypes = [vp, vp, vp, vp, i32, i32, vp, vp]
+    L.bakron_set_factors.restype = i32
+    L.bakron_get_factors.argtypes = [vp, i32, i32, vp, vp, vp, vp, vp]
+    L.bakron_get_factors.restype = i32
+    L.bakron_solve.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, vp, sz, i32, vp]
+    L.bakron_solve.restype = i32
+    L.bakron_read_status.argtypes = [vp, vp]
+    L.bakron_read_status.restype = i32
+    L.bakron_strerror.argtypes = [i32]
+    L.bakron_strerror.restype = ctypes.c_char_p
+    _lib = L
+    return L
+
+
+def strerror(status: int) -> str:
+    return lib().bakron_strerror(int(status)).decode()
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _check(rc, what):
+    if rc != OK:
+        raise BakronError(rc, what)
+
+
+def factors_bytes(m: int, n: int) -> int:
+    return int(lib().bakron_factors_bytes(m, n))
+
+
+def workspace_bytes(m: int, n: int) -> int:
+    return int(lib().bakron_workspace_bytes(m, n))
+
+
+def alloc_workspace(m: int, n: int, device="cuda") -> torch.Tensor:
+    return torch.empty(workspace_bytes(m, n), dtype=torch.uint8, device=device)
+
+
+class Factors:
+    """Opaque device factor buffer for an m x n problem."""
+
+    def __init__(self, m: int, n: int, device="cuda"):
+        self.m, self.n = m, n
+        self.buf = torch.empty(factors_bytes(m, n), dtype=torch.uint8, device=device)
+
+
+def _as_f32_square(t, d, name):
+    if t.dtype != torch.float32 or t.dim() != 2 or tuple(t.shape) != (d, d) or not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA float32 {d}x{d} tensor")
+    return t.contiguous()
+
+
+def bakron_prepare(A, B, damp: float = 0.01, workspace=None, stream=None) -> Factors:
+    n, m = A.shape[0], B.shape[0]
+    A = _as_f32_square(A, n, "A")
+    B = _as_f32_square(B, m, "B")
+    f = Factors(m, n, A.device)
+    ws = workspace if workspace is not None else alloc_workspace(m, n, A.device)
+    rc = lib().bakron_prepare(_ptr(A), _ptr(B), m, n, float(damp), _ptr(f.buf), _ptr(ws),
+                              ws.numel(), _stream(stream))
+    _check(rc, "bakron_prepare")
+    return f
+
+
+def bakron_set_factors(LA, LB, rA=None, rB=None, stream=None) -> Factors:
+    n, m = LA.shape[0], LB.shape[0]
+    LA = _as_f32_square(LA, n, "LA")
+    LB = _as_f32_square(LB, m, "LB")
+    rA = None if rA is None else rA.contiguous().float()
+    rB = None if rB is None else rB.contiguous().float()
+    f = Factors(m, n, LA.device)
+    rc = lib().bakron_set_factors(_ptr(LA), _ptr(LB), _ptr(rA), _ptr(rB), m, n, _ptr(f.buf),
+                                  _stream(stream))
+    _check(rc, "bakron_set_factors")
+    return f
+
+
+def bakron_get_factors(f: Factors, stream=None):
+    dev = f.buf.device
+    LA = torch.empty(f.n, f.n, dtype=torch.float32, device=dev)
+    LB = torch.empty(f.m, f.m, dtype=torch.float32, device=dev)
+    rA = torch.empty(f.n, dtype=torch.float32, device=dev)
+    rB = torch.empty(f.m, dtype=torch.float32, device=dev)
+    rc = lib().bakron_get_factors(_ptr(f.buf), f.m, f.n, _ptr(LA), _ptr(LB), _ptr(rA), _ptr(rB),
+                                  _stream(stream))
+    _check(rc, "bakron_get_factors")
+    return LA, LB, rA, rB
+
+
+def bakron_solve(W, f: Factors, bits: int, group_size: int = 0, workspace=None,
+                 prerounding: bool = False, sync: bool = True, out=None, stream=None):
+    """Round W (CUDA fp32/bf16, unit column stride).  Returns (codes uint8,
+    scales, zeros[, prerounding fp32])."""
+    if not W.is_cuda or W.dim() != 2 or W.stride(1) != 1:
+        raise ValueError("W must be a 2-D CUDA tensor with unit column stride")
+    if W.dtype == torch.float32:
+        dt = F32
+    elif W.dtype == torch.bfloat16:
+        dt = BF16
+    else:
+        raise ValueError("W must be float32 or bfloat16")
+    m, n = W.shape
+    if (f.m, f.n) != (m, n):
+        raise ValueError("factor buffer was built for a different shape")
+    G = 1 if group_size == 0 else n // group_size
+    dev = W.device
+    if out is None:
+        codes = torch.empty(m, n, dtype=torch.uint8, device=dev)
+        scales = torch.empty(m, G, dtype=torch.float32, device=dev)
+        zeros = torch.empty(m, G, dtype=torch.float32, device=dev)
+        xpre = torch.empty(m, n, dtype=torch.float32, device=dev) if prerounding else None
+    else:
+        codes, scales, zeros, xpre = out
+    ws = workspace if workspace is not None else alloc_workspace(m, n, dev)
+    rc = lib().bakron_solve(_ptr(W), dt, m, n, W.stride(0), _ptr(f.buf), int(bits),
+                            int(group_size), _ptr(codes), _ptr(scales), _ptr(zeros), _ptr(xpre),
+                            _ptr(ws), ws.numel(), 1 if sync else 0, _stream(stream))
+    _check(rc, "bakron_solve")
+    return (codes, scales, zeros, xpre) if prerounding else (codes, scales, zeros)
+
+
+def bakron_read_status(workspace, stream=None) -> int:
+    return int(lib().bakron_read_status(_ptr(workspace), _stream(stream)))
+
+
+def dequantize(codes, scales, zeros):
+    """Values s * (c - z) of a code matrix (a convenience for callers)."""
+    m, n = codes.shape
+    g = n // scales.shape[1]
+    s = scales.repeat_interleave(g, dim=1)
+    z = zeros.repeat_interleave(g, dim=1)
+    return s * (codes.float() - z)

@@ -1,0 +1,90 @@
+// Shared definitions of the BaKron CUDA library: buffer layouts, tile sizes,
+// status handling.  Everything here is internal; the C ABI is include/bakron.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <stddef.h>
+
+#include "../../include/bakron.h"
+
+namespace bakron {
+
+// Leaf tile: one warp rounds a TILE x TILE block of W by walking its
+// 2*TILE-1 anti-diagonals (lane = column).
+constexpr int TILE = 32;
+// All matrices are padded to this multiple in both dimensions, so that the
+// GEMM kernels see whole 128 x 128 blocks and TMA boxes never straddle an edge.
+constexpr int PAD = 128;
+
+__host__ __device__ inline int64_t round_up(int64_t x, int64_t r) {
+  return (x + r - 1) / r * r;
+}
+__host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
+
+inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Factor buffer: [L^B  mp x mp][L^A  np x np][rB  mp][rA  np], fp32, each
+// section 256-byte aligned.  L^X is stored dense row-major with exact zeros
+// above the diagonal, ones on it, and an identity extension over the padding.
+struct FactorLayout {
+  int m, n;
+  int64_t mp, np;
+  size_t off_LB, off_LA, off_rB, off_rA, bytes;
+  explicit FactorLayout(int m_, int n_) : m(m_), n(n_) {
+    mp = round_up(m, PAD);
+    np = round_up(n, PAD);
+    off_LB = 0;
+    off_LA = align256(off_LB + size_t(mp * mp) * 4);
+    off_rB = align256(off_LA + size_t(np * np) * 4);
+    off_rA = align256(off_rB + size_t(mp) * 4);
+    bytes = align256(off_rA + size_t(np) * 4);
+  }
+};
+
+// Workspace: [status 256 B][solve: X, E, M  (mp x np fp32 each)] or
+//            [status 256 B][prepare: C, Linv (dp x dp fp64/fp32), scratch].
+struct SolveLayout {
+  int64_t mp, np;
+  size_t off_status, off_X, off_E, off_M, bytes;
+  SolveLayout(int m, int n) {
+    mp = round_up(m, PAD);
+    np = round_up(n, PAD);
+    off_status = 0;
+    off_X = 256;
+    off_E = align256(off_X + size_t(mp * np) * 4);
+    off_M = align256(off_E + size_t(mp * np) * 4);
+    bytes = align256(off_M + size_t(mp * np) * 4);
+  }
+};
+
+// Prepare works on one Gram at a time (the larger side bounds the size).
+// Real type of the factorisation: fp64 (see prepare.cu for the reason).
+struct PrepareLayout {
+  int64_t dp;
+  size_t off_status, off_C, off_Linv, off_T, off_scalar, bytes;
+  PrepareLayout(int m, int n) {
+    int64_t d = m > n ? m : n;
+    dp = round_up(d, PAD);
+    off_status = 0;
+    off_C = 256;
+    off_Linv = align256(off_C + size_t(dp * dp) * 8);
+    off_T = align256(off_Linv + size_t(dp * dp) * 8);
+    off_scalar = align256(off_T + size_t(dp * PAD) * 8);
+    bytes = align256(off_scalar + 256);
+  }
+};
+
+// Device status word (first int of every workspace).  Kernels only ever raise
+// it with atomicMax-free writes of a nonzero code; the host reads and clears.
+__device__ inline void raise_status(int* status, int code) {
+  atomicCAS(status, 0, code);
+}
+
+}  // namespace bakron
+
+#define BK_CUDA_OK(expr)                                   \
+  do {                                                     \
+    cudaError_t err__ = (expr);                            \
+    if (err__ != cudaSuccess) return BAKRON_ERR_CUDA;      \
+  } while (0)

@@ -1,0 +1,31 @@
+"""Shared test helpers: oracle runs on the exact inputs the GPU receives."""
+import numpy as np
+import torch
+
+import oracle as O
+
+TIE_BAND = 1e-4   # grid units: |x/s - (k + 1/2)| below this is a tie (spec bar)
+
+
+def to_np(t):
+    return t.detach().to("cpu", torch.float64).numpy()
+
+
+def oracle_factors_fp32(A, B, damp):
+    """Oracle factors rounded to fp32 (what the GPU solve receives) and the
+    same values back in fp64 (what the oracle solves with)."""
+    f = O.prepare(to_np(A), to_np(B), damp, via_inverse=False)
+    LA32 = f.LA.astype(np.float32)
+    LB32 = f.LB.astype(np.float32)
+    return f, LA32, LB32
+
+
+def compare_codes(W64, codes_gpu, g, LA64, LB64, ref_codes=None):
+    """Teacher-forced certificate + raw match.  Returns a dict of statistics."""
+    X, bad, dist = O.certificate(W64, codes_gpu, g, LA64, LB64)
+    out = {"cert_mismatch": int(bad.sum()),
+           "cert_mismatch_outside_band": int((bad & (dist >= TIE_BAND)).sum()),
+           "n": codes_gpu.size, "X": X}
+    if ref_codes is not None:
+        out["raw_match"] = float((ref_codes == codes_gpu).mean())
+    return out

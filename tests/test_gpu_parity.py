@@ -1,0 +1,192 @@
+"""GPU parity: the CUDA path through the C ABI against the float64 oracle.
+
+Small problems are compared free-running (identical codes, pre-rounding
+values within 1e-4 grid units, objective within 1e-4 relative) on inputs
+that span several 32 x 32 tiles and ragged tails; every comparison also runs
+the teacher-forced certificate (codes may differ from the oracle's rounding
+of their own pre-rounding values only inside the 1e-4 tie band).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import workloads as WL
+from tests._helpers import TIE_BAND, compare_codes, oracle_factors_fp32, to_np
+
+pytestmark = pytest.mark.gpu
+
+if torch.cuda.is_available():
+    import paper_2608_06291_gb300 as P
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    P.build()
+    P.lib()
+
+
+def _solve_small(m, n, seed, bits, group=0, wdtype=torch.float32, ldw_pad=0, w_scale=1.0):
+    W, A, B = WL.small_problem(m, n, seed)
+    W = W * w_scale
+    f, LA32, LB32 = oracle_factors_fp32(A, B, 0.01)
+    dev = "cuda"
+    fac = P.bakron_set_factors(torch.from_numpy(LA32).to(dev), torch.from_numpy(LB32).to(dev),
+                               torch.from_numpy(f.rA.astype(np.float32)).to(dev),
+                               torch.from_numpy(f.rB.astype(np.float32)).to(dev))
+    if ldw_pad:
+        Wbig = torch.zeros(m, n + ldw_pad, dtype=torch.float32)
+        Wbig[:, :n] = W
+        Wd = Wbig.to(dev, wdtype)[:, :n]
+    else:
+        Wd = W.to(dev, wdtype)
+    codes, scales, zeros, X = P.bakron_solve(Wd, fac, bits, group, prerounding=True)
+    torch.cuda.synchronize()
+    W64 = to_np(Wd.float())
+    g = O.quant_grid(W64, bits, group)
+    ref = O.bakron_recursive(W64, LA32.astype(np.float64), LB32.astype(np.float64), g)
+    return dict(W=W64, f=f, g=g, LA=LA32.astype(np.float64), LB=LB32.astype(np.float64),
+                codes=codes.cpu().numpy().astype(np.int64), scales=scales.cpu().numpy(),
+                zeros=zeros.cpu().numpy(), X=X.cpu().numpy().astype(np.float64), ref=ref)
+
+
+def _assert_parity(r):
+    g = r["g"]
+    # grid: bit-identical fp32 scales and zeros
+    np.testing.assert_array_equal(r["scales"], g.s)
+    np.testing.assert_array_equal(r["zeros"], g.z)
+    st = compare_codes(r["W"], r["codes"], g, r["LA"], r["LB"], r["ref"].codes)
+    assert st["cert_mismatch_outside_band"] == 0, st
+    assert st["raw_match"] >= 0.999, st
+    S, _ = g.expand(r["W"].shape[1])
+    same = r["codes"] == r["ref"].codes
+    if same.all():
+        dx = np.abs(r["X"] - r["ref"].X) / S
+        assert dx.max() < TIE_BAND, dx.max()
+        V = O.dequantize(r["codes"], g, r["W"].shape[1])
+        o_gpu = O.objective(r["W"], V, r["f"].A_d, r["f"].B_d)
+        o_ref = O.objective(r["W"], r["ref"].V, r["f"].A_d, r["f"].B_d)
+        assert abs(o_gpu - o_ref) <= 1e-4 * o_ref
+
+
+SHAPES = [(1, 1), (1, 40), (40, 1), (5, 7), (32, 32), (33, 65), (64, 96), (100, 70), (97, 131)]
+
+
+@pytest.mark.parametrize("m,n", SHAPES)
+def test_solve_matches_oracle_shapes(m, n):
+    _assert_parity(_solve_small(m, n, 1000 + m + 3 * n, bits=4))
+
+
+@pytest.mark.parametrize("bits", [1, 2, 3, 8])
+def test_solve_matches_oracle_bits(bits):
+    _assert_parity(_solve_small(70, 90, 77 + bits, bits=bits))
+
+
+@pytest.mark.parametrize("group", [32, 64, 96, 48])
+def test_solve_matches_oracle_groups(group):
+    _assert_parity(_solve_small(45, 192, 12 + group, bits=4, group=group))
+
+
+def test_solve_bf16_and_strided_w():
+    _assert_parity(_solve_small(66, 100, 5, bits=4, wdtype=torch.bfloat16))
+    _assert_parity(_solve_small(66, 100, 6, bits=3, ldw_pad=28))
+
+
+def test_zero_rows_use_unit_grid():
+    r = _solve_small(40, 50, 9, bits=4)
+    W = np.zeros((3, 50))
+    g = O.quant_grid(W, 4)
+    assert np.all(g.s > 0)
+    # a solve with an all-zero W: every code is the zero point
+    fac = P.bakron_set_factors(torch.eye(50, device="cuda"), torch.eye(3, device="cuda"))
+    codes, scales, zeros = P.bakron_solve(torch.zeros(3, 50, device="cuda"), fac, 4)
+    assert (codes.cpu().numpy() == zeros.cpu().numpy().astype(np.uint8)).all()
+    _assert_parity(r)
+
+
+def test_config1_end_to_end():
+    """Config 1 (128 x 128, 4-bit per row): GPU prepare + GPU solve vs the
+    oracle with its own fp64 factors.  Free-running codes and objective."""
+    W, A, B = WL.make(1)
+    cfg = WL.CONFIGS[1]
+    fac = P.bakron_prepare(A.cuda(), B.cuda(), cfg.damp)
+    codes, scales, zeros = P.bakron_solve(W.cuda(), fac, cfg.bits, cfg.group)
+    W64 = to_np(W)
+    f = O.prepare(to_np(A), to_np(B), cfg.damp)
+    g = O.quant_grid(W64, cfg.bits, cfg.group)
+    ref = O.bakron_recursive(W64, f.LA, f.LB, g)
+    c = codes.cpu().numpy().astype(np.int64)
+    st = compare_codes(W64, c, g, f.LA, f.LB, ref.codes)
+    assert st["raw_match"] >= 0.999 and st["cert_mismatch_outside_band"] == 0, st
+    V = O.dequantize(c, g, 128)
+    o_gpu, o_ref = O.objective(W64, V, f.A_d, f.B_d), O.objective(W64, ref.V, f.A_d, f.B_d)
+    assert abs(o_gpu - o_ref) <= 1e-4 * o_ref
+    assert o_gpu < O.objective(W64, O.rtn(W64, g).V, f.A_d, f.B_d)
+
+
+@pytest.mark.parametrize("d", [1, 2, 5, 63, 64, 65, 130, 300])
+def test_prepare_matches_oracle(d):
+    """Device factors vs LAPACK fp64 (computed in fp64 on the device, stored fp32)."""
+    _, A, B = WL.small_problem(d + 3, d, 400 + d)
+    fac = P.bakron_prepare(A.cuda(), B.cuda(), 0.01)
+    LA, LB, rA, rB = (t.cpu().numpy().astype(np.float64) for t in P.bakron_get_factors(fac))
+    f = O.prepare(to_np(A), to_np(B), 0.01)
+    for got, want in ((LA, f.LA), (LB, f.LB)):
+        assert np.allclose(np.triu(got, 1), 0)
+        np.testing.assert_array_equal(np.diag(got), 1.0)
+        # fp64 factorisation rounded once to fp32: relative 2^-24 of each
+        # entry plus kappa * 2^-52 accumulated error
+        np.testing.assert_allclose(got, want, rtol=2e-7, atol=1e-9 * np.abs(want).max())
+    np.testing.assert_allclose(rA, f.rA, rtol=2e-7)
+    np.testing.assert_allclose(rB, f.rB, rtol=2e-7)
+
+
+def test_prepare_rejects_indefinite():
+    _, A, B = WL.small_problem(70, 70, 3)
+    A = A.clone()
+    A[5, 5] = -50.0  # pivot goes negative after damping
+    ws = P.alloc_workspace(70, 70)
+    with pytest.raises(P.BakronError) as e:
+        P.bakron_prepare(A.cuda(), B.cuda(), 0.01, workspace=ws)
+    assert e.value.status == 2
+    # the context is still usable and the status word was cleared
+    fac = P.bakron_prepare(B.cuda(), B.cuda(), 0.01, workspace=ws)
+    assert fac is not None
+
+
+def test_nonfinite_input_is_reported():
+    fac = P.bakron_set_factors(torch.eye(40, device="cuda"), torch.eye(8, device="cuda"))
+    W = torch.randn(8, 40, device="cuda")
+    W[3, 7] = float("nan")
+    with pytest.raises(P.BakronError) as e:
+        P.bakron_solve(W, fac, 4)
+    assert e.value.status == 6
+
+
+def test_invalid_arguments_on_device_buffers():
+    fac = P.bakron_set_factors(torch.eye(40, device="cuda"), torch.eye(8, device="cuda"))
+    W = torch.randn(8, 40, device="cuda")
+    with pytest.raises(P.BakronError) as e:
+        P.bakron_solve(W, fac, 9)
+    assert e.value.status == 1
+    with pytest.raises(P.BakronError) as e:
+        P.bakron_solve(W, fac, 4, group_size=7)
+    assert e.value.status == 1
+    with pytest.raises(P.BakronError) as e:
+        P.bakron_solve(W, fac, 4, workspace=torch.empty(64, dtype=torch.uint8, device="cuda"))
+    assert e.value.status == 5
+
+
+def test_deterministic_and_async():
+    r1 = _solve_small(90, 120, 31, bits=3)
+    W = torch.from_numpy(r1["W"]).float().cuda()
+    fac = P.bakron_set_factors(torch.from_numpy(r1["LA"]).float().cuda(),
+                               torch.from_numpy(r1["LB"]).float().cuda())
+    ws = P.alloc_workspace(90, 120)
+    a = P.bakron_solve(W, fac, 3, workspace=ws)[0].clone()
+    b = P.bakron_solve(W, fac, 3, workspace=ws, sync=False)[0]
+    assert P.bakron_read_status(ws) == 0
+    assert torch.equal(a, b)
+    np.testing.assert_array_equal(a.cpu().numpy(), r1["codes"])

@@ -301,3 +301,21 @@ def test_planted_mistakes_are_caught():
     r = O.bakron_recursive(W, -f.LA + 2 * np.eye(7), f.LB, g)
     _, bad, _ = O.certificate(W, r.codes, g, f.LA, f.LB)
     assert bad.any()
+
+
+def test_row_certificate_matches_full():
+    """The row-sampled certificate (RevCholesky form) equals the full one."""
+    W, f, g = _problem(20, 13, 90, bits=3)
+    r = O.bakron_recursive(W, f.LA, f.LB, g)
+    codes = r.codes.copy()
+    codes[7, 3] = (codes[7, 3] + 1) % (g.qmax + 1)        # make it fail somewhere
+    Xf, badf, df = O.certificate(W, codes, g, f.LA, f.LB)
+    RA, RB = O.rev_cholesky(f.A_d), O.rev_cholesky(f.B_d)
+    V = O.dequantize(codes, g, 13)
+    rows = np.array([0, 1, 7, 8, 19])
+    D = V - W
+    hi = rows.max() + 1
+    Xr, badr, dr = O.certificate_rows(W[rows], codes[rows], D[:hi], O.grid_rows(g, rows), RA,
+                                      RB[rows][:, :hi], rows)
+    np.testing.assert_allclose(Xr, Xf[rows], atol=1e-9)
+    np.testing.assert_array_equal(badr, badf[rows])
