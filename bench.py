@@ -1,0 +1,396 @@
+#!/usr/bin/env python
+"""Throughput of the BaKron solve on GB300: weight entries quantized per second.
+
+Workload (default): the 4096 x 4096 attention-projection layer -- W bf16
+~N(0, 0.02^2) with 0.1% outlier columns x10, A and B power-law Grams from 8192
+samples, 1% damping, 4-bit per-row grid -- drawn by ``workloads`` on the GPU.
+A step is one bakron_solve (grid, leaf wavefronts and all band products) on
+one resident W with the factors prepared beforehand; the device prepare is
+timed separately and reported in ``prepare_ms``.  L2 is flushed (256 MiB
+write) between timed steps, outside the timed events.
+
+Also reported: ``e2e`` (the same solve with W copied from pinned host memory
+and codes/scales/zeros copied back inside the timed region), ``roofline`` of
+the dominant kernel family (timed live with CUDA events on the launch stream
+through the library's profiling hooks), ``cpu_baseline`` (the float64 oracle
+on a bounded exact sub-problem: the top-left block, whose codes depend on
+nothing else), clocks sampled during the timed region, and ``gpu_launches``.
+
+``--impl reference`` times the oracle itself (the reference arm) on the host
+cores, each step a bounded top-left block of the same workload.
+Multi-GPU: the solve does not shard (2-D wavefront); ``--gpus N`` under
+torchrun runs N independent replicas ("replicas only", weak scaling), with a
+barrier and max-over-ranks timing and no data-path collective.
+"""
+from __future__ import annotations
+
+import argparse
+import glob
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "weight entries quantized/sec (4096x4096 BaKron solve, 1 GB300); % of roofline"
+UNIT = "entries/s"
+PAPER_4096_S = 0.288          # paper's BaKron time for 4096 x 4096 (RTX PRO 6000), context
+TILE = 32                     # leaf tile of the library (intra-tile work is the leaf's)
+L2_FLUSH_BYTES = 256 << 20
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        return None
+
+
+def _csrc_hash():
+    h = hashlib.sha256()
+    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2608_06291_gb300", "csrc", "*"))):
+        h.update(open(p, "rb").read())
+    return h.hexdigest()[:16]
+
+
+def _traffic(family):
+    """DRAM bytes per step of a kernel family from the committed ncu summary,
+    or None when the kernels changed since it was taken."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        t = json.load(open(p))
+    except Exception:
+        return None
+    if t.get("csrc_hash") != _csrc_hash():
+        return None
+    return t.get("dram_bytes_per_step", {}).get(family)
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons (read only)."""
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, bus_id=None):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+               "-lms", "100"]
+        if bus_id:
+            cmd += ["-i", bus_id]
+        try:
+            self.p = subprocess.Popen(cmd, stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self, t0, t1):
+        if self.p is None:
+            return None
+        time.sleep(0.25)
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except Exception:
+            self.p.kill()
+        self.f.flush()
+        rows = [r.split(",") for r in open(self.f.name).read().strip().splitlines() if r.strip()]
+        os.unlink(self.f.name)
+        samples = []
+        for r in rows:
+            try:
+                ts = time.mktime(time.strptime(r[0].strip().split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                samples.append((ts, float(r[1]), float(r[2]), [x.strip() for x in r[5:9]]))
+            except Exception:
+                continue
+        inside = [s for s in samples if t0 - 1.0 <= s[0] <= t1 + 1.0] or samples
+        if not inside:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for s in inside for i, v in enumerate(s[3]) if v == "Active"})
+        return {"sm_mhz": statistics.median(s[1] for s in inside),
+                "sm_max_mhz": max(s[2] for s in inside), "reasons": reasons,
+                "samples": len(inside)}
+
+
+# ----------------------------------------------------------------- oracle legs
+def _oracle_block(W64, f, bits, group, k):
+    """Time the float64 oracle (Alg. 4) on the top-left k x k block of the
+    workload: entry (i, j) depends only on entries up-left of it, so with the
+    full problem's factors restricted to the block this is an exact part of
+    the full solve."""
+    import oracle as O
+    Wb = W64[:k, :k]
+    g = O.quant_grid(Wb, bits, group if group and k % group == 0 else 0)
+    c0 = os.times()
+    t0 = time.perf_counter()
+    O.bakron_recursive(Wb, f.LA[:k, :k], f.LB[:k, :k], g)
+    wall = time.perf_counter() - t0
+    c1 = os.times()
+    cpu = (c1.user - c0.user) + (c1.system - c0.system)
+    return wall, max(1, round(cpu / wall)) if wall > 0 else 1
+
+
+def _oracle_factors(A, B, damp):
+    import oracle as O
+    return O.prepare(A.double().cpu().numpy(), B.double().cpu().numpy(), damp, via_inverse=False)
+
+
+def run_reference(args):
+    """The reference arm: the oracle, as it stands, on the host cores."""
+    import torch
+    import workloads as WL
+    ws, rank, local = _dist()
+    if rank != 0:
+        return 0
+    cfg = WL.CONFIGS[args.config]
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    W, A, B = WL.make(cfg, device=dev)
+    f = _oracle_factors(A, B, cfg.damp)
+    W64 = W.double().cpu().numpy()
+    k = args.ref_block
+    for _ in range(args.warmup):
+        _oracle_block(W64, f, cfg.bits, cfg.group, k)
+    times, cores = [], 1
+    for _ in range(args.steps):
+        t, c = _oracle_block(W64, f, cfg.bits, cfg.group, k)
+        times.append(t)
+        cores = max(cores, c)
+    ms = 1e3 * sum(times) / len(times)
+    value = k * k / (ms / 1e3)
+    sample = (f"top-left {k}x{k} block of the {cfg.m}x{cfg.n} workload per step (exact "
+              f"sub-problem, full-problem factors), float64 Alg. 4 oracle")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": _config_dict(cfg),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+    return 0
+
+
+def _config_dict(cfg):
+    return {"workload": f"config {cfg.index}: {cfg.name}, W {str(cfg.w_dtype).split('.')[-1]} "
+                        f"{cfg.w_dist}, {cfg.bits}-bit "
+                        + ("per-row" if cfg.group == 0 else f"g{cfg.group}") + " grid, "
+                        f"power-law Grams from {cfg.n_samples} samples, damp {cfg.damp}",
+            "m": cfg.m, "n": cfg.n, "bits": cfg.bits, "group": cfg.group,
+            "l2": "flushed between timed steps (256 MiB write)", "factors": "precomputed"}
+
+
+# --------------------------------------------------------------------- main arm
+def run_gpu(args):
+    import numpy as np
+    import torch
+
+    import paper_2608_06291_gb300 as P
+    import workloads as WL
+
+    ws_n, rank, local = _dist()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws_n > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    P.build()
+    P.lib()
+    cfg = WL.CONFIGS[args.config]
+    m, n = cfg.m, cfg.n
+    W, A, B = WL.make(cfg, device=dev)
+    work = P.alloc_workspace(m, n, dev)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    fac = P.bakron_prepare(A, B, cfg.damp, workspace=work)
+    torch.cuda.synchronize()
+    prepare_ms = 1e3 * (time.perf_counter() - t0)
+    G = 1 if cfg.group == 0 else n // cfg.group
+    codes = torch.empty(m, n, dtype=torch.uint8, device=dev)
+    scales = torch.empty(m, G, dtype=torch.float32, device=dev)
+    zeros = torch.empty(m, G, dtype=torch.float32, device=dev)
+    out = (codes, scales, zeros, None)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        P.bakron_solve(W, fac, cfg.bits, cfg.group, workspace=work, sync=False, out=out)
+
+    for _ in range(max(3, args.warmup)):
+        flush.fill_(1)
+        step()
+    torch.cuda.synchronize()
+    if P.bakron_read_status(work) != 0:
+        raise RuntimeError("device status set during warm-up")
+
+    bus = None
+    try:
+        bus = torch.cuda.get_device_properties(dev).pci_bus_id
+    except Exception:
+        pass
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(bus) if rank == 0 else None
+    time.sleep(0.3)
+    if ws_n > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    w0 = time.time()
+    launches = 0
+    for i in range(args.steps):
+        flush.fill_(i & 0xFF)
+        starts[i].record(stream)
+        step()
+        ends[i].record(stream)
+        launches += P.bakron_last_launches()
+    torch.cuda.synchronize()
+    if ws_n > 1:
+        torch.distributed.barrier()
+    w1 = time.time()
+    clocks = sampler.stop(w0, w1) if sampler else None
+    ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / args.steps
+    if ws_n > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    if P.bakron_read_status(work) != 0:
+        raise RuntimeError("device status set during the timed steps")
+    value = ws_n * m * n / (ms / 1e3)
+
+    # per-family device time, live, with events on the launch stream
+    P.bakron_profile_enable(True)
+    prof_steps = max(3, min(args.steps, 10))
+    for i in range(prof_steps):
+        flush.fill_(i & 0xFF)
+        step()
+    fam = P.bakron_profile_read()
+    P.bakron_profile_enable(False)
+    fam_ms = {k: v[1] / prof_steps for k, v in fam.items()}
+    fam_n = {k: v[0] // prof_steps for k, v in fam.items()}
+
+    peaks = _peaks() or {}
+    f_alg = float(m) * n * (m + n)                    # flops of L^B E L^A^T (structural nonzeros)
+    f_band = f_alg - 2.0 * TILE * m * n               # minus the intra-tile part (leaf)
+    band_ms = fam_ms["band1"] + fam_ms["band2"]
+    leaf_ms = fam_ms["leaf"]
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    fp32_simt_peak = 152 * 128 * 2 * sm_max * 1e6 / 1e12     # TFLOP/s, FFMA on CUDA cores
+    if band_ms >= leaf_ms:
+        achieved = f_band / (band_ms / 1e3) / 1e12
+        roof = {"kernel": "band products (stage 1 M = L^B E, stage 2 X += M L^A^T), SIMT FP32",
+                "bound": "alu", "achieved": achieved, "peak": fp32_simt_peak, "unit": "TFLOP/s",
+                "frac": achieved / fp32_simt_peak,
+                "peak_source": "152 SMs x 128 FP32 lanes x 2 flop x sm_max_mhz (derived)",
+                "algorithmic_per_step": f_band, "launches_per_step": fam_n["band1"] + fam_n["band2"],
+                "traffic": _traffic("band")}
+    else:
+        bytes_leaf = 17.0 * m * n                     # read X, write X and E, write code, factor blocks
+        hbm = float(peaks.get("hbm_gbs", 6800.0))
+        achieved = bytes_leaf / (leaf_ms / 1e3) / 1e9
+        roof = {"kernel": "leaf wavefront", "bound": "hbm", "achieved": achieved, "peak": hbm,
+                "unit": "GB/s", "frac": achieved / hbm, "peak_source": "MEASURED_PEAKS.json hbm_gbs",
+                "algorithmic_per_step": bytes_leaf, "launches_per_step": fam_n["leaf"],
+                "traffic": _traffic("leaf")}
+    roof["family_ms_per_step"] = fam_ms
+    roof["family_launches_per_step"] = fam_n
+    # whole-solve roofline: GEMM work at the FP32-effective
+    # tensor peak (3xTF32: the TF32 rate, derived from the measured bf16 rate by
+    # the nominal 1.1/2.25 ratio, divided by 3) plus the leaves' bytes at HBM rate
+    bf16_sus = float(peaks.get("bf16_tflops_sustained", 1700.0))
+    p_eff = bf16_sus * (1.1 / 2.25) / 3.0
+    t_roof = f_alg / (p_eff * 1e12) + 17.0 * m * n / (float(peaks.get("hbm_gbs", 6800.0)) * 1e9)
+    solve_roof = {"fp32_effective_tflops": p_eff, "f_alg_flops": f_alg,
+                  "roofline_ms": 1e3 * t_roof, "frac": 1e3 * t_roof / ms,
+                  "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained x 1.1/2.25 / 3"}
+
+    # end to end: pinned host W in, codes/scales/zeros out, inside the timed region
+    Wh = W.cpu().pin_memory()
+    ch = torch.empty(m, n, dtype=torch.uint8).pin_memory()
+    sh = torch.empty(m, G, dtype=torch.float32).pin_memory()
+    zh = torch.empty(m, G, dtype=torch.float32).pin_memory()
+    Wd = torch.empty_like(W)
+    e2e_steps = max(3, min(args.steps, 10))
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    tot = 0.0
+    for i in range(e2e_steps):
+        flush.fill_(i & 0xFF)
+        e0.record(stream)
+        Wd.copy_(Wh, non_blocking=True)
+        P.bakron_solve(Wd, fac, cfg.bits, cfg.group, workspace=work, sync=False, out=out)
+        ch.copy_(codes, non_blocking=True)
+        sh.copy_(scales, non_blocking=True)
+        zh.copy_(zeros, non_blocking=True)
+        e1.record(stream)
+        e1.synchronize()
+        tot += e0.elapsed_time(e1)
+    e2e_ms = tot / e2e_steps
+    if ws_n > 1:
+        t = torch.tensor([e2e_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e = {"value": ws_n * m * n / (e2e_ms / 1e3), "unit": UNIT,
+           "h2d_bytes_per_step": Wh.numel() * Wh.element_size(),
+           "d2h_bytes_per_step": ch.numel() + 4 * (sh.numel() + zh.numel()),
+           "ms_per_step": e2e_ms}
+
+    cpu_base = None
+    if rank == 0 and not args.no_cpu_baseline:
+        f = _oracle_factors(A, B, cfg.damp)
+        W64 = W.double().cpu().numpy()
+        k = args.cpu_block
+        wall, cores = _oracle_block(W64, f, cfg.bits, cfg.group, k)
+        cpu_base = {"value": k * k / wall, "unit": UNIT, "cores": cores, "kind": "oracle",
+                    "sample": f"top-left {k}x{k} block of the {m}x{n} workload (exact "
+                              f"sub-problem with the full problem's factors), float64 Alg. 4 "
+                              f"oracle, {wall:.1f} s wall"}
+
+    if rank == 0:
+        vs = value / (4096 * 4096 / PAPER_4096_S) if (m, n) == (4096, 4096) else None
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws_n, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": vs, "dtype": "f32", "data": "synthetic",
+            "config": dict(_config_dict(cfg), parallelism=f"replicas x{ws_n}"),
+            "prepare_ms": prepare_ms, "roofline": roof, "cpu_baseline": cpu_base, "e2e": e2e,
+            "gpu_launches": launches, "clocks": clocks, "solve_roofline": solve_roof,
+        }
+        print(json.dumps(line))
+    if ws_n > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--cpu-block", type=int, default=1024,
+                    help="side of the top-left block the cpu_baseline oracle solves")
+    ap.add_argument("--ref-block", type=int, default=256,
+                    help="side of the top-left block each reference-arm step solves")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -131,6 +131,22 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw,
  * `workspace` by the last prepare/solve that used it. */
 int bakron_read_status(void* workspace, void* stream);
 
+/*
+ * Instrumentation for benchmarks (no counterpart in the paper).
+ * bakron_profile_enable(1) makes every later bakron_solve bracket each of its
+ * kernel launches with CUDA events on `stream` and accumulate, per kernel
+ * family, the number of launches and their device time.  Families:
+ *   0 grid + workspace init, 1 leaf wavefront, 2 band product stage 1
+ *   (M = L^B E), 3 band product stage 2 (X += M L^A^T), 4 output copy.
+ * bakron_profile_read synchronises the device, then returns the totals since
+ * the last enable/reset of `family` (launches, milliseconds).
+ * bakron_last_launches returns the number of kernels the last bakron_solve
+ * call on this host thread enqueued.
+ */
+int bakron_profile_enable(int on);
+int bakron_profile_read(int family, int* launches, double* ms);
+int bakron_last_launches(void);
+
 /* Static description of a status code. */
 const char* bakron_strerror(int status);
 

@@ -5,6 +5,7 @@ C ABI in include/bakron.h); this package is its build script and a thin
 ctypes binding with the same entry-point names.
 """
 from .bakron import (BakronError, Factors, alloc_workspace, bakron_get_factors,  # noqa: F401
-                     bakron_prepare, bakron_read_status, bakron_set_factors, bakron_solve,
+                     bakron_last_launches, bakron_prepare, bakron_profile_enable,
+                     bakron_profile_read, bakron_read_status, bakron_set_factors, bakron_solve,
                      dequantize, factors_bytes, lib, library_path, strerror, workspace_bytes)
 from .buildlib import build  # noqa: F401

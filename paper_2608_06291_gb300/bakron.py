@@ -54,6 +54,12 @@ def lib() -> ctypes.CDLL:
     L.bakron_solve.restype = i32
     L.bakron_read_status.argtypes = [vp, vp]
     L.bakron_read_status.restype = i32
+    L.bakron_profile_enable.argtypes = [i32]
+    L.bakron_profile_enable.restype = i32
+    L.bakron_profile_read.argtypes = [i32, ctypes.POINTER(i32), ctypes.POINTER(ctypes.c_double)]
+    L.bakron_profile_read.restype = i32
+    L.bakron_last_launches.argtypes = []
+    L.bakron_last_launches.restype = i32
     L.bakron_strerror.argtypes = [i32]
     L.bakron_strerror.restype = ctypes.c_char_p
     _lib = L
@@ -175,6 +181,28 @@ def bakron_solve(W, f: Factors, bits: int, group_size: int = 0, workspace=None,
 
 def bakron_read_status(workspace, stream=None) -> int:
     return int(lib().bakron_read_status(_ptr(workspace), _stream(stream)))
+
+
+PROFILE_FAMILIES = ("init", "leaf", "band1", "band2", "copy")
+
+
+def bakron_profile_enable(on: bool = True) -> None:
+    _check(lib().bakron_profile_enable(1 if on else 0), "bakron_profile_enable")
+
+
+def bakron_profile_read() -> dict:
+    """{family: (launches, milliseconds)} accumulated since the last enable."""
+    out = {}
+    for i, name in enumerate(PROFILE_FAMILIES):
+        n = ctypes.c_int(0)
+        ms = ctypes.c_double(0.0)
+        _check(lib().bakron_profile_read(i, ctypes.byref(n), ctypes.byref(ms)), "bakron_profile_read")
+        out[name] = (n.value, ms.value)
+    return out
+
+
+def bakron_last_launches() -> int:
+    return int(lib().bakron_last_launches())
 
 
 def dequantize(codes, scales, zeros):

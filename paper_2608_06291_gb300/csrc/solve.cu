@@ -18,6 +18,7 @@
 #include <math.h>
 
 #include "common.cuh"
+#include "profile.cuh"
 
 namespace bakron {
 
@@ -268,6 +269,7 @@ struct SolveArgs {
 
 static void leaf(const SolveArgs& a, int K) {
   const int ilo = max(0, K - (a.Nt - 1)), ihi = min(K, a.Mt - 1);
+  LaunchScope ls(kFamLeaf, a.s);
   k_leaf<<<ihi - ilo + 1, 32, 0, a.s>>>(K, a.Mt, a.Nt, a.m, a.n, a.X, a.E, a.np, a.LB, a.mp,
                                         a.LA, a.np, a.scales, a.zeros, a.G, a.gsz, a.qmax,
                                         a.codes, a.status);
@@ -276,8 +278,14 @@ static void leaf(const SolveArgs& a, int K) {
 static void band(const SolveArgs& a, int k, int h, int l) {
   Band bd{k, h, l, a.Mt, a.Nt};
   dim3 g1(h, a.Mt), g2(l - h, a.Mt);
-  k_band1_simt<<<g1, 256, 0, a.s>>>(bd, a.LB, a.mp, a.E, a.M, a.np);
-  k_band2_simt<<<g2, 256, 0, a.s>>>(bd, a.LA, a.np, a.M, a.X, a.np);
+  {
+    LaunchScope ls(kFamBand1, a.s);
+    k_band1_simt<<<g1, 256, 0, a.s>>>(bd, a.LB, a.mp, a.E, a.M, a.np);
+  }
+  {
+    LaunchScope ls(kFamBand2, a.s);
+    k_band2_simt<<<g2, 256, 0, a.s>>>(bd, a.LA, a.np, a.M, a.X, a.np);
+  }
 }
 
 static void rec(const SolveArgs& a, int k, int l) {
@@ -313,17 +321,23 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
   a.scales = scales; a.zeros = zeros; a.codes = codes;
   a.status = (int*)(ws + sl.off_status);
   a.s = s;
+  reset_launch_count();
   BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_status, 0, 256, s));
   {
     const int64_t warps = (int64_t)m * a.G;
+    LaunchScope ls(kFamInit, s);
     k_grid<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(W, wdt, m, n, ldw, a.gsz, a.G,
                                                                  a.qmax, scales, zeros);
+  }
+  {
     const int64_t tot = a.mp * a.np;
+    LaunchScope ls(kFamInit, s);
     k_init<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(W, wdt, m, n, ldw, a.X, a.mp, a.np);
   }
   rec(a, 0, a.Mt + a.Nt - 1);
   if (prerounding) {
     const int64_t tot = (int64_t)m * n;
+    LaunchScope ls(kFamCopy, s);
     k_copy_out<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(a.X, a.np, m, n, prerounding);
   }
   BK_CUDA_OK(cudaGetLastError());
