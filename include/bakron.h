@@ -127,6 +127,37 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw,
                  float* prerounding, void* workspace, size_t workspace_bytes,
                  int sync, void* stream);
 
+/*
+ * bakron_solve_noalloc -- bakron_solve without a caller workspace, for
+ * callers that cannot allocate device memory of their own: for example a
+ * plugin that a host framework hands only its input and output buffers
+ * (the framework owns every allocation), or a process under a fixed device
+ * memory budget that forbids allocating after start-up.  This entry point has
+ * no counterpart in the paper; it is the same solve as bakron_solve.
+ *
+ * Scratch: a fixed array of BAKRON_NOALLOC_SCRATCH_BYTES (64 MiB) inside the
+ * library, on every GPU that loads it, held until the process exits.  A
+ * problem fits when 256 + 12 * mp * np <= 64 MiB, mp and np being m and n
+ * rounded up to multiples of 128 (e.g. 2048 x 2048, 1024 x 4096); larger
+ * problems are rejected with BAKRON_ERR_WORKSPACE before anything is
+ * enqueued.  The call allocates nothing: no cudaMalloc/cudaFree, no
+ * allocating library routine.
+ *
+ * The first call on a device (the device current at the call) looks up the
+ * array's device address once (cudaGetSymbolAddress) and caches it; make
+ * that first call before any stream capture on that device.
+ * Every call on a device shares the one array and leaves its contents behind;
+ * each call clears what must start at zero (the status word) and overwrites
+ * the rest before reading it.  Calls whose work overlaps on the GPU (another
+ * stream, another host thread, same device) race on the array: serialise
+ * them.  Arguments, outputs and `sync` are those of bakron_solve.
+ */
+#define BAKRON_NOALLOC_SCRATCH_BYTES ((size_t)64 << 20)
+int bakron_solve_noalloc(const void* W, int wdtype, int m, int n, int64_t ldw,
+                         const void* factors, int bits, int group_size,
+                         uint8_t* codes, float* scales, float* zeros,
+                         float* prerounding, int sync, void* stream);
+
 /* Synchronise `stream`, return and clear the device status word kept in
  * `workspace` by the last prepare/solve that used it. */
 int bakron_read_status(void* workspace, void* stream);

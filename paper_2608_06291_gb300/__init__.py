@@ -7,5 +7,6 @@ ctypes binding with the same entry-point names.
 from .bakron import (BakronError, Factors, alloc_workspace, bakron_get_factors,  # noqa: F401
                      bakron_last_launches, bakron_prepare, bakron_profile_enable,
                      bakron_profile_read, bakron_read_status, bakron_set_factors, bakron_solve,
+                     bakron_solve_noalloc,
                      dequantize, factors_bytes, lib, library_path, strerror, workspace_bytes)
 from .buildlib import build  # noqa: F401

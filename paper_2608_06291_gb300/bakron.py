@@ -52,6 +52,8 @@ def lib() -> ctypes.CDLL:
     L.bakron_get_factors.restype = i32
     L.bakron_solve.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, vp, sz, i32, vp]
     L.bakron_solve.restype = i32
+    L.bakron_solve_noalloc.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, i32, vp]
+    L.bakron_solve_noalloc.restype = i32
     L.bakron_read_status.argtypes = [vp, vp]
     L.bakron_read_status.restype = i32
     L.bakron_profile_enable.argtypes = [i32]
@@ -176,6 +178,36 @@ def bakron_solve(W, f: Factors, bits: int, group_size: int = 0, workspace=None,
                             int(group_size), _ptr(codes), _ptr(scales), _ptr(zeros), _ptr(xpre),
                             _ptr(ws), ws.numel(), 1 if sync else 0, _stream(stream))
     _check(rc, "bakron_solve")
+    return (codes, scales, zeros, xpre) if prerounding else (codes, scales, zeros)
+
+
+def bakron_solve_noalloc(W, f: Factors, bits: int, group_size: int = 0,
+                         prerounding: bool = False, sync: bool = True, out=None, stream=None):
+    """bakron_solve without a workspace argument, for callers that cannot
+    allocate device scratch: the library's fixed 64 MiB array is used instead
+    (problems up to 12 * mp * np + 256 bytes of scratch).  Outputs are
+    allocated here unless ``out`` is given."""
+    if not W.is_cuda or W.dim() != 2 or W.stride(1) != 1:
+        raise ValueError("W must be a 2-D CUDA tensor with unit column stride")
+    dt = {torch.float32: F32, torch.bfloat16: BF16}.get(W.dtype)
+    if dt is None:
+        raise ValueError("W must be float32 or bfloat16")
+    m, n = W.shape
+    if (f.m, f.n) != (m, n):
+        raise ValueError("factor buffer was built for a different shape")
+    G = 1 if group_size == 0 else n // group_size
+    dev = W.device
+    if out is None:
+        codes = torch.empty(m, n, dtype=torch.uint8, device=dev)
+        scales = torch.empty(m, G, dtype=torch.float32, device=dev)
+        zeros = torch.empty(m, G, dtype=torch.float32, device=dev)
+        xpre = torch.empty(m, n, dtype=torch.float32, device=dev) if prerounding else None
+    else:
+        codes, scales, zeros, xpre = out
+    rc = lib().bakron_solve_noalloc(_ptr(W), dt, m, n, W.stride(0), _ptr(f.buf), int(bits),
+                                    int(group_size), _ptr(codes), _ptr(scales), _ptr(zeros),
+                                    _ptr(xpre), 1 if sync else 0, _stream(stream))
+    _check(rc, "bakron_solve_noalloc")
     return (codes, scales, zeros, xpre) if prerounding else (codes, scales, zeros)
 
 
