@@ -137,10 +137,10 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw,
  *
  * Scratch: a fixed array of BAKRON_NOALLOC_SCRATCH_BYTES (64 MiB) inside the
  * library, on every GPU that loads it, held until the process exits.  A
- * problem fits when 256 + 12 * mp * np <= 64 MiB, mp and np being m and n
- * rounded up to multiples of 128 (e.g. 2048 x 2048, 1024 x 4096); larger
- * problems are rejected with BAKRON_ERR_WORKSPACE before anything is
- * enqueued.  The call allocates nothing: no cudaMalloc/cudaFree, no
+ * problem fits when the solve's scratch, 256 + 20 * mp * np bytes (mp, np: m
+ * and n rounded up to multiples of 128), is at most 64 MiB -- e.g. 1792 x
+ * 1792 or 2048 x 1536; larger problems are rejected with BAKRON_ERR_WORKSPACE
+ * before anything is enqueued.  The call allocates nothing: no cudaMalloc/cudaFree, no
  * allocating library routine.
  *
  * The first call on a device (the device current at the call) looks up the
@@ -177,6 +177,17 @@ int bakron_read_status(void* workspace, void* stream);
 int bakron_profile_enable(int on);
 int bakron_profile_read(int family, int* launches, double* ms);
 int bakron_last_launches(void);
+
+/*
+ * Diagnostic (no counterpart in the paper): C = A B^T on the tensor cores
+ * with the 3xTF32 split the band products use.  A is M x K, B is N x K, C is
+ * M x N, all device fp32 row-major; M and N multiples of 128, K of 32.
+ * workspace >= 256 + 8 (M + N) K bytes.  Synchronises `stream` and returns
+ * the device status (BAKRON_ERR_TIMEOUT if a bounded wait ran out).
+ */
+int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C, int M,
+                            int N, int K, void* workspace,
+                            size_t workspace_bytes, void* stream);
 
 /* Static description of a status code. */
 const char* bakron_strerror(int status);

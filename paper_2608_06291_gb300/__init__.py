@@ -4,7 +4,8 @@ The compute path is libbakron.so (hand-written sm_103a CUDA kernels behind the
 C ABI in include/bakron.h); this package is its build script and a thin
 ctypes binding with the same entry-point names.
 """
-from .bakron import (BakronError, Factors, alloc_workspace, bakron_get_factors,  # noqa: F401
+from .bakron import (BakronError, Factors, alloc_workspace, bakron_diag_gemm_tf32x3,  # noqa: F401
+                     bakron_get_factors,
                      bakron_last_launches, bakron_prepare, bakron_profile_enable,
                      bakron_profile_read, bakron_read_status, bakron_set_factors, bakron_solve,
                      bakron_solve_noalloc,

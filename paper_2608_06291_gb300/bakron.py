@@ -62,6 +62,8 @@ def lib() -> ctypes.CDLL:
     L.bakron_profile_read.restype = i32
     L.bakron_last_launches.argtypes = []
     L.bakron_last_launches.restype = i32
+    L.bakron_diag_gemm_tf32x3.argtypes = [vp, vp, vp, i32, i32, i32, vp, sz, vp]
+    L.bakron_diag_gemm_tf32x3.restype = i32
     L.bakron_strerror.argtypes = [i32]
     L.bakron_strerror.restype = ctypes.c_char_p
     _lib = L
@@ -185,7 +187,7 @@ def bakron_solve_noalloc(W, f: Factors, bits: int, group_size: int = 0,
                          prerounding: bool = False, sync: bool = True, out=None, stream=None):
     """bakron_solve without a workspace argument, for callers that cannot
     allocate device scratch: the library's fixed 64 MiB array is used instead
-    (problems up to 12 * mp * np + 256 bytes of scratch).  Outputs are
+    (problems whose scratch, 20 * mp * np + 256 bytes, fits).  Outputs are
     allocated here unless ``out`` is given."""
     if not W.is_cuda or W.dim() != 2 or W.stride(1) != 1:
         raise ValueError("W must be a 2-D CUDA tensor with unit column stride")
@@ -235,6 +237,20 @@ def bakron_profile_read() -> dict:
 
 def bakron_last_launches() -> int:
     return int(lib().bakron_last_launches())
+
+
+def bakron_diag_gemm_tf32x3(A, B, stream=None):
+    """C = A B^T on the tensor cores with the solve's 3xTF32 split (diagnostic)."""
+    A = A.contiguous()
+    B = B.contiguous()
+    M, K = A.shape
+    N = B.shape[0]
+    C = torch.empty(M, N, dtype=torch.float32, device=A.device)
+    ws = torch.empty(256 + 8 * (M + N) * K, dtype=torch.uint8, device=A.device)
+    rc = lib().bakron_diag_gemm_tf32x3(_ptr(A), _ptr(B), _ptr(C), M, N, K, _ptr(ws), ws.numel(),
+                                       _stream(stream))
+    _check(rc, "bakron_diag_gemm_tf32x3")
+    return C
 
 
 def dequantize(codes, scales, zeros):

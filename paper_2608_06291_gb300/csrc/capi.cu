@@ -22,13 +22,15 @@ static bool dims_ok(int m, int n) { return m >= 1 && n >= 1 && m <= MAX_DIM && n
 // Dense unit-lower L (d x d, row-major, only the strictly-lower part read)
 // into the padded factor section (Lp x Lp) with ones on the diagonal, zeros
 // above it and an identity extension.
-__global__ void k_import(const float* L, int d, float* dst, int64_t Lp) {
+__global__ void k_import(const float* L, int d, float* hi, float* lo, int64_t Lp) {
   const int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (idx >= Lp * Lp) return;
   const int64_t i = idx / Lp, j = idx % Lp;
   float v = (i == j) ? 1.f : 0.f;
   if (i < d && j < d && j < i) v = L[i * d + j];
-  dst[idx] = v;
+  const float h = tf32_hi(v);
+  hi[idx] = h;
+  lo[idx] = v - h;
 }
 
 __global__ void k_import_diag(const float* r, int d, float* dst, int64_t Lp) {
@@ -36,10 +38,11 @@ __global__ void k_import_diag(const float* r, int d, float* dst, int64_t Lp) {
   if (i < Lp) dst[i] = (r && i < d) ? r[i] : 1.f;
 }
 
-__global__ void k_export(const float* src, int64_t Lp, int d, float* L) {
+__global__ void k_export(const float* hi, const float* lo, int64_t Lp, int d, float* L) {
   const int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (idx >= (int64_t)d * d) return;
-  L[idx] = src[(idx / d) * Lp + idx % d];
+  const int64_t k = (idx / d) * Lp + idx % d;
+  L[idx] = hi[k] + lo[k];
 }
 
 static unsigned nblocks(int64_t work, int threads) { return (unsigned)((work + threads - 1) / threads); }
@@ -78,8 +81,10 @@ int bakron_set_factors(const float* LA, const float* LB, const float* rA, const 
   FactorLayout fl(m, n);
   cudaStream_t s = (cudaStream_t)stream;
   char* f = (char*)factors;
-  k_import<<<nblocks(fl.np * fl.np, 256), 256, 0, s>>>(LA, n, (float*)(f + fl.off_LA), fl.np);
-  k_import<<<nblocks(fl.mp * fl.mp, 256), 256, 0, s>>>(LB, m, (float*)(f + fl.off_LB), fl.mp);
+  k_import<<<nblocks(fl.np * fl.np, 256), 256, 0, s>>>(LA, n, (float*)(f + fl.off_LAH),
+                                                       (float*)(f + fl.off_LAL), fl.np);
+  k_import<<<nblocks(fl.mp * fl.mp, 256), 256, 0, s>>>(LB, m, (float*)(f + fl.off_LBH),
+                                                       (float*)(f + fl.off_LBL), fl.mp);
   k_import_diag<<<nblocks(fl.np, 256), 256, 0, s>>>(rA, n, (float*)(f + fl.off_rA), fl.np);
   k_import_diag<<<nblocks(fl.mp, 256), 256, 0, s>>>(rB, m, (float*)(f + fl.off_rB), fl.mp);
   BK_CUDA_OK(cudaGetLastError());
@@ -92,8 +97,12 @@ int bakron_get_factors(const void* factors, int m, int n, float* LA, float* LB, 
   FactorLayout fl(m, n);
   cudaStream_t s = (cudaStream_t)stream;
   const char* f = (const char*)factors;
-  if (LA) k_export<<<nblocks((int64_t)n * n, 256), 256, 0, s>>>((const float*)(f + fl.off_LA), fl.np, n, LA);
-  if (LB) k_export<<<nblocks((int64_t)m * m, 256), 256, 0, s>>>((const float*)(f + fl.off_LB), fl.mp, m, LB);
+  if (LA)
+    k_export<<<nblocks((int64_t)n * n, 256), 256, 0, s>>>(
+        (const float*)(f + fl.off_LAH), (const float*)(f + fl.off_LAL), fl.np, n, LA);
+  if (LB)
+    k_export<<<nblocks((int64_t)m * m, 256), 256, 0, s>>>(
+        (const float*)(f + fl.off_LBH), (const float*)(f + fl.off_LBL), fl.mp, m, LB);
   if (rA) BK_CUDA_OK(cudaMemcpyAsync(rA, f + fl.off_rA, sizeof(float) * n, cudaMemcpyDeviceToDevice, s));
   if (rB) BK_CUDA_OK(cudaMemcpyAsync(rB, f + fl.off_rB, sizeof(float) * m, cudaMemcpyDeviceToDevice, s));
   BK_CUDA_OK(cudaGetLastError());

@@ -24,37 +24,60 @@ __host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; 
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// Factor buffer: [L^B  mp x mp][L^A  np x np][rB  mp][rA  np], fp32, each
-// section 256-byte aligned.  L^X is stored dense row-major with exact zeros
-// above the diagonal, ones on it, and an identity extension over the padding.
+// Split of an fp32 value into an exact tf32 head and an fp32 tail:
+// hi = x with its 13 low mantissa bits cleared (exactly representable in
+// tf32), lo = x - hi (exact in fp32, |lo| < 2^-10 |x|).  hi + lo == x exactly.
+__host__ __device__ inline float tf32_hi(float x) {
+#ifdef __CUDA_ARCH__
+  return __uint_as_float(__float_as_uint(x) & 0xFFFFE000u);
+#else
+  union { float f; uint32_t u; } v;
+  v.f = x;
+  v.u &= 0xFFFFE000u;
+  return v.f;
+#endif
+}
+
+// Factor buffer: [L^B hi][L^B lo] (mp x mp each) [L^A hi][L^A lo] (np x np)
+// [rB mp][rA np], fp32, sections 256-byte aligned.  L^X = hi + lo exactly;
+// stored dense row-major with exact zeros above the diagonal, ones on it and
+// an identity extension over the padding.
 struct FactorLayout {
   int m, n;
   int64_t mp, np;
-  size_t off_LB, off_LA, off_rB, off_rA, bytes;
+  size_t off_LBH, off_LBL, off_LAH, off_LAL, off_rB, off_rA, bytes;
   explicit FactorLayout(int m_, int n_) : m(m_), n(n_) {
     mp = round_up(m, PAD);
     np = round_up(n, PAD);
-    off_LB = 0;
-    off_LA = align256(off_LB + size_t(mp * mp) * 4);
-    off_rB = align256(off_LA + size_t(np * np) * 4);
+    off_LBH = 0;
+    off_LBL = align256(off_LBH + size_t(mp * mp) * 4);
+    off_LAH = align256(off_LBL + size_t(mp * mp) * 4);
+    off_LAL = align256(off_LAH + size_t(np * np) * 4);
+    off_rB = align256(off_LAL + size_t(np * np) * 4);
     off_rA = align256(off_rB + size_t(mp) * 4);
     bytes = align256(off_rA + size_t(np) * 4);
   }
 };
 
-// Workspace: [status 256 B][solve: X, E, M  (mp x np fp32 each)] or
-//            [status 256 B][prepare: C, Linv (dp x dp fp64/fp32), scratch].
+// Solve workspace: [status 256 B][X mp x np][E^T hi, lo: np x mp each]
+// [M hi, lo: mp x np each], fp32.  X holds W widened and, once an entry is
+// rounded, the value it was rounded at.  E^T is the error matrix transposed
+// (row = column index of W) so that it is K-major as the second operand of
+// M = L^B E; M is the stage-1 band product.
 struct SolveLayout {
   int64_t mp, np;
-  size_t off_status, off_X, off_E, off_M, bytes;
+  size_t off_status, off_X, off_EtH, off_EtL, off_MH, off_ML, bytes;
   SolveLayout(int m, int n) {
     mp = round_up(m, PAD);
     np = round_up(n, PAD);
+    const size_t plane = size_t(mp * np) * 4;
     off_status = 0;
     off_X = 256;
-    off_E = align256(off_X + size_t(mp * np) * 4);
-    off_M = align256(off_E + size_t(mp * np) * 4);
-    bytes = align256(off_M + size_t(mp * np) * 4);
+    off_EtH = align256(off_X + plane);
+    off_EtL = align256(off_EtH + plane);
+    off_MH = align256(off_EtL + plane);
+    off_ML = align256(off_MH + plane);
+    bytes = align256(off_ML + plane);
   }
 };
 

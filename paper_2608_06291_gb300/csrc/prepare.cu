@@ -190,7 +190,7 @@ __global__ void k_put_diag(const RT* Dinv, int b, RT* X, int64_t ldx, int i0) {
 // diagonal, 0 above, identity on the padding; rdiag[i] = C[d-1-i][d-1-i].
 template <typename RT>
 __global__ void k_assemble(const RT* C, const RT* Xinv, int64_t dp, int d, float* L,
-                           int64_t ldl, int64_t Lp, float* rdiag) {
+                           float* Llo, int64_t ldl, int64_t Lp, float* rdiag) {
   __shared__ float tile[32][33];
   const int bx = blockIdx.x * 32, by = blockIdx.y * 32;
   // read transposed source block: source row a = d-1-j, col b = d-1-i
@@ -211,7 +211,9 @@ __global__ void k_assemble(const RT* C, const RT* Xinv, int64_t dp, int d, float
       float v = tile[threadIdx.x][yy];
       if (i == j) v = 1.f;
       else if (i >= d || j >= d) v = 0.f;
-      L[(int64_t)i * ldl + j] = v;
+      const float hi = tf32_hi(v);
+      L[(int64_t)i * ldl + j] = hi;
+      Llo[(int64_t)i * ldl + j] = v - hi;
     }
   }
   if (blockIdx.x == 0 && threadIdx.y == 0) {
@@ -222,8 +224,8 @@ __global__ void k_assemble(const RT* C, const RT* Xinv, int64_t dp, int d, float
 
 // One Gram -> one unit-lower factor (fp32, Lp x Lp) and its RevCholesky diagonal.
 template <typename RT>
-static int factor_one(const float* H, int d, float damp, float* L, int64_t Lp, float* rdiag,
-                      void* workspace, const PrepareLayout& lay, cudaStream_t s) {
+static int factor_one(const float* H, int d, float damp, float* L, float* Llo, int64_t Lp,
+                      float* rdiag, void* workspace, const PrepareLayout& lay, cudaStream_t s) {
   char* ws = (char*)workspace;
   int* status = (int*)(ws + lay.off_status);
   const int64_t dp = round_up(d, PAD);
@@ -273,7 +275,7 @@ static int factor_one(const float* H, int d, float damp, float* L, int64_t Lp, f
   }
   {
     dim3 blk(32, 8), grid((unsigned)(Lp / 32), (unsigned)(Lp / 32));
-    k_assemble<RT><<<grid, blk, 0, s>>>(C, X, dp, d, L, Lp, Lp, rdiag);
+    k_assemble<RT><<<grid, blk, 0, s>>>(C, X, dp, d, L, Llo, Lp, Lp, rdiag);
   }
   BK_CUDA_OK(cudaGetLastError());
   return BAKRON_OK;
@@ -289,17 +291,17 @@ int prepare_impl(const float* A, const float* B, int m, int n, float damp, void*
   BK_CUDA_OK(cudaMemsetAsync((char*)workspace + pl.off_status, 0, 256, s));
   int rc;
   if (fp32) {
-    rc = factor_one<float>(A, n, damp, (float*)(f + fl.off_LA), fl.np, (float*)(f + fl.off_rA),
-                           workspace, pl, s);
+    rc = factor_one<float>(A, n, damp, (float*)(f + fl.off_LAH), (float*)(f + fl.off_LAL),
+                           fl.np, (float*)(f + fl.off_rA), workspace, pl, s);
     if (rc == BAKRON_OK)
-      rc = factor_one<float>(B, m, damp, (float*)(f + fl.off_LB), fl.mp, (float*)(f + fl.off_rB),
-                             workspace, pl, s);
+      rc = factor_one<float>(B, m, damp, (float*)(f + fl.off_LBH), (float*)(f + fl.off_LBL),
+                             fl.mp, (float*)(f + fl.off_rB), workspace, pl, s);
   } else {
-    rc = factor_one<double>(A, n, damp, (float*)(f + fl.off_LA), fl.np, (float*)(f + fl.off_rA),
-                            workspace, pl, s);
+    rc = factor_one<double>(A, n, damp, (float*)(f + fl.off_LAH), (float*)(f + fl.off_LAL),
+                            fl.np, (float*)(f + fl.off_rA), workspace, pl, s);
     if (rc == BAKRON_OK)
-      rc = factor_one<double>(B, m, damp, (float*)(f + fl.off_LB), fl.mp, (float*)(f + fl.off_rB),
-                              workspace, pl, s);
+      rc = factor_one<double>(B, m, damp, (float*)(f + fl.off_LBH), (float*)(f + fl.off_LBL),
+                              fl.mp, (float*)(f + fl.off_rB), workspace, pl, s);
   }
   return rc;
 }

@@ -1,0 +1,574 @@
+// Band products of Alg. 5 on the 5th-generation tensor cores (tcgen05), with
+// FP32-accurate "3xTF32" arithmetic.
+//
+// The update between the two halves of an Alg. 5 node is two restricted band
+// products (Appendix, complexity of BaKron):
+//     stage 1:  M = L^B E_{S1}                 (E masked to the band S1)
+//     stage 2:  X[S2] += Pi_{S2}(M L^A^T)      (only tiles of the band S2 written)
+// Both are plain C = A B^T contractions with A and B K-major (row-major with
+// the contraction index contiguous): stage 1 reads L^B (rows i, K = i') and
+// E^T (rows j', K = i'); stage 2 reads M (rows i, K = j') and L^A (rows j,
+// K = j').  Zeros of the triangular factors above their diagonal come from the
+// data; the only masking is (a) stage-1 E sub-tiles outside S1, which are
+// zero-filled in shared memory instead of loaded, and (b) stage-2 output
+// tiles outside S2, which the epilogue leaves untouched.
+//
+// Precision: every operand is kept in global memory as an exact tf32 pair
+// x = hi + lo (hi = x with the 13 low mantissa bits cleared), and
+//     A B^T ~= A_hi B_hi^T + A_hi B_lo^T + A_lo B_hi^T,
+// three kind::tf32 MMAs into one fp32 TMEM accumulator (the error-compensated
+// split of Markidis et al. 2018 / Ootomo & Yokota 2022).  The dropped
+// lo*lo term and the tf32 rounding of the lo parts are ~2^-20 relative.
+//
+// CTA (192 threads): warp 0 produces (TMA loads, zero fills), warp 1
+// allocates TMEM and issues the MMAs (one thread), warps 2..5 run the
+// epilogue (tcgen05.ld of their 32-lane TMEM quarter).  One 128 x 128 output
+// block per CTA, K staged 32 at a time through a 3-deep shared-memory ring.
+// Every wait is bounded: a timed-out wait records BAKRON_ERR_TIMEOUT and the
+// CTA winds down, draining its own TMA copies and MMAs (with a separate,
+// generous limit) before it frees TMEM.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+#include <stdint.h>
+#include <stdlib.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "profile.cuh"
+#include "tc_gemm.cuh"
+
+namespace bakron {
+
+namespace {
+
+constexpr int BM = 128, BN = 128, BK = 32;     // output block and K stage (fp32 elements)
+constexpr int STAGES = 3;
+constexpr int THREADS = 192;
+constexpr uint32_t TILE_BYTES = BM * BK * 4;   // 16 KiB: one operand plane of one stage
+constexpr uint32_t STAGE_BYTES = 4 * TILE_BYTES;  // A hi, A lo, B hi, B lo
+constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+constexpr uint32_t TMEM_COLS = 128;
+
+enum Mode { MODE_DENSE = 0, MODE_STAGE1 = 1, MODE_STAGE2 = 2 };
+
+struct TcParams {
+  int mode;
+  int k, h, l;          // band node (tile anti-diagonals), stage 1/2
+  int Mt, Nt;           // real 32-tiles per side
+  int nb_rows;          // output 128-blocks along rows (grid.y)
+  int K;                // dense mode: contraction length (multiple of 32)
+  float* out_hi;        // stage 1: M hi; dense: C
+  float* out_lo;        // stage 1: M lo
+  float* X;             // stage 2: accumulated in place
+  int64_t ldo;          // leading dimension of out_hi/out_lo/X (elements)
+  int* status;
+  long long spin_cycles;  // bound of the working waits (clock64 cycles)
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait for the phase of `bar` with the given parity to complete, for at most
+// `limit` cycles.  Returns false on time-out.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, long long limit) {
+  if (mbar_test(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (mbar_test(bar, parity)) return true;
+    if (clock64() - t0 > limit) return false;
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
+                                            int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
+// 128 bytes, 8-row core groups 1024 bytes apart (SBO), version 1.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((addr & 0x3FFFF) >> 4);            // start address
+  d |= (uint64_t)1 << 16;                             // leading byte offset (unused, 1)
+  d |= (uint64_t)(1024 >> 4) << 32;                   // stride byte offset
+  d |= (uint64_t)1 << 46;                             // descriptor version
+  d |= (uint64_t)2 << 61;                             // swizzle: 128 B
+  return d;
+}
+
+// Instruction descriptor: kind::tf32, D fp32, A and B tf32 K-major, M x N.
+__host__ __device__ constexpr uint32_t idesc_tf32(int M, int N) {
+  return (1u << 4)            // D format fp32
+         | (2u << 7)          // A format tf32
+         | (2u << 10)         // B format tf32
+         | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_tf32(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Output block and K range of this CTA.  Returns false if the block has no
+// work at all (stage 2 outside the band, or beyond the real tiles).
+struct Block {
+  int rb, cb;         // output block (128-row block, 128-col block)
+  int k0, nk;         // first K tile (32 wide) and number of K tiles
+};
+
+__device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
+  b.rb = blockIdx.y;
+  const int I0 = 4 * b.rb;                     // first 32-tile row of the block
+  if (P.mode == MODE_DENSE) {
+    b.cb = blockIdx.x;
+    b.k0 = 0;
+    b.nk = P.K / BK;
+    return true;
+  }
+  if (I0 >= P.Mt) return false;
+  // output 32-tiles (I, J) of the band S2 = [h, l) in rows I0..I0+3
+  const int Ilast = min(I0 + 3, P.Mt - 1);
+  const int jout_lo = max(0, P.h - Ilast);
+  const int jout_hi = min(P.Nt - 1, P.l - 1 - I0);
+  if (jout_lo > jout_hi) return false;
+  if (P.mode == MODE_STAGE1) {
+    // M tiles (I, J') needed by stage 2 for these rows
+    const int jp_lo = max(0, P.k - Ilast);
+    const int jp_hi = min(P.h - 1, jout_hi);
+    if (jp_lo > jp_hi) return false;
+    b.cb = jp_lo / 4 + blockIdx.x;
+    if (b.cb > jp_hi / 4) return false;
+    // K tiles I' with some (I', J') in S1, J' in this column block, I' <= I
+    const int J0 = 4 * b.cb;
+    const int ilo = max(0, P.k - (J0 + 3));
+    const int ihi = min(I0 + 3, P.h - 1 - J0);
+    b.k0 = ilo;
+    b.nk = ihi >= ilo ? ihi - ilo + 1 : 0;
+    return true;
+  }
+  // stage 2 (K starts where stage 1's M coverage of these rows starts; M tiles
+  // of real rows below k - I are exact zeros there)
+  b.cb = jout_lo / 4 + blockIdx.x;
+  if (b.cb > jout_hi / 4) return false;
+  const int J0 = 4 * b.cb;
+  const int jlo = max(0, P.k - Ilast);
+  const int jhi = min(J0 + 3, P.h - 1);
+  b.k0 = jlo;
+  b.nk = jhi >= jlo ? jhi - jlo + 1 : 0;
+  return true;
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUtensorMap mapAl,
+          const __grid_constant__ CUtensorMap mapBh, const __grid_constant__ CUtensorMap mapBl,
+          const TcParams P) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  // 1024-byte alignment for the 128-byte swizzle atoms
+  unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint64_t* bars = (uint64_t*)(smem + STAGES * STAGE_BYTES);
+  uint64_t* full = bars;                 // [STAGES]
+  uint64_t* empty = bars + STAGES;       // [STAGES]
+  uint64_t* accum = bars + 2 * STAGES;   // [1]
+  uint32_t* tmem_slot = (uint32_t*)(bars + 2 * STAGES + 1);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  Block blk;
+  const bool has_block = block_of(P, blk);
+  if (!has_block) return;   // uniform over the CTA: nothing allocated yet
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(accum, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = *tmem_slot;
+  const long long drain = 4000000000LL;   // ~2 s at 2 GHz: wind-down bound
+  const int nk = blk.nk;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------- producer
+    int issued = 0;
+    for (int i = 0; i < nk; ++i) {
+      const int s = i % STAGES;
+      const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
+      bool ok = true;
+      if (lane == 0) ok = mbar_wait(&empty[s], ph ^ 1u, P.spin_cycles);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok || *abort_flag) {
+        if (lane == 0 && !ok) { raise_status(P.status, BAKRON_ERR_TIMEOUT); *abort_flag = 1; }
+        break;
+      }
+      unsigned char* st = smem + s * STAGE_BYTES;
+      unsigned char *a_hi = st, *a_lo = st + TILE_BYTES, *b_hi = st + 2 * TILE_BYTES,
+                    *b_lo = st + 3 * TILE_BYTES;
+      const int kt = blk.k0 + i;            // K tile index (32 wide)
+      uint32_t bytes = 2 * TILE_BYTES;      // A hi + A lo always loaded
+      unsigned valid = 0xF;                 // stage 1: B sub-tiles in the band
+      if (P.mode == MODE_STAGE1) {
+        valid = 0;
+        for (int sub = 0; sub < 4; ++sub) {
+          const int Jp = 4 * blk.cb + sub;
+          const bool v = Jp < P.Nt && kt < P.Mt && kt + Jp >= P.k && kt + Jp < P.h;
+          if (v) valid |= 1u << sub;
+        }
+        // zero-fill the sub-tiles outside the band (4 KiB each, hi and lo)
+        for (int sub = 0; sub < 4; ++sub) {
+          if (valid & (1u << sub)) continue;
+          float4* zh = reinterpret_cast<float4*>(b_hi + sub * 4096);
+          float4* zl = reinterpret_cast<float4*>(b_lo + sub * 4096);
+          for (int e = lane; e < 256; e += 32) {
+            zh[e] = make_float4(0.f, 0.f, 0.f, 0.f);
+            zl[e] = make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        bytes += 2u * 4096u * (uint32_t)__popc(valid);
+      } else {
+        bytes += 2 * TILE_BYTES;
+      }
+      if (lane == 0) {
+        mbar_expect_tx(&full[s], bytes);
+        tma_load_2d(a_hi, &mapAh, &full[s], kt * BK, blk.rb * BM);
+        tma_load_2d(a_lo, &mapAl, &full[s], kt * BK, blk.rb * BM);
+        if (P.mode == MODE_STAGE1) {
+          for (int sub = 0; sub < 4; ++sub) {
+            if (!(valid & (1u << sub))) continue;
+            const int y = (4 * blk.cb + sub) * 32;
+            tma_load_2d(b_hi + sub * 4096, &mapBh, &full[s], kt * BK, y);
+            tma_load_2d(b_lo + sub * 4096, &mapBl, &full[s], kt * BK, y);
+          }
+        } else {
+          tma_load_2d(b_hi, &mapBh, &full[s], kt * BK, blk.cb * BN);
+          tma_load_2d(b_lo, &mapBl, &full[s], kt * BK, blk.cb * BN);
+        }
+      }
+      __syncwarp();
+      issued = i + 1;
+    }
+    // drain: every copy this warp issued has landed before the CTA winds down
+    if (lane == 0) {
+      const int first = issued > STAGES ? issued - STAGES : 0;
+      for (int i = first; i < issued; ++i) {
+        if (!mbar_wait(&full[i % STAGES], (uint32_t)(i / STAGES) & 1u, drain))
+          raise_status(P.status, BAKRON_ERR_TIMEOUT);
+      }
+    }
+  } else if (warp == 1) {
+    // --------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = idesc_tf32(BM, BN);
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % STAGES;
+        const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
+        if (!mbar_wait(&full[s], ph, P.spin_cycles) || *abort_flag) {
+          raise_status(P.status, BAKRON_ERR_TIMEOUT);
+          *abort_flag = 1;
+          break;
+        }
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t st = smem_u32(smem + s * STAGE_BYTES);
+        const uint32_t a_hi = st, a_lo = st + TILE_BYTES, b_hi = st + 2 * TILE_BYTES,
+                       b_lo = st + 3 * TILE_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < BK / 8; ++kk) {
+          const uint32_t off = kk * 32;   // 8 tf32 = 32 bytes along K inside the swizzle row
+          const uint32_t acc0 = (i > 0 || kk > 0) ? 1u : 0u;
+          mma_tf32(tmem, smem_desc(a_hi + off), smem_desc(b_hi + off), idesc, acc0);
+          mma_tf32(tmem, smem_desc(a_hi + off), smem_desc(b_lo + off), idesc, 1u);
+          mma_tf32(tmem, smem_desc(a_lo + off), smem_desc(b_hi + off), idesc, 1u);
+        }
+        mma_commit(&empty[s]);   // frees the stage when these MMAs are done
+      }
+      if (nk > 0) mma_commit(accum);  // tracks every MMA issued above
+      else mbar_arrive(accum);
+      // wind-down guard: all issued MMAs complete before anyone frees TMEM
+      if (!mbar_wait(accum, 0, drain)) raise_status(P.status, BAKRON_ERR_TIMEOUT);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;                 // TMEM lane quarter of this warp
+    const int row = q * 32 + lane;          // row inside the 128 x 128 block
+    // one lane waits; the decision is warp-uniform (tcgen05.ld is warp-collective)
+    int ok = 1;
+    if (lane == 0) {
+      ok = mbar_wait(accum, 0, P.spin_cycles) ? 1 : 0;
+      if (!ok) raise_status(P.status, BAKRON_ERR_TIMEOUT);
+      if (*abort_flag) ok = 0;
+    }
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const bool write = ok != 0;
+    const int64_t gi = (int64_t)blk.rb * BM + row;
+#pragma unroll 1
+    for (int c = 0; c < BN / 32; ++c) {
+      float v[32];
+      if (nk > 0 && write) {
+        tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(c * 32), v);
+      } else {
+#pragma unroll
+        for (int u = 0; u < 32; ++u) v[u] = 0.f;
+      }
+      if (!write) continue;
+      const int64_t gj = (int64_t)blk.cb * BN + c * 32;
+      if (P.mode == MODE_DENSE) {
+        float4* o = reinterpret_cast<float4*>(P.out_hi + gi * P.ldo + gj);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) o[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+      } else if (P.mode == MODE_STAGE1) {
+        float4* oh = reinterpret_cast<float4*>(P.out_hi + gi * P.ldo + gj);
+        float4* ol = reinterpret_cast<float4*>(P.out_lo + gi * P.ldo + gj);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          float hi[4], lo[4];
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            hi[w] = tf32_hi(v[4 * u + w]);
+            lo[w] = v[4 * u + w] - hi[w];
+          }
+          oh[u] = make_float4(hi[0], hi[1], hi[2], hi[3]);
+          ol[u] = make_float4(lo[0], lo[1], lo[2], lo[3]);
+        }
+      } else {
+        // stage 2: add into X only on tiles of the band S2
+        const int I = (int)(gi / 32), J = (int)(gj / 32);
+        if (nk == 0 || I >= P.Mt || J >= P.Nt || I + J < P.h || I + J >= P.l) continue;
+        float4* o = reinterpret_cast<float4*>(P.X + gi * P.ldo + gj);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          float4 x = o[u];
+          x.x += v[4 * u];
+          x.y += v[4 * u + 1];
+          x.z += v[4 * u + 2];
+          x.w += v[4 * u + 3];
+          o[u] = x;
+        }
+      }
+    }
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 1) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// ------------------------------------------------------------- host side
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+bool get_encode() {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+  });
+  return g_encode != nullptr;
+}
+
+// 2-D fp32 row-major matrix (rows x cols, row stride ld elements), box of
+// 32 columns (128 bytes, one swizzle row) by box_rows rows, 128-byte swizzle.
+bool make_map(CUtensorMap* map, const float* base, int64_t rows, int64_t cols, int64_t ld,
+              int box_rows) {
+  if (!get_encode()) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)(ld * 4)};
+  cuuint32_t box[2] = {32u, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1u, 1u};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, (void*)base, dims, strides, box,
+                        estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+long long spin_cycles_from_env() {
+  const char* e = getenv("BAKRON_SPIN_CYCLES");
+  if (e && *e) {
+    long long v = atoll(e);
+    if (v >= 0) return v;
+  }
+  return 4000000000LL;  // ~2 s at 2 GHz
+}
+
+bool g_attr_done = false;
+std::mutex g_attr_mu;
+
+cudaError_t ensure_attr() {
+  std::lock_guard<std::mutex> lk(g_attr_mu);
+  if (g_attr_done) return cudaSuccess;
+  cudaError_t e =
+      cudaFuncSetAttribute(k_tc_band, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  if (e == cudaSuccess) g_attr_done = true;
+  return e;
+}
+
+// hi/lo split of a dense matrix (diagnostic GEMM only)
+__global__ void k_split(const float* src, int64_t count, float* hi, float* lo) {
+  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i >= count) return;
+  const float v = src[i], h = tf32_hi(v);
+  hi[i] = h;
+  lo[i] = v - h;
+}
+
+}  // namespace
+
+bool tc_band_maps(TcMaps& maps, const TcOperands& op) {
+  // stage 1: A = L^B (mp x mp), B = E^T (np x mp) in 32-row boxes
+  // stage 2: A = M (mp x np), B = L^A (np x np)
+  bool ok = true;
+  ok &= make_map(&maps.LBh, op.LBH, op.mp, op.mp, op.mp, BM);
+  ok &= make_map(&maps.LBl, op.LBL, op.mp, op.mp, op.mp, BM);
+  ok &= make_map(&maps.Eth, op.EtH, op.np, op.mp, op.mp, 32);
+  ok &= make_map(&maps.Etl, op.EtL, op.np, op.mp, op.mp, 32);
+  ok &= make_map(&maps.Mh, op.MH, op.mp, op.np, op.np, BM);
+  ok &= make_map(&maps.Ml, op.ML, op.mp, op.np, op.np, BM);
+  ok &= make_map(&maps.LAh, op.LAH, op.np, op.np, op.np, BN);
+  ok &= make_map(&maps.LAl, op.LAL, op.np, op.np, op.np, BN);
+  return ok;
+}
+
+int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, int h, int l,
+                  cudaStream_t s) {
+  if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
+  TcParams P{};
+  P.mode = stage == 1 ? MODE_STAGE1 : MODE_STAGE2;
+  P.k = k; P.h = h; P.l = l;
+  P.Mt = op.Mt; P.Nt = op.Nt;
+  P.nb_rows = (int)(op.mp / BM);
+  P.out_hi = op.MH; P.out_lo = op.ML; P.X = op.X;
+  P.ldo = op.np;
+  P.status = op.status;
+  P.spin_cycles = spin_cycles_from_env();
+  // grid.x spans the widest row of output blocks
+  const int width = stage == 1 ? (h + 3) / 4 + 2 : (l - h + 3) / 4 + 2;
+  dim3 grid(width, P.nb_rows);
+  if (stage == 1)
+    k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(maps.LBh, maps.LBl, maps.Eth, maps.Etl, P);
+  else
+    k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(maps.Mh, maps.Ml, maps.LAh, maps.LAl, P);
+  return cudaGetLastError() == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
+}
+
+}  // namespace bakron
+
+using namespace bakron;
+
+extern "C" int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C, int M, int N,
+                                       int K, void* workspace, size_t workspace_bytes,
+                                       void* stream) {
+  if (!A || !B || !C || !workspace || M <= 0 || N <= 0 || K <= 0) return BAKRON_ERR_INVALID_ARG;
+  if (M % BM || N % BN || K % BK) return BAKRON_ERR_INVALID_ARG;
+  const size_t need = 256 + size_t(2) * (size_t(M) + N) * K * 4;
+  if (workspace_bytes < need) return BAKRON_ERR_WORKSPACE;
+  if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
+  cudaStream_t s = (cudaStream_t)stream;
+  char* ws = (char*)workspace;
+  int* status = (int*)ws;
+  float* Ah = (float*)(ws + 256);
+  float* Al = Ah + (size_t)M * K;
+  float* Bh = Al + (size_t)M * K;
+  float* Bl = Bh + (size_t)N * K;
+  BK_CUDA_OK(cudaMemsetAsync(status, 0, 256, s));
+  k_split<<<(unsigned)(((int64_t)M * K + 255) / 256), 256, 0, s>>>(A, (int64_t)M * K, Ah, Al);
+  k_split<<<(unsigned)(((int64_t)N * K + 255) / 256), 256, 0, s>>>(B, (int64_t)N * K, Bh, Bl);
+  CUtensorMap mA, mAl, mB, mBl;
+  if (!make_map(&mA, Ah, M, K, K, BM) || !make_map(&mAl, Al, M, K, K, BM) ||
+      !make_map(&mB, Bh, N, K, K, BN) || !make_map(&mBl, Bl, N, K, K, BN))
+    return BAKRON_ERR_CUDA;
+  TcParams P{};
+  P.mode = MODE_DENSE;
+  P.K = K;
+  P.nb_rows = M / BM;
+  P.out_hi = C;
+  P.ldo = N;
+  P.status = status;
+  P.spin_cycles = spin_cycles_from_env();
+  dim3 grid(N / BN, M / BM);
+  k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(mA, mAl, mB, mBl, P);
+  BK_CUDA_OK(cudaGetLastError());
+  return bakron_read_status(workspace, stream);
+}

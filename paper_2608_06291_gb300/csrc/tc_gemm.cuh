@@ -1,0 +1,30 @@
+// Tensor-core (tcgen05, 3xTF32) band products: host interface (tc_gemm.cu).
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace bakron {
+
+// Device operands of the band products, in the solve's workspace/factor layout.
+struct TcOperands {
+  int64_t mp, np;      // padded sides (multiples of 128)
+  int Mt, Nt;          // real 32-tiles per side
+  const float *LBH, *LBL, *LAH, *LAL;
+  float *EtH, *EtL, *MH, *ML, *X;
+  int* status;
+};
+
+// TMA descriptors of every operand plane (built on the host per solve call).
+struct TcMaps {
+  CUtensorMap LBh, LBl, Eth, Etl, Mh, Ml, LAh, LAl;
+};
+
+bool tc_band_maps(TcMaps& maps, const TcOperands& op);
+
+// Stage 1 (M = L^B E on the band [k, h)) or stage 2 (X += M L^A^T on the
+// band [h, l)) of one Alg. 5 node, over 128 x 128 output blocks.
+int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, int h, int l,
+                  cudaStream_t s);
+
+}  // namespace bakron
