@@ -5,7 +5,8 @@ Workload (default): the 4096 x 4096 attention-projection layer -- W bf16
 ~N(0, 0.02^2) with 0.1% outlier columns x10, A and B power-law Grams from 8192
 samples, 1% damping, 4-bit per-row grid -- drawn by ``workloads`` on the GPU.
 A step is one bakron_solve (grid, leaf wavefronts and all band products) on
-one resident W with the factors prepared beforehand; the device prepare is
+one resident W with the factors prepared beforehand, replayed from a CUDA
+graph captured once (``--no-graph`` launches eagerly); the device prepare is
 timed separately and reported in ``prepare_ms``.  L2 is flushed (256 MiB
 write) between timed steps, outside the timed events.
 
@@ -226,15 +227,31 @@ def run_gpu(args):
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
-    def step():
+    def eager_step():
         P.bakron_solve(W, fac, cfg.bits, cfg.group, workspace=work, sync=False, out=out)
 
     for _ in range(max(3, args.warmup)):
         flush.fill_(1)
-        step()
+        eager_step()
     torch.cuda.synchronize()
     if P.bakron_read_status(work) != 0:
         raise RuntimeError("device status set during warm-up")
+    launches_per_solve = P.bakron_last_launches()
+    graph = None
+    if not args.no_graph:
+        # the solve's launch sequence depends only on shapes and buffers: capture
+        # it once and replay it (no host enqueue cost per kernel)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            eager_step()
+        graph.replay()
+        torch.cuda.synchronize()
+
+    def step():
+        if graph is not None:
+            graph.replay()
+        else:
+            eager_step()
 
     bus = None
     try:
@@ -255,7 +272,7 @@ def run_gpu(args):
         starts[i].record(stream)
         step()
         ends[i].record(stream)
-        launches += P.bakron_last_launches()
+        launches += launches_per_solve
     torch.cuda.synchronize()
     if ws_n > 1:
         torch.distributed.barrier()
@@ -275,43 +292,59 @@ def run_gpu(args):
     prof_steps = max(3, min(args.steps, 10))
     for i in range(prof_steps):
         flush.fill_(i & 0xFF)
-        step()
+        eager_step()
     fam = P.bakron_profile_read()
     P.bakron_profile_enable(False)
     fam_ms = {k: v[1] / prof_steps for k, v in fam.items()}
     fam_n = {k: v[0] // prof_steps for k, v in fam.items()}
+    fam_fl = {k: v[2] / prof_steps for k, v in fam.items()}
 
     peaks = _peaks() or {}
     f_alg = float(m) * n * (m + n)                    # flops of L^B E L^A^T (structural nonzeros)
-    f_band = f_alg - 2.0 * TILE * m * n               # minus the intra-tile part (leaf)
-    band_ms = fam_ms["band1"] + fam_ms["band2"]
-    leaf_ms = fam_ms["leaf"]
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    bf16_sus = float(peaks.get("bf16_tflops_sustained", 1700.0))
+    p_eff = bf16_sus * (1.1 / 2.25) / 3.0             # 3xTF32: tf32 rate (nominal ratio) / 3
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
     fp32_simt_peak = 152 * 128 * 2 * sm_max * 1e6 / 1e12     # TFLOP/s, FFMA on CUDA cores
-    if band_ms >= leaf_ms:
-        achieved = f_band / (band_ms / 1e3) / 1e12
-        roof = {"kernel": "band products (stage 1 M = L^B E, stage 2 X += M L^A^T), SIMT FP32",
+    groups = {
+        "tc": (fam_ms["tc1"] + fam_ms["tc2"], fam_fl["tc1"] + fam_fl["tc2"],
+               fam_n["tc1"] + fam_n["tc2"]),
+        "simt": (fam_ms["band1"] + fam_ms["band2"] + fam_ms["fused"],
+                 fam_fl["band1"] + fam_fl["band2"] + fam_fl["fused"],
+                 fam_n["band1"] + fam_n["band2"] + fam_n["fused"]),
+        "leaf": (fam_ms["leaf"], 17.0 * m * n, fam_n["leaf"]),
+    }
+    dom = max(groups, key=lambda g: groups[g][0])
+    g_ms, g_work, g_n = groups[dom]
+    if dom == "tc":
+        achieved = g_work / (g_ms / 1e3) / 1e12
+        roof = {"kernel": "k_tc_band: band products on tcgen05, 3xTF32 (stages 1 and 2)",
+                "bound": "tensor", "achieved": achieved, "peak": p_eff, "unit": "TFLOP/s",
+                "frac": achieved / p_eff,
+                "peak_source": "of measured: bf16_tflops_sustained x 1.1/2.25 (tf32/bf16) / 3",
+                "algorithmic_per_step": g_work, "launches_per_step": g_n,
+                "traffic": _traffic("tc")}
+    elif dom == "simt":
+        achieved = g_work / (g_ms / 1e3) / 1e12
+        roof = {"kernel": "k_band1_simt/k_band2_simt/k_band_fused_simt: narrow band products",
                 "bound": "alu", "achieved": achieved, "peak": fp32_simt_peak, "unit": "TFLOP/s",
                 "frac": achieved / fp32_simt_peak,
                 "peak_source": "152 SMs x 128 FP32 lanes x 2 flop x sm_max_mhz (derived)",
-                "algorithmic_per_step": f_band, "launches_per_step": fam_n["band1"] + fam_n["band2"],
-                "traffic": _traffic("band")}
+                "algorithmic_per_step": g_work, "launches_per_step": g_n,
+                "traffic": _traffic("simt")}
     else:
-        bytes_leaf = 17.0 * m * n                     # read X, write X and E, write code, factor blocks
-        hbm = float(peaks.get("hbm_gbs", 6800.0))
-        achieved = bytes_leaf / (leaf_ms / 1e3) / 1e9
-        roof = {"kernel": "leaf wavefront", "bound": "hbm", "achieved": achieved, "peak": hbm,
-                "unit": "GB/s", "frac": achieved / hbm, "peak_source": "MEASURED_PEAKS.json hbm_gbs",
-                "algorithmic_per_step": bytes_leaf, "launches_per_step": fam_n["leaf"],
-                "traffic": _traffic("leaf")}
+        achieved = g_work / (g_ms / 1e3) / 1e9
+        roof = {"kernel": "k_leaf: anti-diagonal wavefront of 32x32 tiles", "bound": "hbm",
+                "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                "peak_source": "of measured: hbm_gbs", "algorithmic_per_step": g_work,
+                "launches_per_step": g_n, "traffic": _traffic("leaf")}
+    roof["groups_ms_per_step"] = {k: v[0] for k, v in groups.items()}
     roof["family_ms_per_step"] = fam_ms
     roof["family_launches_per_step"] = fam_n
-    # whole-solve roofline: GEMM work at the FP32-effective
-    # tensor peak (3xTF32: the TF32 rate, derived from the measured bf16 rate by
-    # the nominal 1.1/2.25 ratio, divided by 3) plus the leaves' bytes at HBM rate
-    bf16_sus = float(peaks.get("bf16_tflops_sustained", 1700.0))
-    p_eff = bf16_sus * (1.1 / 2.25) / 3.0
-    t_roof = f_alg / (p_eff * 1e12) + 17.0 * m * n / (float(peaks.get("hbm_gbs", 6800.0)) * 1e9)
+    roof["family_flops_per_step"] = fam_fl
+    # whole-solve roofline: F_alg at the FP32-effective tensor rate plus the
+    # leaves' bytes at HBM rate
+    t_roof = f_alg / (p_eff * 1e12) + 17.0 * m * n / (hbm * 1e9)
     solve_roof = {"fp32_effective_tflops": p_eff, "f_alg_flops": f_alg,
                   "roofline_ms": 1e3 * t_roof, "frac": 1e3 * t_roof / ms,
                   "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained x 1.1/2.25 / 3"}
@@ -321,7 +354,6 @@ def run_gpu(args):
     ch = torch.empty(m, n, dtype=torch.uint8).pin_memory()
     sh = torch.empty(m, G, dtype=torch.float32).pin_memory()
     zh = torch.empty(m, G, dtype=torch.float32).pin_memory()
-    Wd = torch.empty_like(W)
     e2e_steps = max(3, min(args.steps, 10))
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -329,8 +361,8 @@ def run_gpu(args):
     for i in range(e2e_steps):
         flush.fill_(i & 0xFF)
         e0.record(stream)
-        Wd.copy_(Wh, non_blocking=True)
-        P.bakron_solve(Wd, fac, cfg.bits, cfg.group, workspace=work, sync=False, out=out)
+        W.copy_(Wh, non_blocking=True)      # the solve's (captured) input buffer
+        step()
         ch.copy_(codes, non_blocking=True)
         sh.copy_(scales, non_blocking=True)
         zh.copy_(zeros, non_blocking=True)
@@ -364,7 +396,8 @@ def run_gpu(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws_n, "steps": args.steps,
             "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": vs, "dtype": "f32", "data": "synthetic",
-            "config": dict(_config_dict(cfg), parallelism=f"replicas x{ws_n}"),
+            "config": dict(_config_dict(cfg), parallelism=f"replicas x{ws_n}",
+                           launch="cuda graph replay" if graph is not None else "eager"),
             "prepare_ms": prepare_ms, "roofline": roof, "cpu_baseline": cpu_base, "e2e": e2e,
             "gpu_launches": launches, "clocks": clocks, "solve_roofline": solve_roof,
         }
@@ -386,6 +419,8 @@ def main():
     ap.add_argument("--ref-block", type=int, default=256,
                     help="side of the top-left block each reference-arm step solves")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="launch each solve's kernels eagerly instead of replaying a CUDA graph")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

@@ -166,16 +166,22 @@ int bakron_read_status(void* workspace, void* stream);
  * Instrumentation for benchmarks (no counterpart in the paper).
  * bakron_profile_enable(1) makes every later bakron_solve bracket each of its
  * kernel launches with CUDA events on `stream` and accumulate, per kernel
- * family, the number of launches and their device time.  Families:
- *   0 grid + workspace init, 1 leaf wavefront, 2 band product stage 1
- *   (M = L^B E), 3 band product stage 2 (X += M L^A^T), 4 output copy.
+ * family, the number of launches, their device time and their algorithmic
+ * floating-point work.  Families:
+ *   0 grid + workspace init, 1 leaf wavefront (2*32^3 flops per tile),
+ *   2 / 3 band product stage 1 (M = L^B E) / stage 2 (X += M L^A^T) on CUDA
+ *   cores, 4 output copy, 5 / 6 stage 1 / stage 2 on the tensor cores,
+ *   7 both stages of a narrow node fused in one launch on CUDA cores.
+ *   A band stage counts 2*32^3 flops per 32x32 tile product it must form
+ *   (tile pairs inside the band, triangular diagonal blocks counted whole).
  * bakron_profile_read synchronises the device, then returns the totals since
- * the last enable/reset of `family` (launches, milliseconds).
+ * the last bakron_profile_enable (launches, milliseconds, flops; `flops` may
+ * be NULL).
  * bakron_last_launches returns the number of kernels the last bakron_solve
  * call on this host thread enqueued.
  */
 int bakron_profile_enable(int on);
-int bakron_profile_read(int family, int* launches, double* ms);
+int bakron_profile_read(int family, int* launches, double* ms, double* flops);
 int bakron_last_launches(void);
 
 /*

@@ -58,7 +58,8 @@ def lib() -> ctypes.CDLL:
     L.bakron_read_status.restype = i32
     L.bakron_profile_enable.argtypes = [i32]
     L.bakron_profile_enable.restype = i32
-    L.bakron_profile_read.argtypes = [i32, ctypes.POINTER(i32), ctypes.POINTER(ctypes.c_double)]
+    L.bakron_profile_read.argtypes = [i32, ctypes.POINTER(i32), ctypes.POINTER(ctypes.c_double),
+                                      ctypes.POINTER(ctypes.c_double)]
     L.bakron_profile_read.restype = i32
     L.bakron_last_launches.argtypes = []
     L.bakron_last_launches.restype = i32
@@ -217,7 +218,7 @@ def bakron_read_status(workspace, stream=None) -> int:
     return int(lib().bakron_read_status(_ptr(workspace), _stream(stream)))
 
 
-PROFILE_FAMILIES = ("init", "leaf", "band1", "band2", "copy")
+PROFILE_FAMILIES = ("init", "leaf", "band1", "band2", "copy", "tc1", "tc2", "fused")
 
 
 def bakron_profile_enable(on: bool = True) -> None:
@@ -225,13 +226,15 @@ def bakron_profile_enable(on: bool = True) -> None:
 
 
 def bakron_profile_read() -> dict:
-    """{family: (launches, milliseconds)} accumulated since the last enable."""
+    """{family: (launches, milliseconds, flops)} accumulated since the last enable."""
     out = {}
     for i, name in enumerate(PROFILE_FAMILIES):
         n = ctypes.c_int(0)
         ms = ctypes.c_double(0.0)
-        _check(lib().bakron_profile_read(i, ctypes.byref(n), ctypes.byref(ms)), "bakron_profile_read")
-        out[name] = (n.value, ms.value)
+        fl = ctypes.c_double(0.0)
+        _check(lib().bakron_profile_read(i, ctypes.byref(n), ctypes.byref(ms), ctypes.byref(fl)),
+               "bakron_profile_read")
+        out[name] = (n.value, ms.value, fl.value)
     return out
 
 

@@ -25,15 +25,19 @@ __host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Split of an fp32 value into an exact tf32 head and an fp32 tail:
-// hi = x with its 13 low mantissa bits cleared (exactly representable in
-// tf32), lo = x - hi (exact in fp32, |lo| < 2^-10 |x|).  hi + lo == x exactly.
+// hi = x rounded to the nearest value with 10 mantissa bits (the 13 low bits
+// cleared after adding half of their range), lo = x - hi, exact in fp32 with
+// |lo| <= 2^-11 |x|, so hi + lo == x exactly.  Rounding (not truncating) hi
+// makes lo symmetric around zero, so the tensor core's truncation of lo to
+// tf32 errs with random sign instead of always toward x: no bias builds up
+// over long contractions.
 __host__ __device__ inline float tf32_hi(float x) {
 #ifdef __CUDA_ARCH__
-  return __uint_as_float(__float_as_uint(x) & 0xFFFFE000u);
+  return __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
 #else
   union { float f; uint32_t u; } v;
   v.f = x;
-  v.u &= 0xFFFFE000u;
+  v.u = (v.u + 0x1000u) & 0xFFFFE000u;
   return v.f;
 #endif
 }
@@ -97,6 +101,33 @@ struct PrepareLayout {
     bytes = align256(off_scalar + 256);
   }
 };
+
+// Programmatic dependent launch.  Every kernel of the solve waits for the
+// previous kernel on the stream to complete (pdl_wait) before it touches data
+// that kernel or its predecessors wrote, and only then lets the next kernel
+// launch (pdl_trigger).  So the next kernel's launch and prologue overlap this
+// kernel's work, and anything it reads before its own pdl_wait was produced at
+// least two kernels earlier.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
 
 // Device status word (first int of every workspace).  Kernels only ever raise
 // it with atomicMax-free writes of a nonzero code; the host reads and clears.

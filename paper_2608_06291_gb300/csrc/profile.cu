@@ -14,6 +14,7 @@ namespace {
 struct Pending {
   int family;
   cudaEvent_t a, b;
+  double flops;
 };
 std::mutex g_mu;
 bool g_on = false;
@@ -21,6 +22,7 @@ std::vector<Pending> g_pending;
 std::vector<cudaEvent_t> g_free;
 int g_launches[kFamilies] = {};
 double g_ms[kFamilies] = {};
+double g_flops[kFamilies] = {};
 thread_local int t_launch_count = 0;
 
 cudaEvent_t take_event() {
@@ -40,6 +42,7 @@ void drain_locked() {
     cudaEventSynchronize(p.b);
     cudaEventElapsedTime(&ms, p.a, p.b);
     g_ms[p.family] += ms;
+    g_flops[p.family] += p.flops;
     g_launches[p.family] += 1;
     g_free.push_back(p.a);
     g_free.push_back(p.b);
@@ -48,7 +51,8 @@ void drain_locked() {
 }
 }  // namespace
 
-LaunchScope::LaunchScope(int family, cudaStream_t s) : family_(family), s_(s), a_(nullptr) {
+LaunchScope::LaunchScope(int family, cudaStream_t s, double flops)
+    : family_(family), s_(s), a_(nullptr), flops_(flops) {
   ++t_launch_count;
   if (!g_on) return;
   std::lock_guard<std::mutex> lk(g_mu);
@@ -61,10 +65,12 @@ LaunchScope::~LaunchScope() {
   std::lock_guard<std::mutex> lk(g_mu);
   cudaEvent_t b = take_event();
   cudaEventRecord(b, s_);
-  g_pending.push_back({family_, (cudaEvent_t)a_, b});
+  g_pending.push_back({family_, (cudaEvent_t)a_, b, flops_});
 }
 
 void reset_launch_count() { t_launch_count = 0; }
+
+bool profiling_on() { return g_on; }
 
 }  // namespace bakron
 
@@ -73,17 +79,18 @@ using namespace bakron;
 extern "C" int bakron_profile_enable(int on) {
   std::lock_guard<std::mutex> lk(g_mu);
   drain_locked();
-  for (int f = 0; f < kFamilies; ++f) { g_launches[f] = 0; g_ms[f] = 0.0; }
+  for (int f = 0; f < kFamilies; ++f) { g_launches[f] = 0; g_ms[f] = 0.0; g_flops[f] = 0.0; }
   g_on = on != 0;
   return BAKRON_OK;
 }
 
-extern "C" int bakron_profile_read(int family, int* launches, double* ms) {
+extern "C" int bakron_profile_read(int family, int* launches, double* ms, double* flops) {
   if (family < 0 || family >= kFamilies || !launches || !ms) return BAKRON_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> lk(g_mu);
   drain_locked();
   *launches = g_launches[family];
   *ms = g_ms[family];
+  if (flops) *flops = g_flops[family];
   return BAKRON_OK;
 }
 

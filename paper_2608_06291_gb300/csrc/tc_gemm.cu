@@ -13,17 +13,21 @@
 // zero-filled in shared memory instead of loaded, and (b) stage-2 output
 // tiles outside S2, which the epilogue leaves untouched.
 //
-// Precision: every operand is kept in global memory as an exact tf32 pair
-// x = hi + lo (hi = x with the 13 low mantissa bits cleared), and
+// Precision: every operand is kept in global memory as a pair x = hi + lo
+// (hi = x rounded to tf32, lo = x - hi exact in fp32), and
 //     A B^T ~= A_hi B_hi^T + A_hi B_lo^T + A_lo B_hi^T,
 // three kind::tf32 MMAs into one fp32 TMEM accumulator (the error-compensated
-// split of Markidis et al. 2018 / Ootomo & Yokota 2022).  The dropped
-// lo*lo term and the tf32 rounding of the lo parts are ~2^-20 relative.
+// split of Markidis et al. 2018 / Ootomo & Yokota 2022).  The dropped lo*lo
+// term is <= 2^-22 relative and the tensor core's truncation of lo <= 2^-21,
+// with random sign because hi is rounded to nearest.
 //
 // CTA (192 threads): warp 0 produces (TMA loads, zero fills), warp 1
-// allocates TMEM and issues the MMAs (one thread), warps 2..5 run the
-// epilogue (tcgen05.ld of their 32-lane TMEM quarter).  One 128 x 128 output
-// block per CTA, K staged 32 at a time through a 3-deep shared-memory ring.
+// allocates TMEM and issues the MMAs (one thread), warps 2..5 sum the K
+// stages: each 32-wide stage is accumulated afresh in one of two TMEM
+// accumulators and added, in fp32 round-to-nearest, into registers by the
+// warps that own its 32-lane quarter (tcgen05.ld), overlapping the next
+// stage's MMAs.  One 128 x 128 output block per CTA, K staged 32 at a time
+// through a 3-deep shared-memory ring.
 // Every wait is bounded: a timed-out wait records BAKRON_ERR_TIMEOUT and the
 // CTA winds down, draining its own TMA copies and MMAs (with a separate,
 // generous limit) before it frees TMEM.
@@ -49,7 +53,7 @@ constexpr int THREADS = 192;
 constexpr uint32_t TILE_BYTES = BM * BK * 4;   // 16 KiB: one operand plane of one stage
 constexpr uint32_t STAGE_BYTES = 4 * TILE_BYTES;  // A hi, A lo, B hi, B lo
 constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
-constexpr uint32_t TMEM_COLS = 128;
+constexpr uint32_t TMEM_COLS = 2 * BN;          // two accumulators, alternating per K stage
 
 enum Mode { MODE_DENSE = 0, MODE_STAGE1 = 1, MODE_STAGE2 = 2 };
 
@@ -228,16 +232,22 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
   // 1024-byte alignment for the 128-byte swizzle atoms
   unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint64_t* bars = (uint64_t*)(smem + STAGES * STAGE_BYTES);
-  uint64_t* full = bars;                 // [STAGES]
-  uint64_t* empty = bars + STAGES;       // [STAGES]
-  uint64_t* accum = bars + 2 * STAGES;   // [1]
-  uint32_t* tmem_slot = (uint32_t*)(bars + 2 * STAGES + 1);
+  uint64_t* full = bars;                 // [STAGES] smem stage loaded
+  uint64_t* empty = bars + STAGES;       // [STAGES] smem stage consumed by the MMAs
+  uint64_t* accum = bars + 2 * STAGES;   // [1] every MMA of the CTA complete
+  uint64_t* accF = accum + 1;            // [2] accumulator holds a finished K stage
+  uint64_t* accE = accum + 3;            // [2] accumulator read out by the epilogue
+  uint32_t* tmem_slot = (uint32_t*)(accum + 5);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   Block blk;
   const bool has_block = block_of(P, blk);
-  if (!has_block) return;   // uniform over the CTA: nothing allocated yet
+  if (!has_block) {          // uniform over the CTA: nothing allocated yet
+    pdl_wait();
+    pdl_trigger();
+    return;
+  }
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -245,6 +255,10 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
       mbar_init(&empty[s], 1);
     }
     mbar_init(accum, 1);
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&accF[a], 1);
+      mbar_init(&accE[a], 4);          // lane 0 of each epilogue warp
+    }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -259,6 +273,9 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = *tmem_slot;
+  // everything above touched no global memory: now wait for the previous kernel
+  pdl_wait();
+  pdl_trigger();
   const long long drain = 4000000000LL;   // ~2 s at 2 GHz: wind-down bound
   const int nk = blk.nk;
 
@@ -333,12 +350,20 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
     }
   } else if (warp == 1) {
     // --------------------------------------------------------- MMA issuer
+    // Each K stage accumulates afresh into accumulator (stage & 1); the
+    // epilogue adds the stages in fp32 registers.  The tensor core's TF32
+    // accumulation is not round-to-nearest, and its error grows with the
+    // number of MMAs summed in place; restarting every 32 of K bounds it.
     if (lane == 0) {
       const uint32_t idesc = idesc_tf32(BM, BN);
       for (int i = 0; i < nk; ++i) {
         const int s = i % STAGES;
         const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
-        if (!mbar_wait(&full[s], ph, P.spin_cycles) || *abort_flag) {
+        const int a = i & 1;
+        bool ok = mbar_wait(&full[s], ph, P.spin_cycles);
+        // accumulator a was last used by stage i - 2: wait until it was read out
+        if (ok && i >= 2) ok = mbar_wait(&accE[a], (uint32_t)((i >> 1) - 1) & 1u, P.spin_cycles);
+        if (!ok || *abort_flag) {
           raise_status(P.status, BAKRON_ERR_TIMEOUT);
           *abort_flag = 1;
           break;
@@ -347,15 +372,16 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
         const uint32_t st = smem_u32(smem + s * STAGE_BYTES);
         const uint32_t a_hi = st, a_lo = st + TILE_BYTES, b_hi = st + 2 * TILE_BYTES,
                        b_lo = st + 3 * TILE_BYTES;
+        const uint32_t d = tmem + (uint32_t)(a * BN);
 #pragma unroll
         for (int kk = 0; kk < BK / 8; ++kk) {
           const uint32_t off = kk * 32;   // 8 tf32 = 32 bytes along K inside the swizzle row
-          const uint32_t acc0 = (i > 0 || kk > 0) ? 1u : 0u;
-          mma_tf32(tmem, smem_desc(a_hi + off), smem_desc(b_hi + off), idesc, acc0);
-          mma_tf32(tmem, smem_desc(a_hi + off), smem_desc(b_lo + off), idesc, 1u);
-          mma_tf32(tmem, smem_desc(a_lo + off), smem_desc(b_hi + off), idesc, 1u);
+          mma_tf32(d, smem_desc(a_hi + off), smem_desc(b_hi + off), idesc, kk > 0 ? 1u : 0u);
+          mma_tf32(d, smem_desc(a_hi + off), smem_desc(b_lo + off), idesc, 1u);
+          mma_tf32(d, smem_desc(a_lo + off), smem_desc(b_hi + off), idesc, 1u);
         }
-        mma_commit(&empty[s]);   // frees the stage when these MMAs are done
+        mma_commit(&empty[s]);    // frees the smem stage when these MMAs are done
+        mma_commit(&accF[a]);     // hands the stage's sum to the epilogue
       }
       if (nk > 0) mma_commit(accum);  // tracks every MMA issued above
       else mbar_arrive(accum);
@@ -367,27 +393,38 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;                 // TMEM lane quarter of this warp
     const int row = q * 32 + lane;          // row inside the 128 x 128 block
-    // one lane waits; the decision is warp-uniform (tcgen05.ld is warp-collective)
-    int ok = 1;
-    if (lane == 0) {
-      ok = mbar_wait(accum, 0, P.spin_cycles) ? 1 : 0;
-      if (!ok) raise_status(P.status, BAKRON_ERR_TIMEOUT);
-      if (*abort_flag) ok = 0;
-    }
-    ok = __shfl_sync(0xffffffffu, ok, 0);
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    const bool write = ok != 0;
-    const int64_t gi = (int64_t)blk.rb * BM + row;
-#pragma unroll 1
-    for (int c = 0; c < BN / 32; ++c) {
-      float v[32];
-      if (nk > 0 && write) {
-        tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(c * 32), v);
-      } else {
+    float acc[BN];
 #pragma unroll
-        for (int u = 0; u < 32; ++u) v[u] = 0.f;
+    for (int u = 0; u < BN; ++u) acc[u] = 0.f;
+    bool write = true;
+    for (int i = 0; i < nk; ++i) {
+      const int a = i & 1;
+      // one lane waits; the decision is warp-uniform (tcgen05.ld is warp-collective)
+      int ok = 1;
+      if (lane == 0) {
+        ok = mbar_wait(&accF[a], (uint32_t)(i >> 1) & 1u, P.spin_cycles) ? 1 : 0;
+        if (!ok) raise_status(P.status, BAKRON_ERR_TIMEOUT);
+        if (*abort_flag) ok = 0;
       }
-      if (!write) continue;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) { write = false; break; }
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll
+      for (int c = 0; c < BN / 32; ++c) {
+        float v[32];
+        tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * BN + c * 32), v);
+#pragma unroll
+        for (int u = 0; u < 32; ++u) acc[c * 32 + u] += v[u];
+      }
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&accE[a]);
+    }
+    const int64_t gi = (int64_t)blk.rb * BM + row;
+#pragma unroll
+    for (int c = 0; c < BN / 32; ++c) {
+      if (!write) break;
+      const float* v = &acc[c * 32];
       const int64_t gj = (int64_t)blk.cb * BN + c * 32;
       if (P.mode == MODE_DENSE) {
         float4* o = reinterpret_cast<float4*>(P.out_hi + gi * P.ldo + gj);
@@ -400,9 +437,9 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
         for (int u = 0; u < 8; ++u) {
           float hi[4], lo[4];
 #pragma unroll
-          for (int w = 0; w < 4; ++w) {
-            hi[w] = tf32_hi(v[4 * u + w]);
-            lo[w] = v[4 * u + w] - hi[w];
+          for (int w2 = 0; w2 < 4; ++w2) {
+            hi[w2] = tf32_hi(v[4 * u + w2]);
+            lo[w2] = v[4 * u + w2] - hi[w2];
           }
           oh[u] = make_float4(hi[0], hi[1], hi[2], hi[3]);
           ol[u] = make_float4(lo[0], lo[1], lo[2], lo[3]);
@@ -526,11 +563,14 @@ int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, in
   // grid.x spans the widest row of output blocks
   const int width = stage == 1 ? (h + 3) / 4 + 2 : (l - h + 3) / 4 + 2;
   dim3 grid(width, P.nb_rows);
+  cudaError_t e;
   if (stage == 1)
-    k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(maps.LBh, maps.LBl, maps.Eth, maps.Etl, P);
+    e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.LBh, maps.LBl, maps.Eth,
+                   maps.Etl, P);
   else
-    k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(maps.Mh, maps.Ml, maps.LAh, maps.LAl, P);
-  return cudaGetLastError() == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
+    e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.Mh, maps.Ml, maps.LAh,
+                   maps.LAl, P);
+  return e == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
 }
 
 }  // namespace bakron

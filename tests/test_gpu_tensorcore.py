@@ -80,3 +80,12 @@ def test_bounded_waits_report_timeout_and_recover(monkeypatch):
     assert e.value.status == 4
     monkeypatch.delenv("BAKRON_SPIN_CYCLES")
     _assert_parity(_solve_small(200, 260, 5, bits=4))
+
+
+@pytest.mark.parametrize("fused", ["0", "4", "64"])
+def test_solve_with_fused_narrow_bands(fused, monkeypatch):
+    """Narrow Alg. 5 nodes with both stages fused in one launch (all widths up
+    to 64 when forced) give the oracle's codes."""
+    monkeypatch.setenv("BAKRON_FUSED_MAX_BAND", fused)
+    monkeypatch.setenv("BAKRON_TC_MIN_BAND", "0")
+    _assert_parity(_solve_small(160, 230, 404, bits=4))
