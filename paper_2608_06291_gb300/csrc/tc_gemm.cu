@@ -21,13 +21,14 @@
 // term is <= 2^-22 relative and the tensor core's truncation of lo <= 2^-21,
 // with random sign because hi is rounded to nearest.
 //
-// CTA (192 threads): warp 0 produces (TMA loads, zero fills), warp 1
-// allocates TMEM and issues the MMAs (one thread), warps 2..5 sum the K
-// stages: each 32-wide stage is accumulated afresh in one of two TMEM
-// accumulators and added, in fp32 round-to-nearest, into registers by the
-// warps that own its 32-lane quarter (tcgen05.ld), overlapping the next
-// stage's MMAs.  One 128 x 128 output block per CTA, K staged 32 at a time
-// through a 3-deep shared-memory ring.
+// CTA (320 threads): warp 0 produces (TMA loads, zero fills), warp 1
+// allocates TMEM and issues the MMAs (one thread), warps 2..9 sum the K
+// stages: each 32-wide stage is accumulated afresh in one of four TMEM
+// accumulators and added, in fp32 round-to-nearest, into registers by the two
+// warps that own its 32-lane quarter (64 columns each, tcgen05.ld), while the
+// MMAs of the next stages run.  One 128 x 128 output block per CTA, K staged
+// 32 at a time through a 3-deep shared-memory ring.  The grid covers exactly
+// the bounding box of the output blocks that have work (rows from row0).
 // Every wait is bounded: a timed-out wait records BAKRON_ERR_TIMEOUT and the
 // CTA winds down, draining its own TMA copies and MMAs (with a separate,
 // generous limit) before it frees TMEM.
@@ -37,6 +38,7 @@
 #include <stdint.h>
 #include <stdlib.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "common.cuh"
@@ -49,11 +51,14 @@ namespace {
 
 constexpr int BM = 128, BN = 128, BK = 32;     // output block and K stage (fp32 elements)
 constexpr int STAGES = 3;
-constexpr int THREADS = 192;
+constexpr int EPI_WARPS = 8;                   // two per TMEM lane quarter
+constexpr int THREADS = 32 * (2 + EPI_WARPS);
+constexpr int EPI_COLS = BN / 2;               // columns summed by one epilogue warp
 constexpr uint32_t TILE_BYTES = BM * BK * 4;   // 16 KiB: one operand plane of one stage
 constexpr uint32_t STAGE_BYTES = 4 * TILE_BYTES;  // A hi, A lo, B hi, B lo
 constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
-constexpr uint32_t TMEM_COLS = 2 * BN;          // two accumulators, alternating per K stage
+constexpr int NACC = 4;                         // TMEM accumulators, rotating per K stage
+constexpr uint32_t TMEM_COLS = NACC * BN;       // all 512 columns: one CTA per SM (shared memory)
 
 enum Mode { MODE_DENSE = 0, MODE_STAGE1 = 1, MODE_STAGE2 = 2 };
 
@@ -61,7 +66,7 @@ struct TcParams {
   int mode;
   int k, h, l;          // band node (tile anti-diagonals), stage 1/2
   int Mt, Nt;           // real 32-tiles per side
-  int nb_rows;          // output 128-blocks along rows (grid.y)
+  int row0;             // first output 128-block row (grid.y counts from here)
   int K;                // dense mode: contraction length (multiple of 32)
   float* out_hi;        // stage 1: M hi; dense: C
   float* out_lo;        // stage 1: M lo
@@ -158,8 +163,9 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
       : "memory");
 }
 
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-  uint32_t r[32];
+// 32 lanes x 32 consecutive fp32 columns of TMEM into v (one per column) of
+// each thread; the values are valid only after tmem_wait_ld().
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
       "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
@@ -170,42 +176,61 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
         "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
         "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Output block and K range of this CTA.  Returns false if the block has no
-// work at all (stage 2 outside the band, or beyond the real tiles).
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Output block and K range of this CTA.
 struct Block {
   int rb, cb;         // output block (128-row block, 128-col block)
   int k0, nk;         // first K tile (32 wide) and number of K tiles
 };
 
+// Column blocks [cb_lo, cb_hi] of 128-row block rb that have work in a band
+// stage; false if the row block has none.  Shared by the kernel (which block
+// is this CTA) and the host (the grid's bounding box).
+__host__ __device__ inline bool band_row_span(int mode, int k, int h, int l, int Mt, int Nt, int rb,
+                                              int& cb_lo, int& cb_hi) {
+  const int I0 = 4 * rb;                     // first 32-tile row of the block
+  if (I0 >= Mt) return false;
+  // output 32-tiles (I, J) of the band S2 = [h, l) in rows I0..I0+3
+  const int Ilast = min(I0 + 3, Mt - 1);
+  const int jout_lo = max(0, h - Ilast);
+  const int jout_hi = min(Nt - 1, l - 1 - I0);
+  if (jout_lo > jout_hi) return false;
+  if (mode == MODE_STAGE1) {
+    // M tiles (I, J') needed by stage 2 for these rows
+    const int jp_lo = max(0, k - Ilast);
+    const int jp_hi = min(h - 1, jout_hi);
+    if (jp_lo > jp_hi) return false;
+    cb_lo = jp_lo / 4;
+    cb_hi = jp_hi / 4;
+    return true;
+  }
+  cb_lo = jout_lo / 4;
+  cb_hi = jout_hi / 4;
+  return true;
+}
+
+// Returns false if the block has no work at all (beyond its row's span).
 __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
-  b.rb = blockIdx.y;
-  const int I0 = 4 * b.rb;                     // first 32-tile row of the block
+  b.rb = P.row0 + blockIdx.y;
   if (P.mode == MODE_DENSE) {
     b.cb = blockIdx.x;
     b.k0 = 0;
     b.nk = P.K / BK;
     return true;
   }
-  if (I0 >= P.Mt) return false;
-  // output 32-tiles (I, J) of the band S2 = [h, l) in rows I0..I0+3
-  const int Ilast = min(I0 + 3, P.Mt - 1);
-  const int jout_lo = max(0, P.h - Ilast);
-  const int jout_hi = min(P.Nt - 1, P.l - 1 - I0);
-  if (jout_lo > jout_hi) return false;
+  int cb_lo, cb_hi;
+  if (!band_row_span(P.mode, P.k, P.h, P.l, P.Mt, P.Nt, b.rb, cb_lo, cb_hi)) return false;
+  b.cb = cb_lo + blockIdx.x;
+  if (b.cb > cb_hi) return false;
+  const int I0 = 4 * b.rb, Ilast = min(I0 + 3, P.Mt - 1);
+  const int J0 = 4 * b.cb;
   if (P.mode == MODE_STAGE1) {
-    // M tiles (I, J') needed by stage 2 for these rows
-    const int jp_lo = max(0, P.k - Ilast);
-    const int jp_hi = min(P.h - 1, jout_hi);
-    if (jp_lo > jp_hi) return false;
-    b.cb = jp_lo / 4 + blockIdx.x;
-    if (b.cb > jp_hi / 4) return false;
     // K tiles I' with some (I', J') in S1, J' in this column block, I' <= I
-    const int J0 = 4 * b.cb;
     const int ilo = max(0, P.k - (J0 + 3));
     const int ihi = min(I0 + 3, P.h - 1 - J0);
     b.k0 = ilo;
@@ -214,9 +239,6 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
   }
   // stage 2 (K starts where stage 1's M coverage of these rows starts; M tiles
   // of real rows below k - I are exact zeros there)
-  b.cb = jout_lo / 4 + blockIdx.x;
-  if (b.cb > jout_hi / 4) return false;
-  const int J0 = 4 * b.cb;
   const int jlo = max(0, P.k - Ilast);
   const int jhi = min(J0 + 3, P.h - 1);
   b.k0 = jlo;
@@ -235,9 +257,9 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
   uint64_t* full = bars;                 // [STAGES] smem stage loaded
   uint64_t* empty = bars + STAGES;       // [STAGES] smem stage consumed by the MMAs
   uint64_t* accum = bars + 2 * STAGES;   // [1] every MMA of the CTA complete
-  uint64_t* accF = accum + 1;            // [2] accumulator holds a finished K stage
-  uint64_t* accE = accum + 3;            // [2] accumulator read out by the epilogue
-  uint32_t* tmem_slot = (uint32_t*)(accum + 5);
+  uint64_t* accF = accum + 1;            // [NACC] accumulator holds a finished K stage
+  uint64_t* accE = accum + 1 + NACC;     // [NACC] accumulator read out by the epilogue
+  uint32_t* tmem_slot = (uint32_t*)(accum + 1 + 2 * NACC);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -255,9 +277,9 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
       mbar_init(&empty[s], 1);
     }
     mbar_init(accum, 1);
-    for (int a = 0; a < 2; ++a) {
+    for (int a = 0; a < NACC; ++a) {
       mbar_init(&accF[a], 1);
-      mbar_init(&accE[a], 4);          // lane 0 of each epilogue warp
+      mbar_init(&accE[a], EPI_WARPS);  // lane 0 of each epilogue warp
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -350,7 +372,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
     }
   } else if (warp == 1) {
     // --------------------------------------------------------- MMA issuer
-    // Each K stage accumulates afresh into accumulator (stage & 1); the
+    // Each K stage accumulates afresh into accumulator (stage mod NACC); the
     // epilogue adds the stages in fp32 registers.  The tensor core's TF32
     // accumulation is not round-to-nearest, and its error grows with the
     // number of MMAs summed in place; restarting every 32 of K bounds it.
@@ -359,10 +381,11 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
       for (int i = 0; i < nk; ++i) {
         const int s = i % STAGES;
         const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
-        const int a = i & 1;
+        const int a = i % NACC;
         bool ok = mbar_wait(&full[s], ph, P.spin_cycles);
-        // accumulator a was last used by stage i - 2: wait until it was read out
-        if (ok && i >= 2) ok = mbar_wait(&accE[a], (uint32_t)((i >> 1) - 1) & 1u, P.spin_cycles);
+        // accumulator a was last used by stage i - NACC: wait until it was read out
+        if (ok && i >= NACC)
+          ok = mbar_wait(&accE[a], (uint32_t)(i / NACC - 1) & 1u, P.spin_cycles);
         if (!ok || *abort_flag) {
           raise_status(P.status, BAKRON_ERR_TIMEOUT);
           *abort_flag = 1;
@@ -392,29 +415,33 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
   } else {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;                 // TMEM lane quarter of this warp
+    const int c0 = ((warp - 2) >> 2) * EPI_COLS;   // its half of the 128 columns
     const int row = q * 32 + lane;          // row inside the 128 x 128 block
-    float acc[BN];
+    float acc[EPI_COLS];
 #pragma unroll
-    for (int u = 0; u < BN; ++u) acc[u] = 0.f;
+    for (int u = 0; u < EPI_COLS; ++u) acc[u] = 0.f;
     bool write = true;
     for (int i = 0; i < nk; ++i) {
-      const int a = i & 1;
+      const int a = i % NACC;
       // one lane waits; the decision is warp-uniform (tcgen05.ld is warp-collective)
       int ok = 1;
       if (lane == 0) {
-        ok = mbar_wait(&accF[a], (uint32_t)(i >> 1) & 1u, P.spin_cycles) ? 1 : 0;
+        ok = mbar_wait(&accF[a], (uint32_t)(i / NACC) & 1u, P.spin_cycles) ? 1 : 0;
         if (!ok) raise_status(P.status, BAKRON_ERR_TIMEOUT);
         if (*abort_flag) ok = 0;
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) { write = false; break; }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const uint32_t ta = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * BN + c0);
+      uint32_t r0[32], r1[32];
+      tmem_ld32(ta, r0);
+      tmem_ld32(ta + 32, r1);
+      tmem_wait_ld();
 #pragma unroll
-      for (int c = 0; c < BN / 32; ++c) {
-        float v[32];
-        tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * BN + c * 32), v);
-#pragma unroll
-        for (int u = 0; u < 32; ++u) acc[c * 32 + u] += v[u];
+      for (int u = 0; u < 32; ++u) {
+        acc[u] += __uint_as_float(r0[u]);
+        acc[32 + u] += __uint_as_float(r1[u]);
       }
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       __syncwarp();
@@ -422,10 +449,10 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
     }
     const int64_t gi = (int64_t)blk.rb * BM + row;
 #pragma unroll
-    for (int c = 0; c < BN / 32; ++c) {
+    for (int c = 0; c < EPI_COLS / 32; ++c) {
       if (!write) break;
       const float* v = &acc[c * 32];
-      const int64_t gj = (int64_t)blk.cb * BN + c * 32;
+      const int64_t gj = (int64_t)blk.cb * BN + c0 + c * 32;
       if (P.mode == MODE_DENSE) {
         float4* o = reinterpret_cast<float4*>(P.out_hi + gi * P.ldo + gj);
 #pragma unroll
@@ -555,14 +582,24 @@ int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, in
   P.mode = stage == 1 ? MODE_STAGE1 : MODE_STAGE2;
   P.k = k; P.h = h; P.l = l;
   P.Mt = op.Mt; P.Nt = op.Nt;
-  P.nb_rows = (int)(op.mp / BM);
   P.out_hi = op.MH; P.out_lo = op.ML; P.X = op.X;
   P.ldo = op.np;
   P.status = op.status;
   P.spin_cycles = spin_cycles_from_env();
-  // grid.x spans the widest row of output blocks
-  const int width = stage == 1 ? (h + 3) / 4 + 2 : (l - h + 3) / 4 + 2;
-  dim3 grid(width, P.nb_rows);
+  // bounding box of the output blocks with work: rows [rlo, rhi], and the
+  // widest row's span of column blocks
+  int rlo = -1, rhi = -1, width = 0;
+  const int nb_rows = (int)(op.mp / BM);
+  for (int rb = 0; rb < nb_rows; ++rb) {
+    int cl, ch;
+    if (!band_row_span(P.mode, k, h, l, op.Mt, op.Nt, rb, cl, ch)) continue;
+    if (rlo < 0) rlo = rb;
+    rhi = rb;
+    width = std::max(width, ch - cl + 1);
+  }
+  if (rlo < 0) return BAKRON_OK;   // nothing to do in this stage
+  P.row0 = rlo;
+  dim3 grid(width, rhi - rlo + 1);
   cudaError_t e;
   if (stage == 1)
     e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.LBh, maps.LBl, maps.Eth,
@@ -602,7 +639,7 @@ extern "C" int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C,
   TcParams P{};
   P.mode = MODE_DENSE;
   P.K = K;
-  P.nb_rows = M / BM;
+  P.row0 = 0;
   P.out_hi = C;
   P.ldo = N;
   P.status = status;
