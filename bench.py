@@ -312,7 +312,8 @@ def run_gpu(args):
         "simt": (fam_ms["band1"] + fam_ms["band2"] + fam_ms["fused"],
                  fam_fl["band1"] + fam_fl["band2"] + fam_fl["fused"],
                  fam_n["band1"] + fam_n["band2"] + fam_n["fused"]),
-        "leaf": (fam_ms["leaf"], 17.0 * m * n, fam_n["leaf"]),
+        "leaf": (fam_ms["leaf"] + fam_ms["subtree"], 17.0 * m * n,
+                 fam_n["leaf"] + fam_n["subtree"]),
     }
     dom = max(groups, key=lambda g: groups[g][0])
     g_ms, g_work, g_n = groups[dom]
@@ -334,7 +335,9 @@ def run_gpu(args):
                 "traffic": _traffic("simt")}
     else:
         achieved = g_work / (g_ms / 1e3) / 1e9
-        roof = {"kernel": "k_leaf: anti-diagonal wavefront of 32x32 tiles", "bound": "hbm",
+        roof = {"kernel": "k_leaf / k_subtree: anti-diagonal wavefront of 32x32 tiles "
+                          "(k_subtree: persistent launches of the narrow ranges, leaves plus "
+                          "their band products)", "bound": "hbm",
                 "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
                 "peak_source": "of measured: hbm_gbs", "algorithmic_per_step": g_work,
                 "launches_per_step": g_n, "traffic": _traffic("leaf")}

@@ -171,7 +171,9 @@ int bakron_read_status(void* workspace, void* stream);
  *   0 grid + workspace init, 1 leaf wavefront (2*32^3 flops per tile),
  *   2 / 3 band product stage 1 (M = L^B E) / stage 2 (X += M L^A^T) on CUDA
  *   cores, 4 output copy, 5 / 6 stage 1 / stage 2 on the tensor cores,
- *   7 both stages of a narrow node fused in one launch on CUDA cores.
+ *   7 both stages of a narrow node fused in one launch on CUDA cores,
+ *   8 one persistent launch running a narrow range of the recursion (its
+ *   leaves and band products, separated by grid-wide barriers).
  *   A band stage counts 2*32^3 flops per 32x32 tile product it must form
  *   (tile pairs inside the band, triangular diagonal blocks counted whole).
  * bakron_profile_read synchronises the device, then returns the totals since

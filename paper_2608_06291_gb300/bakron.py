@@ -218,7 +218,7 @@ def bakron_read_status(workspace, stream=None) -> int:
     return int(lib().bakron_read_status(_ptr(workspace), _stream(stream)))
 
 
-PROFILE_FAMILIES = ("init", "leaf", "band1", "band2", "copy", "tc1", "tc2", "fused")
+PROFILE_FAMILIES = ("init", "leaf", "band1", "band2", "copy", "tc1", "tc2", "fused", "subtree")
 
 
 def bakron_profile_enable(on: bool = True) -> None:

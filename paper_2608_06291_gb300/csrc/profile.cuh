@@ -13,7 +13,8 @@ enum {
   kFamTc1 = 5,      // tensor-core band stage 1
   kFamTc2 = 6,      // tensor-core band stage 2
   kFamFused = 7,    // both SIMT stages of a narrow node in one launch
-  kFamilies = 8
+  kFamSubtree = 8,  // persistent cooperative launch of a narrow range (leaves + bands)
+  kFamilies = 9
 };
 
 // Counts one kernel launch; when profiling is on, records an event on the

@@ -22,6 +22,8 @@
 #include "tc_gemm.cuh"
 #include <stdlib.h>
 
+#include <mutex>
+
 namespace bakron {
 
 // ------------------------------------------------------------------ grid
@@ -89,66 +91,164 @@ __global__ void k_copy_out(const float* X, int64_t np, int m, int n, float* out)
 // Intra-tile feedback, with G_q[i] = sum_{j<=q} e_ij L^A[q][j] (row i's
 // committed errors seen from column q), is
 //     x_pq = X_pq + sum_i L^B[p][i] G_q[i].
-// Errors committed on step d - 1 reach (p, q) only through its upper
-// neighbour (p - 1, q) and its left neighbour (p, q - 1), because L^B and L^A
-// are lower triangular with a unit diagonal, so
-//     x_pq = pre_pq + L^B[p][p-1] e_{p-1,q} + L^A[q][q-1] e_{p,q-1},
-//     pre_pq = X_pq + sum_i L^B[p][i] G_q^{(d-2)}[i].
-// Warp 0 runs only that two-term chain and the rounding.  Warps 1..4 each
-// hold 8 rows of G for every column, fold in the errors of step d - 1 and
-// leave partial sums of step d + 1's pre in shared memory, one step ahead of
-// warp 0; one barrier per step orders both directions.
-// A step is latency bound (about fifteen dependent floating-point operations,
-// one shared-memory round and the barrier), so each step moves as few
-// shared-memory words as possible: errors are broadcast indexed by row (every
-// row written every step, zero when off the tile), a helper keeps its L^A
-// values in registers rotated by 8 every 8 steps (compile-time slots), the
-// grid and the sub-diagonal of L^B travel as one float4, and codes are staged
-// in shared memory and stored coalesced at the end.
+// Errors committed on the last few steps reach (p, q) only from a few
+// entries up and to the left of it, because L^B and L^A are lower triangular
+// with a unit diagonal: step d - t contributes the entries (p - a, q - b)
+// with a + b = t, weighted L^B[p][p-a] L^A[q][q-b].  So the work splits into
+//   * the chain (warp 0, lane q = column q): adds the errors of the last two
+//     or three steps explicitly (in registers and shuffles) to a partial pre
+//     and rounds, step after step;
+//   * three helper warps (12 rows of G each): fold older errors into G and
+//     form the partial pre of later steps, sum_i L^B[p][i] G_q[i] (+ X_pq),
+//     which they leave in shared memory.
+// The two sides hand over once per two steps (one barrier); see the
+// wavefront below for the exact lag.  A step is latency bound (a dependent
+// chain of a shuffle and about eight floating-point operations), and every
+// warp of the leaf issues from a scheduler of its own: errors are broadcast
+// indexed by row (every row written every step, zero when off the tile), a
+// helper keeps its L^A values in registers rotated by 8 every 8 steps
+// (compile-time slots), and codes are staged in shared memory and stored
+// coalesced at the end.
 // x / s is evaluated as x * fl(1/s); it can differ from the correctly rounded
 // quotient by one ulp, which only matters within 1e-6 grid units of a
 // rounding boundary.
 // Outputs: codes, X (pre-rounding values) and E^T as a tf32 hi/lo pair.
-constexpr int LEAF_HELPERS = 4;
+// Three helper warps, so that each of the SM's four schedulers runs one warp
+// of the leaf (warp w issues from scheduler w mod 4) and the chain shares its
+// scheduler with nobody; 12 rows each (the last one's rows 32..35 are padding
+// with zero errors and zero L^B).
+constexpr int LEAF_HELPERS = 3;
 constexpr int LEAF_THREADS = 32 * (1 + LEAF_HELPERS);
-constexpr int LEAF_ROWS_PER_HELPER = TILE / LEAF_HELPERS;
+constexpr int LEAF_ROWS_PER_HELPER = 12;
+constexpr int LEAF_ROWS_PADDED = LEAF_HELPERS * LEAF_ROWS_PER_HELPER;   // 36
+static_assert(LEAF_ROWS_PADDED >= TILE && LEAF_ROWS_PADDED <= 36 && LEAF_ROWS_PER_HELPER % 4 == 0,
+              "helper rows: float4 groups inside the 36-wide LBs rows");
 constexpr int LEAF_PER_THREAD = (TILE * TILE + LEAF_THREADS - 1) / LEAF_THREADS;
 
-__global__ void __launch_bounds__(LEAF_THREADS)
-k_leaf(int K, int Mt, int Nt, int m, int n, float* __restrict__ X, int64_t ldx,
-       float* __restrict__ EtH, float* __restrict__ EtL, int64_t ldt,
-       const float* __restrict__ LBH, const float* __restrict__ LBL, int64_t ldb,
-       const float* __restrict__ LAH, const float* __restrict__ LAL, int64_t lda,
-       const float* __restrict__ scales, const float* __restrict__ zeros, int G, int gsz,
-       int qmax, uint8_t* __restrict__ codes, int* status) {
-  const int I = max(0, K - (Nt - 1)) + blockIdx.x;
-  const int J = K - I;
+// Everything a leaf reads besides its tile coordinates.
+struct LeafArgs {
+  int Mt, Nt, m, n;
+  float* X;
+  int64_t ldx;
+  float *EtH, *EtL;
+  int64_t ldt;
+  const float *LBH, *LBL;
+  int64_t ldb;
+  const float *LAH, *LAL;
+  int64_t lda;
+  const float *scales, *zeros;
+  int G, gsz, qmax;
+  uint8_t* codes;
+  int* status;
+};
+
+constexpr int KM = 36;   // row stride of k-major product operands: float4 rows
+
+struct LeafSmem {
+  float Xs[TILE][TILE];                   // W after inbound updates
+  __align__(16) float LBs[TILE][36];      // stride 36: conflict-free float4 row reads
+  float LAs[TILE][TILE + 1];
+  float T1s[TILE][TILE + 1];              // left neighbour's feedback: initial G (absorbing leaf)
+  __align__(16) float Ebr[4][LEAF_ROWS_PADDED];   // errors of a step, by row (ring of 4 steps)
+  float Part[4][LEAF_HELPERS][TILE];              // partial pre of a step (ring of 4 steps)
+  float4 Lsub[TILE];                              // (L^B[p][p-1], L^B[p][p-2], L^B[p][p-3], 0)
+  union {
+    struct {   // prologue of an absorbing leaf: k-major product operands
+      __align__(16) float EL[TILE][KM];   // EL[j][i] = E[I, J-1][i][j]; later U[p][q]
+      __align__(16) float EU[TILE][KM];   // EU[j][i] = E[I-1, J][i][j]
+      __align__(16) float LAt[TILE][KM];  // LAt[j][q] = L^A[J, J-1][q][j]
+      __align__(16) float LBt[TILE][KM];  // LBt[i][p] = L^B[I, I-1][p][i]
+      __align__(16) float T2[TILE][KM];   // T2[i][q] = (E[I-1, J] L^A[J, J]^T)[i][q]
+    } pro;
+    struct {   // the wavefront
+      union {
+        __align__(16) float4 Srzl[TILE][TILE];  // (s, 1/s, -z, 0) per entry
+        float EsT[TILE][TILE + 1];              // after the wavefront: E transposed
+      };
+      __align__(8) float2 XE[TILE][TILE];     // (pre-rounding value, error)
+      uint8_t Cs[TILE][TILE];
+    } w;
+  } u;
+};
+
+// C[r][c] = sum_k At[k][r] B(k, c) for the 4 x 2 block of thread t < 128
+// (rows 4 (t >> 4) .. +3, columns 2 (t & 15) .. +1), k ascending.  At is
+// k-major with row stride KM; B(k, c) = B[k * bsk + c * bsc].
+__device__ __forceinline__ void mm_4x2(const float* At, const float* B, int bsk, int bsc, int t,
+                                       float (&acc)[4][2]) {
+  const int r = 4 * (t >> 4), c = 2 * (t & 15);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) acc[i][0] = acc[i][1] = 0.f;
+#pragma unroll 8
+  for (int k = 0; k < TILE; ++k) {
+    const float4 av = *reinterpret_cast<const float4*>(At + k * KM + r);
+    const float b0 = B[k * bsk + c * bsc], b1 = B[k * bsk + (c + 1) * bsc];
+    acc[0][0] = fmaf(av.x, b0, acc[0][0]);
+    acc[0][1] = fmaf(av.x, b1, acc[0][1]);
+    acc[1][0] = fmaf(av.y, b0, acc[1][0]);
+    acc[1][1] = fmaf(av.y, b1, acc[1][1]);
+    acc[2][0] = fmaf(av.z, b0, acc[2][0]);
+    acc[2][1] = fmaf(av.z, b1, acc[2][1]);
+    acc[3][0] = fmaf(av.w, b0, acc[3][0]);
+    acc[3][1] = fmaf(av.w, b1, acc[3][1]);
+  }
+}
+
+// The leaf's warps (0 .. 4) synchronise on hardware barrier 1 only, so a CTA
+// with more warps can run a leaf while the others wait elsewhere.
+__device__ __forceinline__ void leaf_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(LEAF_THREADS) : "memory");
+}
+
+// Rounds tile (I, J); run by threads 0 .. LEAF_THREADS-1 of the CTA.  With
+// PDL, the factor blocks and the grid (read-only during the solve, the grid
+// written by the solve's first kernel, more than one kernel ago) are loaded
+// before waiting for the previous kernel.
+//
+// An absorbing leaf also applies the Alg. 5 node (K-1, K, K+1) whose band
+// carries the errors of anti-diagonal K-1 into this one: for tile (I, J) that
+// is  L^B[I,I] E[I,J-1] L^A[J,J-1]^T + L^B[I,I-1] E[I-1,J] L^A[J,J]^T.  The
+// first term enters the wavefront as the initial value of G (which the
+// wavefront multiplies by L^B[I,I] anyway): T1 = E[I,J-1] L^A[J,J-1]^T.  The
+// second, U = L^B[I,I-1] (E[I-1,J] L^A[J,J]^T), is added to X before the
+// wavefront.
+template <bool PDL>
+__device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, bool absorb,
+                                          LeafSmem& S) {
   const int t = threadIdx.x, w = t >> 5, lane = t & 31;
-  __shared__ float Xs[TILE][TILE];               // W after inbound updates
-  __shared__ __align__(16) float LBs[TILE][36];  // stride 36: conflict-free float4 row reads
-  __shared__ float LAs[TILE][TILE + 1];
-  __shared__ __align__(16) float4 Srzl[TILE][TILE];   // (s, 1/s, z, L^B[p][p-1]) per entry
-  __shared__ __align__(8) float2 XE[TILE][TILE];      // (pre-rounding value, error)
-  __shared__ float EsT[TILE][TILE + 1];
-  __shared__ uint8_t Cs[TILE][TILE];
-  __shared__ __align__(16) float Ebr[2][TILE];        // errors of a step, indexed by row
-  __shared__ float Part[2][LEAF_HELPERS][TILE];
   const int64_t r0 = (int64_t)I * TILE, c0 = (int64_t)J * TILE;
-  // factor blocks and grid: read-only during the solve (the grid is written by
-  // the solve's first kernel, more than one kernel ago), so load before waiting
+  const bool has_left = absorb && J > 0, has_up = absorb && I > 0;
+  if (has_left || has_up) {
+    // sub-diagonal factor blocks, transposed to k-major (read-only: before the wait)
+#pragma unroll
+    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+      const int e = t + k * LEAF_THREADS;
+      if (e < TILE * TILE) {
+        const int p = e / TILE, c = e % TILE;
+        if (has_left) {
+          const int64_t o = (c0 + p) * a.lda + c0 - TILE + c;
+          S.u.pro.LAt[c][p] = a.LAH[o] + a.LAL[o];
+        }
+        if (has_up) {
+          const int64_t o = (r0 + p) * a.ldb + r0 - TILE + c;
+          S.u.pro.LBt[c][p] = a.LBH[o] + a.LBL[o];
+        }
+      }
+    }
+  }
   float lbv[LEAF_PER_THREAD], lav[LEAF_PER_THREAD], scv[LEAF_PER_THREAD], zv[LEAF_PER_THREAD];
 #pragma unroll
   for (int k = 0; k < LEAF_PER_THREAD; ++k) {
     const int e = t + k * LEAF_THREADS;
     if (e < TILE * TILE) {
       const int p = e / TILE, c = e % TILE;
-      const int64_t ob = (r0 + p) * ldb + r0 + c, oa = (c0 + p) * lda + c0 + c;
-      lbv[k] = LBH[ob] + LBL[ob];
-      lav[k] = LAH[oa] + LAL[oa];
-      const bool real = (r0 + p) < m && (c0 + c) < n;
-      const int64_t og = (r0 + p) * G + (c0 + c) / gsz;
-      scv[k] = real ? scales[og] : 1.f;
-      zv[k] = real ? zeros[og] : 0.f;
+      const int64_t ob = (r0 + p) * a.ldb + r0 + c, oa = (c0 + p) * a.lda + c0 + c;
+      lbv[k] = a.LBH[ob] + a.LBL[ob];
+      lav[k] = a.LAH[oa] + a.LAL[oa];
+      const bool real = (r0 + p) < a.m && (c0 + c) < a.n;
+      const int64_t og = (r0 + p) * a.G + (c0 + c) / a.gsz;
+      scv[k] = real ? a.scales[og] : 1.f;
+      zv[k] = real ? a.zeros[og] : 0.f;
     }
   }
 #pragma unroll
@@ -156,108 +256,230 @@ k_leaf(int K, int Mt, int Nt, int m, int n, float* __restrict__ X, int64_t ldx,
     const int e = t + k * LEAF_THREADS;
     if (e < TILE * TILE) {
       const int p = e / TILE, c = e % TILE;
-      LBs[p][c] = lbv[k];
-      LAs[p][c] = lav[k];
+      S.LBs[p][c] = lbv[k];
+      S.LAs[p][c] = lav[k];
     }
   }
-  pdl_wait();
-  pdl_trigger();
+  if (t < TILE * (36 - TILE)) S.LBs[t / (36 - TILE)][TILE + t % (36 - TILE)] = 0.f;  // padding rows
+  if (PDL) {
+    pdl_wait();
+    pdl_trigger();
+  }
   float xv[LEAF_PER_THREAD];
 #pragma unroll
   for (int k = 0; k < LEAF_PER_THREAD; ++k) {
     const int e = t + k * LEAF_THREADS;
-    if (e < TILE * TILE) xv[k] = X[(r0 + e / TILE) * ldx + c0 + e % TILE];
+    if (e < TILE * TILE) xv[k] = __ldcg(a.X + (r0 + e / TILE) * a.ldx + c0 + e % TILE);
   }
-  __syncthreads();   // LBs complete: the sub-diagonal can be read
+  if (has_left || has_up) {
+    // errors of the neighbours on anti-diagonal K-1, k-major as E^T stores them
+#pragma unroll
+    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+      const int e = t + k * LEAF_THREADS;
+      if (e < TILE * TILE) {
+        const int j = e / TILE, i = e % TILE;
+        if (has_left) {
+          const int64_t o = (c0 - TILE + j) * a.ldt + r0 + i;
+          S.u.pro.EL[j][i] = __ldcg(a.EtH + o) + __ldcg(a.EtL + o);
+        }
+        if (has_up) {
+          const int64_t o = (c0 + j) * a.ldt + r0 - TILE + i;
+          S.u.pro.EU[j][i] = __ldcg(a.EtH + o) + __ldcg(a.EtL + o);
+        }
+      }
+    }
+  }
+  leaf_sync();   // LBs, LAs and the absorbed operands complete
+  if (has_left || has_up) {
+    const int pr = 4 * (t >> 4), pc = 2 * (t & 15);
+    float acc[4][2];
+    if (t < 128) {
+      if (has_left) {   // T1[i][q] = sum_j E[I,J-1][i][j] L^A[J,J-1][q][j]
+        mm_4x2(&S.u.pro.EL[0][0], &S.u.pro.LAt[0][0], KM, 1, t, acc);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          S.T1s[pr + i][pc] = acc[i][0];
+          S.T1s[pr + i][pc + 1] = acc[i][1];
+        }
+      }
+      if (has_up) {     // T2[i][q] = sum_j E[I-1,J][i][j] L^A[J,J][q][j]
+        mm_4x2(&S.u.pro.EU[0][0], &S.LAs[0][0], 1, TILE + 1, t, acc);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          S.u.pro.T2[pr + i][pc] = acc[i][0];
+          S.u.pro.T2[pr + i][pc + 1] = acc[i][1];
+        }
+      }
+    }
+    leaf_sync();
+    if (has_up) {
+      if (t < 128) {    // U[p][q] = sum_i L^B[I,I-1][p][i] T2[i][q], into EL's place
+        mm_4x2(&S.u.pro.LBt[0][0], &S.u.pro.T2[0][0], KM, 1, t, acc);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          S.u.pro.EL[pr + i][pc] = acc[i][0];
+          S.u.pro.EL[pr + i][pc + 1] = acc[i][1];
+        }
+      }
+      leaf_sync();
+#pragma unroll
+      for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+        const int e = t + k * LEAF_THREADS;
+        if (e < TILE * TILE) xv[k] += S.u.pro.EL[e / TILE][e % TILE];
+      }
+      leaf_sync();   // the wavefront's arrays overlay the prologue's
+    }
+  }
 #pragma unroll
   for (int k = 0; k < LEAF_PER_THREAD; ++k) {
     const int e = t + k * LEAF_THREADS;
     if (e < TILE * TILE) {
       const int p = e / TILE, c = e % TILE;
-      Xs[p][c] = xv[k];
-      Srzl[p][c] = make_float4(scv[k], 1.f / scv[k], zv[k], p > 0 ? LBs[p][p - 1] : 0.f);
+      S.Xs[p][c] = xv[k];
+      S.u.w.Srzl[p][c] = make_float4(scv[k], 1.f / scv[k], -zv[k], 0.f);
     }
   }
-  if (t < 2 * TILE) (&Ebr[0][0])[t] = 0.f;
-  for (int e = t; e < 2 * LEAF_HELPERS * TILE; e += LEAF_THREADS) (&Part[0][0][0])[e] = 0.f;
-  // the pre of step 0 (row 0, only lane 0 is on the tile) is just X[0][q]; thread
-  // t < 32 zeroed exactly this word above and holds X[0][t] in xv[0]
-  if (t < TILE) Part[0][0][t] = xv[0];
-  __syncthreads();
+  if (t < TILE)
+    S.Lsub[t] = make_float4(t >= 1 ? S.LBs[t][t - 1] : 0.f, t >= 2 ? S.LBs[t][t - 2] : 0.f,
+                            t >= 3 ? S.LBs[t][t - 3] : 0.f, 0.f);
+  for (int e = t; e < 4 * LEAF_ROWS_PADDED; e += LEAF_THREADS) (&S.Ebr[0][0])[e] = 0.f;
+  leaf_sync();
+  // ---------------------------------------------------------- the wavefront
+  // Steps go in intervals of two (steps 2k and 2k+1) with one barrier at the
+  // end of each.  In interval k the helpers fold the errors of steps 2k-2 and
+  // 2k-1 (published at the barrier before it) and leave the partial pre of
+  // steps 2k+2 and 2k+3, so the pre of step d covers the errors of steps up
+  // to d-3 (d even) or d-4 (d odd).  The chain adds the rest itself: every
+  // error of the last two (three) steps that reaches (p, q), i.e. entry
+  // (p-a, q-b) for 1 <= a+b <= 2 (3), with weight L^B[p][p-a] L^A[q][q-b].
+  // Its own column's errors it keeps in registers (E1..E3: steps d-1..d-3);
+  // those of the columns to its left (L1_*: column q-1, L2_*: q-2, L3_3:
+  // q-3, each from the step its suffix names back) arrive by shuffles, and
+  // only L1_1, the left neighbour's newest error, is on the critical path.
   const int q = lane;
   if (w == 0) {
     // ------------------------------------------------ the chain
-    const bool col_real = (c0 + q) < n;
-    const float la_sub = q > 0 ? LAs[q][q - 1] : 0.f;
-    const float fq = (float)qmax;
-    bool bad = false;
-    float e_prev = 0.f;
-#pragma unroll 1
-    for (int d = 0; d < 2 * TILE - 1; ++d) {
+    const bool col_real = (c0 + q) < a.n;
+    const int rows_real = a.m - (int)r0;     // rows p < rows_real are inside W
+    const float la1 = q >= 1 ? S.LAs[q][q - 1] : 0.f;
+    const float la2 = q >= 2 ? S.LAs[q][q - 2] : 0.f;
+    const float la3 = q >= 3 ? S.LAs[q][q - 3] : 0.f;
+    const float fq = (float)a.qmax;
+    float E1 = 0.f, E2 = 0.f, E3 = 0.f;
+    float L1_1 = 0.f, L1_2 = 0.f, L1_3 = 0.f, L2_2 = 0.f, L2_3 = 0.f, L3_3 = 0.f;
+    // one step: explicit terms of the last two (ODD: three) steps, then round
+    auto step = [&](int d, bool odd, float pre, const float4& g, const float4& lb) {
       const int p = d - q;
       const bool act = p >= 0 && p < TILE;
-      const int pr = p & (TILE - 1);         // the row this lane writes in Ebr
-      const float e_left = __shfl_up_sync(0xffffffffu, e_prev, 1);
-      float e = 0.f;
-      if (act) {
-        const float* part = &Part[d & 1][0][q];
-        const float pre = (part[0] + part[TILE]) + (part[2 * TILE] + part[3 * TILE]);
-        const float4 g = Srzl[p][q];
-        const float x = fmaf(g.w, e_prev, fmaf(la_sub, e_left, pre));
-        float c = rintf(x * g.y) + g.z;
-        c = fminf(fmaxf(c, 0.f), fq);
-        const float v = __fmul_rn(g.x, __fsub_rn(c, g.z));
-        e = __fsub_rn(v, x);
-        const bool real = (r0 + p) < m && col_real;
-        if (!real) e = 0.f;
-        bad |= !isfinite(x);
-        XE[p][q] = make_float2(x, e);
-        Cs[p][q] = (uint8_t)c;
+      // age the left columns' errors by one step, then fetch the new ones
+      L1_3 = L1_2;
+      L1_2 = L1_1;
+      L2_3 = L2_2;
+      L2_2 = __shfl_up_sync(0xffffffffu, L1_2, 1);   // column q-2, step d-2
+      L3_3 = __shfl_up_sync(0xffffffffu, L2_3, 1);   // column q-3, step d-3
+      L1_1 = __shfl_up_sync(0xffffffffu, E1, 1);     // column q-1, step d-1
+      float r = fmaf(lb.x, fmaf(la1, L1_2, E1), fmaf(la2, L2_2, pre));
+      r = fmaf(lb.y, E2, r);
+      if (odd) {
+        r = fmaf(la3, L3_3, r);
+        r = fmaf(lb.x, la2 * L2_3, r);
+        r = fmaf(lb.y, la1 * L1_3, r);
+        r = fmaf(lb.z, E3, r);
       }
-      Ebr[d & 1][pr] = e;
-      e_prev = e;
-      __syncthreads();
+      const float x = fmaf(la1, L1_1, r);
+      // code c = clamp(rint(x / s) + z, 0, qmax); with the integer z the
+      // clamp moves before the rounding and the offset after it:
+      // c - z = rint(clamp(x / s, -z, qmax - z)), exactly
+      const float cz = rintf(fminf(fmaxf(x * g.y, g.z), fq + g.z));
+      float e = fmaf(g.x, cz, -x);         // s (c - z) - x, rounded once
+      if (!(act && p < rows_real && col_real)) e = 0.f;
+      if (act) {
+        S.u.w.XE[p][q] = make_float2(x, e);
+        S.u.w.Cs[p][q] = (uint8_t)(cz - g.z);
+      }
+      S.Ebr[d & 3][p & (TILE - 1)] = e;    // rows off the tile get a zero
+      E3 = E2;
+      E2 = E1;
+      E1 = e;
+    };
+    leaf_sync();   // the helpers' pre of steps 0 and 1
+#pragma unroll 1
+    for (int k = 0; k < TILE; ++k) {
+      const int d0 = 2 * k, d1 = 2 * k + 1;
+      const int p0 = (d0 - q) & (TILE - 1), p1 = (d1 - q) & (TILE - 1);
+      const float* pa = &S.Part[d0 & 3][0][q];
+      const float* pb = &S.Part[d1 & 3][0][q];
+      static_assert(LEAF_HELPERS == 3, "the chain sums three partials");
+      const float pre0 = (pa[0] + pa[TILE]) + pa[2 * TILE];
+      const float pre1 = (pb[0] + pb[TILE]) + pb[2 * TILE];
+      const float4 g0 = S.u.w.Srzl[p0][q], g1 = S.u.w.Srzl[p1][q];
+      const float4 lb0 = S.Lsub[p0], lb1 = S.Lsub[p1];
+      step(d0, false, pre0, g0, lb0);
+      if (d1 < 2 * TILE - 1) step(d1, true, pre1, g1, lb1);
+      leaf_sync();
     }
-    if (bad) raise_status(status, BAKRON_ERR_NONFINITE);
   } else {
-    // ------------------------------------------------ helpers: rows i0..i0+7
+    // ------------------------------------------------ helpers: rows i0..i0+11
     const int g = w - 1, i0 = LEAF_ROWS_PER_HELPER * g;
-    // L^A[q][j] in slot (j + 1 + i0 - 8b) mod 32 during steps [8b, 8b + 8), so the
-    // column j = d - 1 - i0 - r folded into row i0 + r sits in slot (u - r) mod 32
+    // L^A[q][j] sits in slot (j + 2 + i0 - 8b) mod 32 during steps [8b, 8b + 8)
+    // (intervals 4b .. 4b+3): the column j = s - i0 - r of row i0 + r that
+    // step s = 8b + 2v - 2 (+1) brings is in slot 2v - r (+1) mod 32
     float LAr[TILE];
 #pragma unroll
-    for (int s = 0; s < TILE; ++s) LAr[s] = LAs[q][(s - 1 - i0) & (TILE - 1)];
+    for (int sl = 0; sl < TILE; ++sl) LAr[sl] = S.LAs[q][(sl - 2 - i0) & (TILE - 1)];
     float Gg[LEAF_ROWS_PER_HELPER];
 #pragma unroll
-    for (int r = 0; r < LEAF_ROWS_PER_HELPER; ++r) Gg[r] = 0.f;
-#pragma unroll 1
-    for (int b = 0; b < (2 * TILE) / 8; ++b) {
+    for (int r = 0; r < LEAF_ROWS_PER_HELPER; ++r)
+      Gg[r] = (has_left && i0 + r < TILE) ? S.T1s[i0 + r][q] : 0.f;
+    // partial pre of step d's entry (row d - q) over these rows
+    auto dot = [&](int d) {
+      const int pn = d - q;
+      float acc = 0.f;
+      if (pn >= 0 && pn < TILE) {
+        float a4[LEAF_ROWS_PER_HELPER / 4];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int d = 8 * b + u;
-        if (d < 2 * TILE - 1) {
-          // fold step d-1's errors: row i0 + r came from column j = d - 1 - i0 - r
-          if (d >= 1) {
-            const float4 e0 = *reinterpret_cast<const float4*>(&Ebr[(d - 1) & 1][i0]);
-            const float4 e1 = *reinterpret_cast<const float4*>(&Ebr[(d - 1) & 1][i0 + 4]);
-            const float ev[8] = {e0.x, e0.y, e0.z, e0.w, e1.x, e1.y, e1.z, e1.w};
-#pragma unroll
-            for (int r = 0; r < LEAF_ROWS_PER_HELPER; ++r)
-              Gg[r] = fmaf(ev[r], LAr[(u - r) & (TILE - 1)], Gg[r]);
-          }
-          // partial pre of step d+1's entry (row d + 1 - q) over these rows
-          const int pn = d + 1 - q;
-          float acc = 0.f;
-          if (pn >= 0 && pn < TILE) {
-            const float4 l0 = *reinterpret_cast<const float4*>(&LBs[pn][i0]);
-            const float4 l1 = *reinterpret_cast<const float4*>(&LBs[pn][i0 + 4]);
-            acc = fmaf(l0.x, Gg[0], fmaf(l0.y, Gg[1], fmaf(l0.z, Gg[2], l0.w * Gg[3]))) +
-                  fmaf(l1.x, Gg[4], fmaf(l1.y, Gg[5], fmaf(l1.z, Gg[6], l1.w * Gg[7])));
-            if (g == 0) acc += Xs[pn][q];
-          }
-          Part[(d + 1) & 1][g][q] = acc;
-          __syncthreads();
+        for (int v = 0; v < LEAF_ROWS_PER_HELPER / 4; ++v) {
+          const float4 l = *reinterpret_cast<const float4*>(&S.LBs[pn][i0 + 4 * v]);
+          a4[v] = fmaf(l.x, Gg[4 * v],
+                       fmaf(l.y, Gg[4 * v + 1], fmaf(l.z, Gg[4 * v + 2], l.w * Gg[4 * v + 3])));
         }
+        static_assert(LEAF_ROWS_PER_HELPER == 12, "three float4 groups per helper");
+        acc = (a4[0] + a4[1]) + a4[2];
+        if (g == 0) acc += S.Xs[pn][q];
+      }
+      S.Part[d & 3][g][q] = acc;
+    };
+    // fold the errors of step sidx (its row i0 + r came from column sidx - i0 - r)
+    auto fold = [&](int sidx, int slot0) {
+      float ev[LEAF_ROWS_PER_HELPER];
+#pragma unroll
+      for (int v = 0; v < LEAF_ROWS_PER_HELPER / 4; ++v) {
+        const float4 e4 = *reinterpret_cast<const float4*>(&S.Ebr[sidx & 3][i0 + 4 * v]);
+        ev[4 * v] = e4.x;
+        ev[4 * v + 1] = e4.y;
+        ev[4 * v + 2] = e4.z;
+        ev[4 * v + 3] = e4.w;
+      }
+#pragma unroll
+      for (int r = 0; r < LEAF_ROWS_PER_HELPER; ++r)
+        Gg[r] = fmaf(ev[r], LAr[(slot0 - r) & (TILE - 1)], Gg[r]);
+    };
+    // the pre of steps 0 and 1: nothing folded yet
+    dot(0);
+    dot(1);
+    leaf_sync();   // the chain's interval 0 may start
+#pragma unroll 1
+    for (int b = 0; b < TILE / 4; ++b) {
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        const int k = 4 * b + v;
+        if (k >= 1) {             // steps 2k-2 and 2k-1 were published at the last barrier
+          fold(2 * k - 2, 2 * v);
+          fold(2 * k - 1, 2 * v + 1);
+        }
+        if (2 * k + 2 < 2 * TILE - 1) dot(2 * k + 2);
+        if (2 * k + 3 < 2 * TILE - 1) dot(2 * k + 3);
+        leaf_sync();
       }
       // next block: the slot of every column drops by 8, i.e. new slot s = old slot s + 8
       float tmp[TILE];
@@ -267,22 +489,35 @@ k_leaf(int K, int Mt, int Nt, int m, int n, float* __restrict__ X, int64_t ldx,
       for (int j = 0; j < TILE; ++j) LAr[j] = tmp[j];
     }
   }
+  leaf_sync();   // the wavefront is done: its arrays are free
   // transpose E through a padded buffer (conflict-free both ways)
   for (int e = t; e < TILE * TILE; e += LEAF_THREADS) {
-    const int a = e / TILE, b = e % TILE;
-    EsT[b][a] = XE[a][b].y;
+    const int r = e / TILE, c = e % TILE;
+    S.u.w.EsT[c][r] = S.u.w.XE[r][c].y;
   }
-  __syncthreads();
+  leaf_sync();
+  bool bad = false;
   for (int e = t; e < TILE * TILE; e += LEAF_THREADS) {
-    const int a = e / TILE, b = e % TILE;
-    X[(r0 + a) * ldx + c0 + b] = XE[a][b].x;
-    if ((r0 + a) < m && (c0 + b) < n) codes[(r0 + a) * n + c0 + b] = Cs[a][b];
-    const float ev = EsT[a][b];            // E^T row c0 + a, column r0 + b
+    const int r = e / TILE, c = e % TILE;
+    const float xr = S.u.w.XE[r][c].x;
+    bad |= !isfinite(xr);
+    a.X[(r0 + r) * a.ldx + c0 + c] = xr;
+    if ((r0 + r) < a.m && (c0 + c) < a.n) a.codes[(r0 + r) * a.n + c0 + c] = S.u.w.Cs[r][c];
+    const float ev = S.u.w.EsT[r][c];        // E^T row c0 + r, column r0 + c
     const float hi = tf32_hi(ev);
-    const int64_t o = (c0 + a) * ldt + r0 + b;
-    EtH[o] = hi;
-    EtL[o] = ev - hi;
+    const int64_t o = (c0 + r) * a.ldt + r0 + c;
+    a.EtH[o] = hi;
+    a.EtL[o] = ev - hi;
   }
+  if (bad) raise_status(a.status, BAKRON_ERR_NONFINITE);
+  leaf_sync();   // shared memory free for the next tile of this CTA
+}
+
+// One CTA per tile of tile anti-diagonal K.
+__global__ void __launch_bounds__(LEAF_THREADS) k_leaf(int K, int absorb, LeafArgs a) {
+  __shared__ LeafSmem S;
+  const int I = max(0, K - (a.Nt - 1)) + blockIdx.x;
+  leaf_tile<true>(a, I, K - I, absorb != 0, S);
 }
 
 // ------------------------------------------------------- band products (SIMT)
@@ -311,7 +546,7 @@ struct TileRegs {
     for (int k = 0; k < SIMT_PER; ++k) {
       const int e = t + SIMT_THREADS * k;
       const int64_t o = (row0 + e / TILE) * ld + col0 + e % TILE;
-      v[k] = hi[o] + lo[o];
+      v[k] = __ldcg(hi + o) + __ldcg(lo + o);   // L2: coherent within a persistent kernel
     }
   }
   // as stored (S[r][c] = tile[r][c]) or transposed (S[c][r] = tile[r][c])
@@ -336,105 +571,110 @@ __device__ __forceinline__ void tile_mac(const float (*A)[TILE + 1], const float
   }
 }
 
-// Stage 1: M[I, J'] = sum_{I' in S1 column J', I' <= I} L^B[I, I'] E[I', J'].
-// grid.y walks the rows that have outputs (from row_lo), grid.x the J' span.
-__global__ void __launch_bounds__(SIMT_THREADS)
-k_band1_simt(Band bd, const float* __restrict__ LBH, const float* __restrict__ LBL, int64_t ldb,
-             const float* __restrict__ EtH, const float* __restrict__ EtL, int64_t ldt,
-             float* __restrict__ MH, float* __restrict__ ML, int64_t ldm) {
-  pdl_wait();
-  pdl_trigger();
-  const int I = bd.row_lo + blockIdx.y;
+struct BandSmem {
+  float As[TILE][TILE + 1];
+  float Bs[TILE][TILE + 1];
+  float Ts[TILE][TILE + 1];
+};
+
+// Operands of the SIMT band products.
+struct BandArgs {
+  const float *LBH, *LBL;
+  int64_t ldb;
+  const float *EtH, *EtL;
+  int64_t ldt;
+  const float *LAH, *LAL;
+  int64_t lda;
+  float *MH, *ML;
+  int64_t ldm;
+  float* X;
+  int64_t ldx;
+};
+
+// Unit (x, y) of stage 1: M tile (I, J') with I = row_lo + y, J' = max(0, k - I) + x.
+__device__ __forceinline__ bool band1_index(const Band& bd, int x, int y, int& I, int& Jp) {
+  I = bd.row_lo + y;
   const int jo_hi = bd.jout_hi(I);
-  if (bd.jout_lo(I) > jo_hi) return;
-  const int Jp = max(0, bd.k - I) + blockIdx.x;
-  if (Jp > min(bd.h - 1, jo_hi)) return;
+  if (bd.jout_lo(I) > jo_hi) return false;
+  Jp = max(0, bd.k - I) + x;
+  return Jp <= min(bd.h - 1, jo_hi);
+}
+
+// Unit (x, y) of stage 2 (and of the fused form): output tile (I, J) of S2.
+__device__ __forceinline__ bool band2_index(const Band& bd, int x, int y, int& I, int& J) {
+  I = bd.row_lo + y;
+  J = bd.jout_lo(I) + x;
+  return J <= bd.jout_hi(I);
+}
+
+// Stage 1: M[I, J'] = sum_{I' in S1 column J', I' <= I} L^B[I, I'] E[I', J'].
+__device__ __forceinline__ void band1_unit(const Band& bd, const BandArgs& a, int I, int Jp,
+                                           BandSmem& S) {
   const int i_lo = max(0, bd.k - Jp), i_hi = min(I, bd.h - 1 - Jp);
-  __shared__ float As[TILE][TILE + 1];
-  __shared__ float Bs[TILE][TILE + 1];
   const int t = threadIdx.x, tr = t / 8, tc = (t % 8) * 4;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
   TileRegs ra, rb;
   // B[kk][col] = E[I'*T + kk][J'*T + col] = E^T[J'*T + col][I'*T + kk]
-  ra.load(LBH, LBL, ldb, (int64_t)I * TILE, (int64_t)i_lo * TILE, t);
-  rb.load(EtH, EtL, ldt, (int64_t)Jp * TILE, (int64_t)i_lo * TILE, t);
+  ra.load(a.LBH, a.LBL, a.ldb, (int64_t)I * TILE, (int64_t)i_lo * TILE, t);
+  rb.load(a.EtH, a.EtL, a.ldt, (int64_t)Jp * TILE, (int64_t)i_lo * TILE, t);
   for (int Ip = i_lo; Ip <= i_hi; ++Ip) {
-    ra.store(As, false, t);
-    rb.store(Bs, true, t);
+    ra.store(S.As, false, t);
+    rb.store(S.Bs, true, t);
     __syncthreads();
     if (Ip < i_hi) {
-      ra.load(LBH, LBL, ldb, (int64_t)I * TILE, (int64_t)(Ip + 1) * TILE, t);
-      rb.load(EtH, EtL, ldt, (int64_t)Jp * TILE, (int64_t)(Ip + 1) * TILE, t);
+      ra.load(a.LBH, a.LBL, a.ldb, (int64_t)I * TILE, (int64_t)(Ip + 1) * TILE, t);
+      rb.load(a.EtH, a.EtL, a.ldt, (int64_t)Jp * TILE, (int64_t)(Ip + 1) * TILE, t);
     }
-    tile_mac(As, Bs, tr, tc, acc);
+    tile_mac(S.As, S.Bs, tr, tc, acc);
     __syncthreads();
   }
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
-    const int64_t o = ((int64_t)I * TILE + tr) * ldm + (int64_t)Jp * TILE + tc + u;
+    const int64_t o = ((int64_t)I * TILE + tr) * a.ldm + (int64_t)Jp * TILE + tc + u;
     const float hi = tf32_hi(acc[u]);
-    MH[o] = hi;
-    ML[o] = acc[u] - hi;
+    a.MH[o] = hi;
+    a.ML[o] = acc[u] - hi;
   }
 }
 
 // Stage 2: X[I, J] += sum_{J' in [max(0, k - I), min(J, h - 1)]} M[I, J'] L^A[J, J']^T.
-__global__ void __launch_bounds__(SIMT_THREADS)
-k_band2_simt(Band bd, const float* __restrict__ LAH, const float* __restrict__ LAL, int64_t lda,
-             const float* __restrict__ MH, const float* __restrict__ ML, int64_t ldm,
-             float* __restrict__ X, int64_t ldx) {
-  pdl_wait();
-  pdl_trigger();
-  const int I = bd.row_lo + blockIdx.y;
-  const int J = bd.jout_lo(I) + blockIdx.x;
-  if (J > bd.jout_hi(I)) return;
+__device__ __forceinline__ void band2_unit(const Band& bd, const BandArgs& a, int I, int J,
+                                           BandSmem& S) {
   const int j_lo = max(0, bd.k - I), j_hi = min(J, bd.h - 1);
-  __shared__ float As[TILE][TILE + 1];
-  __shared__ float Bs[TILE][TILE + 1];   // Bs[t][c] = L^A[J*T + c][J'*T + t]
   const int t = threadIdx.x, tr = t / 8, tc = (t % 8) * 4;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
   TileRegs ra, rb;
-  ra.load(MH, ML, ldm, (int64_t)I * TILE, (int64_t)j_lo * TILE, t);
-  rb.load(LAH, LAL, lda, (int64_t)J * TILE, (int64_t)j_lo * TILE, t);
+  // Bs[t][c] = L^A[J*T + c][J'*T + t]
+  ra.load(a.MH, a.ML, a.ldm, (int64_t)I * TILE, (int64_t)j_lo * TILE, t);
+  rb.load(a.LAH, a.LAL, a.lda, (int64_t)J * TILE, (int64_t)j_lo * TILE, t);
   for (int Jp = j_lo; Jp <= j_hi; ++Jp) {
-    ra.store(As, false, t);
-    rb.store(Bs, true, t);
+    ra.store(S.As, false, t);
+    rb.store(S.Bs, true, t);
     __syncthreads();
     if (Jp < j_hi) {
-      ra.load(MH, ML, ldm, (int64_t)I * TILE, (int64_t)(Jp + 1) * TILE, t);
-      rb.load(LAH, LAL, lda, (int64_t)J * TILE, (int64_t)(Jp + 1) * TILE, t);
+      ra.load(a.MH, a.ML, a.ldm, (int64_t)I * TILE, (int64_t)(Jp + 1) * TILE, t);
+      rb.load(a.LAH, a.LAL, a.lda, (int64_t)J * TILE, (int64_t)(Jp + 1) * TILE, t);
     }
-    tile_mac(As, Bs, tr, tc, acc);
+    tile_mac(S.As, S.Bs, tr, tc, acc);
     __syncthreads();
   }
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
-    float* p = X + ((int64_t)I * TILE + tr) * ldx + (int64_t)J * TILE + tc + u;
-    *p += acc[u];
+    float* p = a.X + ((int64_t)I * TILE + tr) * a.ldx + (int64_t)J * TILE + tc + u;
+    *p = __ldcg(p) + acc[u];
   }
 }
 
-// Both stages of a narrow node in one launch: each CTA owns one output tile
-// (I, J) of S2 and forms the M tiles it needs in shared memory,
+// Both stages for one output tile (I, J) of S2, forming the M tiles it needs
+// in shared memory,
 //     X[I, J] += sum_{J'} ( sum_{I'} L^B[I, I'] E[I', J'] ) L^A[J, J']^T,
 // with the same ranges as the two stages.  Narrow nodes have few (I', J')
 // pairs per output, so recomputing an M tile per output costs little and
-// saves a launch and the round trip of M through global memory.  The pairs
-// are walked as one flat sequence so the next pair's tiles are in flight
-// while the current pair is multiplied.
-__global__ void __launch_bounds__(SIMT_THREADS)
-k_band_fused_simt(Band bd, const float* __restrict__ LBH, const float* __restrict__ LBL,
-                  int64_t ldb, const float* __restrict__ EtH, const float* __restrict__ EtL,
-                  int64_t ldt, const float* __restrict__ LAH, const float* __restrict__ LAL,
-                  int64_t lda, float* __restrict__ X, int64_t ldx) {
-  pdl_wait();
-  pdl_trigger();
-  const int I = bd.row_lo + blockIdx.y;
-  const int J = bd.jout_lo(I) + blockIdx.x;
-  if (J > bd.jout_hi(I)) return;
-  __shared__ float As[TILE][TILE + 1];
-  __shared__ float Bs[TILE][TILE + 1];
-  __shared__ float Ts[TILE][TILE + 1];
+// saves a launch (or a grid-wide barrier) and the round trip of M through
+// global memory.  The pairs are walked as one flat sequence so the next
+// pair's tiles are in flight while the current pair is multiplied.
+__device__ __forceinline__ void fused_unit(const Band& bd, const BandArgs& a, int I, int J,
+                                           BandSmem& S) {
   const int t = threadIdx.x, tr = t / 8, tc = (t % 8) * 4;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
   const int j_lo = max(0, bd.k - I), j_hi = min(J, bd.h - 1);
@@ -443,33 +683,33 @@ k_band_fused_simt(Band bd, const float* __restrict__ LBH, const float* __restric
   TileRegs ra, rb, rl;
   int Jp = j_lo, Ip = ilo(j_lo);
   if (Jp <= j_hi) {
-    ra.load(LBH, LBL, ldb, (int64_t)I * TILE, (int64_t)Ip * TILE, t);
-    rb.load(EtH, EtL, ldt, (int64_t)Jp * TILE, (int64_t)Ip * TILE, t);
-    rl.load(LAH, LAL, lda, (int64_t)J * TILE, (int64_t)Jp * TILE, t);
+    ra.load(a.LBH, a.LBL, a.ldb, (int64_t)I * TILE, (int64_t)Ip * TILE, t);
+    rb.load(a.EtH, a.EtL, a.ldt, (int64_t)Jp * TILE, (int64_t)Ip * TILE, t);
+    rl.load(a.LAH, a.LAL, a.lda, (int64_t)J * TILE, (int64_t)Jp * TILE, t);
   }
   float m4[4] = {0.f, 0.f, 0.f, 0.f};
   while (Jp <= j_hi) {
-    ra.store(As, false, t);
-    rb.store(Bs, true, t);
+    ra.store(S.As, false, t);
+    rb.store(S.Bs, true, t);
     __syncthreads();
     // next (I', J') pair of the flat walk
     int nJp = Jp, nIp = Ip + 1;
     if (nIp > ihi(Jp)) { nJp = Jp + 1; nIp = nJp <= j_hi ? ilo(nJp) : 0; }
     const bool last_of_col = nJp != Jp;
     if (nJp <= j_hi) {
-      ra.load(LBH, LBL, ldb, (int64_t)I * TILE, (int64_t)nIp * TILE, t);
-      rb.load(EtH, EtL, ldt, (int64_t)nJp * TILE, (int64_t)nIp * TILE, t);
+      ra.load(a.LBH, a.LBL, a.ldb, (int64_t)I * TILE, (int64_t)nIp * TILE, t);
+      rb.load(a.EtH, a.EtL, a.ldt, (int64_t)nJp * TILE, (int64_t)nIp * TILE, t);
     }
-    tile_mac(As, Bs, tr, tc, m4);
+    tile_mac(S.As, S.Bs, tr, tc, m4);
     __syncthreads();
     if (last_of_col) {
       // M[I, J'] complete: multiply by L^A[J, J']^T
 #pragma unroll
-      for (int u = 0; u < 4; ++u) Ts[tr][tc + u] = m4[u];
-      rl.store(Bs, true, t);
+      for (int u = 0; u < 4; ++u) S.Ts[tr][tc + u] = m4[u];
+      rl.store(S.Bs, true, t);
       __syncthreads();
-      if (nJp <= j_hi) rl.load(LAH, LAL, lda, (int64_t)J * TILE, (int64_t)nJp * TILE, t);
-      tile_mac(Ts, Bs, tr, tc, acc);
+      if (nJp <= j_hi) rl.load(a.LAH, a.LAL, a.lda, (int64_t)J * TILE, (int64_t)nJp * TILE, t);
+      tile_mac(S.Ts, S.Bs, tr, tc, acc);
       __syncthreads();
 #pragma unroll
       for (int u = 0; u < 4; ++u) m4[u] = 0.f;
@@ -479,12 +719,159 @@ k_band_fused_simt(Band bd, const float* __restrict__ LBH, const float* __restric
   }
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
-    float* p = X + ((int64_t)I * TILE + tr) * ldx + (int64_t)J * TILE + tc + u;
-    *p += acc[u];
+    float* p = a.X + ((int64_t)I * TILE + tr) * a.ldx + (int64_t)J * TILE + tc + u;
+    *p = __ldcg(p) + acc[u];
+  }
+}
+
+// Standalone launches: grid.y walks the rows with outputs (from row_lo),
+// grid.x the span of the row.
+__global__ void __launch_bounds__(SIMT_THREADS) k_band1_simt(Band bd, BandArgs a) {
+  pdl_wait();
+  pdl_trigger();
+  __shared__ BandSmem S;
+  int I, Jp;
+  if (band1_index(bd, blockIdx.x, blockIdx.y, I, Jp)) band1_unit(bd, a, I, Jp, S);
+}
+
+__global__ void __launch_bounds__(SIMT_THREADS) k_band2_simt(Band bd, BandArgs a) {
+  pdl_wait();
+  pdl_trigger();
+  __shared__ BandSmem S;
+  int I, J;
+  if (band2_index(bd, blockIdx.x, blockIdx.y, I, J)) band2_unit(bd, a, I, J, S);
+}
+
+__global__ void __launch_bounds__(SIMT_THREADS) k_band_fused_simt(Band bd, BandArgs a) {
+  pdl_wait();
+  pdl_trigger();
+  __shared__ BandSmem S;
+  int I, J;
+  if (band2_index(bd, blockIdx.x, blockIdx.y, I, J)) fused_unit(bd, a, I, J, S);
+}
+
+// ------------------------------------------------- persistent subtree
+// The bottom of the recursion, rec(k, l) for a narrow range, in one
+// cooperative launch: its leaves and band products run as phases in the
+// order rec would enqueue them, separated by grid-wide barriers instead of
+// kernel boundaries.  Each phase spreads its units (tiles of a leaf, output
+// or M tiles of a band stage) over the CTAs; a CTA runs a leaf with its first
+// five warps and a band unit with all eight.
+enum PhaseType { PH_LEAF = 0, PH_FUSED = 1, PH_STAGE1 = 2, PH_STAGE2 = 3, PH_LEAF_ABSORB = 4 };
+struct Phase {
+  int type, k, h, l;
+};
+constexpr int MAX_SUBTREE = 32;  // widest range run as one subtree (anti-diagonals)
+constexpr int MAX_PHASES = 128;  // >= MAX_SUBTREE leaves + 2 phases per band node
+
+struct SubtreeArgs {
+  LeafArgs leaf;
+  BandArgs band;
+  unsigned* bar_count;   // grid barrier: arrivals of the current generation
+  unsigned* bar_gen;     // grid barrier: generation, bumped by the last arrival
+  long long spin_cycles;
+  int nph;
+  Phase ph[MAX_PHASES];
+};
+
+// Grid-wide barrier of a cooperative launch (every CTA resident).  Thread 0
+// of each CTA publishes the CTA's writes (fence), arrives on the counter and
+// waits, for at most `limit` cycles, for the last arrival to bump the
+// generation.  Returns false on time-out, with BAKRON_ERR_TIMEOUT recorded;
+// the caller then leaves the kernel (the other CTAs time out at their next
+// barrier in turn).  Data written before the barrier is read after it with
+// L2 (coherent) loads.
+__device__ bool grid_sync(unsigned* count, unsigned* gen, long long limit, int* status) {
+  __shared__ int ok_s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int ok = 1;
+    volatile unsigned* vgen = gen;
+    const unsigned g = *vgen;
+    __threadfence();
+    const unsigned arrived = atomicAdd(count, 1u);
+    if (arrived == gridDim.x - 1) {
+      atomicExch(count, 0u);
+      __threadfence();
+      atomicAdd(gen, 1u);
+    } else {
+      const long long t0 = clock64();
+      while (*vgen == g) {
+        if (clock64() - t0 > limit) {
+          ok = 0;
+          break;
+        }
+      }
+    }
+    __threadfence();
+    if (!ok) raise_status(status, BAKRON_ERR_TIMEOUT);
+    ok_s = ok;
+  }
+  __syncthreads();
+  return ok_s != 0;
+}
+
+union SubtreeSmem {
+  LeafSmem leaf;
+  BandSmem band;
+};
+
+__global__ void __launch_bounds__(SIMT_THREADS) k_subtree(const __grid_constant__ SubtreeArgs A) {
+  extern __shared__ __align__(16) unsigned char subtree_smem[];
+  SubtreeSmem& S = *reinterpret_cast<SubtreeSmem*>(subtree_smem);
+  const int Mt = A.leaf.Mt, Nt = A.leaf.Nt;
+  for (int ph = 0; ph < A.nph; ++ph) {
+    const Phase P = A.ph[ph];
+    if (P.type == PH_LEAF || P.type == PH_LEAF_ABSORB) {
+      const int ilo = max(0, P.k - (Nt - 1)), ihi = min(P.k, Mt - 1);
+      if (threadIdx.x < LEAF_THREADS)
+        for (int I = ilo + (int)blockIdx.x; I <= ihi; I += gridDim.x)
+          leaf_tile<false>(A.leaf, I, P.k - I, P.type == PH_LEAF_ABSORB, S.leaf);
+    } else {
+      const int row_lo = max(0, P.h - (Nt - 1)), row_hi = min(Mt - 1, P.l - 1);
+      const Band bd{P.k, P.h, P.l, Mt, Nt, row_lo};
+      const int span = P.type == PH_STAGE1 ? min(P.h, P.l - P.k) : P.l - P.h;
+      const int units = row_hi >= row_lo ? span * (row_hi - row_lo + 1) : 0;
+      for (int u = blockIdx.x; u < units; u += gridDim.x) {
+        const int x = u % span, y = u / span;
+        int I, J;
+        if (P.type == PH_STAGE1) {
+          if (band1_index(bd, x, y, I, J)) band1_unit(bd, A.band, I, J, S.band);
+        } else if (band2_index(bd, x, y, I, J)) {
+          if (P.type == PH_FUSED) fused_unit(bd, A.band, I, J, S.band);
+          else band2_unit(bd, A.band, I, J, S.band);
+        }
+      }
+    }
+    if (ph + 1 < A.nph && !grid_sync(A.bar_count, A.bar_gen, A.spin_cycles, A.leaf.status))
+      return;
   }
 }
 
 // ---------------------------------------------------------------- driver
+// CTAs of k_subtree that fit on the current device at once (occupancy x SMs),
+// queried once per device; -1 on a CUDA error.
+static int subtree_capacity() {
+  static std::mutex mu;
+  static int cap[64];
+  static bool done[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return -1;
+  std::lock_guard<std::mutex> lk(mu);
+  if (dev < 64 && done[dev]) return cap[dev];
+  int sms = 0, per_sm = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return -1;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_subtree, SIMT_THREADS,
+                                                    sizeof(SubtreeSmem)) != cudaSuccess)
+    return -1;
+  const int c = sms * per_sm;
+  if (dev < 64) {
+    cap[dev] = c;
+    done[dev] = true;
+  }
+  return c;
+}
+
 struct SolveArgs {
   int m, n, Mt, Nt, G, gsz, qmax;
   int64_t mp, np;
@@ -497,10 +884,15 @@ struct SolveArgs {
   // tensor-core band products for nodes spanning >= tc_min_band tile anti-diagonals
   int tc_min_band;
   int fused_max_band;   // nodes spanning <= this many tile anti-diagonals: one fused launch
+  int subtree_max;      // ranges spanning <= this many: one persistent cooperative launch
+  int subtree_grid;     // CTAs a cooperative launch may hold (resident at once)
+  long long spin_cycles;
   bool tc_ready;
   bool profiling;
   TcOperands tco;
   TcMaps tcm;
+  LeafArgs la;
+  BandArgs ba;
   int rc;
 };
 
@@ -521,12 +913,17 @@ static void note(SolveArgs& a, cudaError_t e) {
   if (e != cudaSuccess) a.rc = BAKRON_ERR_CUDA;
 }
 
-static void leaf(SolveArgs& a, int K) {
+// Leaf of anti-diagonal K; `absorb`: it also applies the node (K-1, K, K+1).
+static void leaf(SolveArgs& a, int K, int absorb) {
   const int ilo = max(0, K - (a.Nt - 1)), ihi = min(K, a.Mt - 1);
-  LaunchScope ls(kFamLeaf, a.s, 2.0 * TILE * TILE * TILE * (ihi - ilo + 1));
-  note(a, launch_pdl(k_leaf, dim3(ihi - ilo + 1), dim3(LEAF_THREADS), 0, a.s, K, a.Mt, a.Nt, a.m,
-                     a.n, a.X, a.np, a.EtH, a.EtL, a.mp, a.LBH, a.LBL, a.mp, a.LAH, a.LAL, a.np,
-                     a.scales, a.zeros, a.G, a.gsz, a.qmax, a.codes, a.status));
+  double flops = 2.0 * TILE * TILE * TILE * (ihi - ilo + 1);
+  if (absorb && a.profiling) {
+    double p1, p2;
+    band_tile_products(a, K - 1, K, K + 1, p1, p2);
+    flops += 2.0 * TILE * TILE * TILE * (p1 + p2);
+  }
+  LaunchScope ls(kFamLeaf, a.s, flops);
+  note(a, launch_pdl(k_leaf, dim3(ihi - ilo + 1), dim3(LEAF_THREADS), 0, a.s, K, absorb, a.la));
 }
 
 static void band(SolveArgs& a, int k, int h, int l) {
@@ -554,25 +951,102 @@ static void band(SolveArgs& a, int k, int h, int l) {
   dim3 g1(min(h, l - k), row_hi - row_lo + 1), g2(l - h, row_hi - row_lo + 1);
   if (l - k <= a.fused_max_band) {
     LaunchScope ls(kFamFused, a.s, f * (p1 + p2));
-    note(a, launch_pdl(k_band_fused_simt, g2, dim3(256), 0, a.s, bd, a.LBH, a.LBL, a.mp, a.EtH,
-                       a.EtL, a.mp, a.LAH, a.LAL, a.np, a.X, a.np));
+    note(a, launch_pdl(k_band_fused_simt, g2, dim3(SIMT_THREADS), 0, a.s, bd, a.ba));
     return;
   }
   {
     LaunchScope ls(kFamBand1, a.s, f * p1);
-    note(a, launch_pdl(k_band1_simt, g1, dim3(256), 0, a.s, bd, a.LBH, a.LBL, a.mp, a.EtH,
-                       a.EtL, a.mp, a.MH, a.ML, a.np));
+    note(a, launch_pdl(k_band1_simt, g1, dim3(SIMT_THREADS), 0, a.s, bd, a.ba));
   }
   {
     LaunchScope ls(kFamBand2, a.s, f * p2);
-    note(a, launch_pdl(k_band2_simt, g2, dim3(256), 0, a.s, bd, a.LAH, a.LAL, a.np, a.MH, a.ML,
-                       a.np, a.X, a.np));
+    note(a, launch_pdl(k_band2_simt, g2, dim3(SIMT_THREADS), 0, a.s, bd, a.ba));
   }
+}
+
+// Phases of rec(k, l) in the order rec enqueues them.
+static void subtree_phases(const SolveArgs& a, int k, int l, SubtreeArgs& A) {
+  if (l == k + 1) {
+    A.ph[A.nph++] = Phase{PH_LEAF, k, k, l};
+    return;
+  }
+  if (l == k + 2) {   // the node (k, k+1, k+2) is applied by its second leaf
+    A.ph[A.nph++] = Phase{PH_LEAF, k, k, k + 1};
+    A.ph[A.nph++] = Phase{PH_LEAF_ABSORB, k + 1, k + 1, l};
+    return;
+  }
+  const int h = (k + l) / 2;
+  subtree_phases(a, k, h, A);
+  if (l - k <= a.fused_max_band) {
+    A.ph[A.nph++] = Phase{PH_FUSED, k, h, l};
+  } else {
+    A.ph[A.nph++] = Phase{PH_STAGE1, k, h, l};
+    A.ph[A.nph++] = Phase{PH_STAGE2, k, h, l};
+  }
+  subtree_phases(a, h, l, A);
+}
+
+static void subtree(SolveArgs& a, int k, int l) {
+  SubtreeArgs A;
+  A.leaf = a.la;
+  A.band = a.ba;
+  char* st = (char*)a.status;
+  A.bar_count = (unsigned*)(st + 64);
+  A.bar_gen = (unsigned*)(st + 128);
+  A.spin_cycles = a.spin_cycles;
+  A.nph = 0;
+  subtree_phases(a, k, l, A);
+  // as many CTAs as the widest leaf of the range has tiles (band phases
+  // spread their units over the same CTAs)
+  int widest = 1;
+  for (int K = k; K < l; ++K)
+    widest = max(widest, min(K, a.Mt - 1) - max(0, K - (a.Nt - 1)) + 1);
+  const int grid = min(widest, a.subtree_grid);
+  double flops = 0.0;
+  if (a.profiling) {
+    for (int i = 0; i < A.nph; ++i) {
+      const Phase& P = A.ph[i];
+      if (P.type == PH_LEAF || P.type == PH_LEAF_ABSORB) {
+        flops += 2.0 * TILE * TILE * TILE *
+                 (min(P.k, a.Mt - 1) - max(0, P.k - (a.Nt - 1)) + 1);
+        if (P.type == PH_LEAF_ABSORB) {
+          double p1, p2;
+          band_tile_products(a, P.k - 1, P.k, P.k + 1, p1, p2);
+          flops += 2.0 * TILE * TILE * TILE * (p1 + p2);
+        }
+      } else if (P.type != PH_STAGE2) {
+        double p1, p2;
+        band_tile_products(a, P.k, P.h, P.l, p1, p2);
+        flops += 2.0 * TILE * TILE * TILE * (p1 + p2);
+      }
+    }
+  }
+  LaunchScope ls(kFamSubtree, a.s, flops);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(SIMT_THREADS);
+  cfg.dynamicSmemBytes = sizeof(SubtreeSmem);
+  cfg.stream = a.s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  note(a, cudaLaunchKernelEx(&cfg, k_subtree, A));
 }
 
 static void rec(SolveArgs& a, int k, int l) {
   if (l == k + 1) {
-    leaf(a, k);
+    leaf(a, k, 0);
+    return;
+  }
+  if (l == k + 2) {   // the node (k, k+1, k+2) is applied by its second leaf
+    leaf(a, k, 0);
+    leaf(a, k + 1, 1);
+    return;
+  }
+  if (l - k <= a.subtree_max && a.subtree_grid > 0) {
+    subtree(a, k, l);
     return;
   }
   const int h = (k + l) / 2;
@@ -608,12 +1082,26 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
   a.status = (int*)(ws + sl.off_status);
   a.s = s;
   a.rc = BAKRON_OK;
+  a.la = LeafArgs{a.Mt, a.Nt, m, n, a.X, a.np, a.EtH, a.EtL, a.mp, a.LBH, a.LBL, a.mp,
+                  a.LAH, a.LAL, a.np, scales, zeros, a.G, a.gsz, a.qmax, codes, a.status};
+  a.ba = BandArgs{a.LBH, a.LBL, a.mp, a.EtH, a.EtL, a.mp, a.LAH, a.LAL, a.np,
+                  a.MH, a.ML, a.np, a.X, a.np};
   a.profiling = profiling_on();
   {
     const char* e = getenv("BAKRON_TC_MIN_BAND");
     a.tc_min_band = (e && *e) ? atoi(e) : 16;   // 0 or less: tensor cores off
     const char* f2 = getenv("BAKRON_FUSED_MAX_BAND");
     a.fused_max_band = (f2 && *f2) ? atoi(f2) : 4;
+    const char* f3 = getenv("BAKRON_SUBTREE_MAX");
+    a.subtree_max = (f3 && *f3) ? atoi(f3) : 0;   // 0 or 1: no persistent subtrees
+    if (a.subtree_max > MAX_SUBTREE) a.subtree_max = MAX_SUBTREE;
+    a.subtree_grid = 0;
+    if (a.subtree_max >= 2) {
+      const int cap = subtree_capacity();
+      if (cap < 0) return BAKRON_ERR_CUDA;
+      a.subtree_grid = cap;
+    }
+    a.spin_cycles = spin_cycles_from_env();
     a.tc_ready = false;
     if (a.tc_min_band > 0) {
       a.tco = TcOperands{a.mp, a.np, a.Mt, a.Nt, a.LBH, a.LBL, a.LAH, a.LAL,

@@ -528,15 +528,6 @@ bool make_map(CUtensorMap* map, const float* base, int64_t rows, int64_t cols, i
   return r == CUDA_SUCCESS;
 }
 
-long long spin_cycles_from_env() {
-  const char* e = getenv("BAKRON_SPIN_CYCLES");
-  if (e && *e) {
-    long long v = atoll(e);
-    if (v >= 0) return v;
-  }
-  return 4000000000LL;  // ~2 s at 2 GHz
-}
-
 bool g_attr_done = false;
 std::mutex g_attr_mu;
 
@@ -559,6 +550,15 @@ __global__ void k_split(const float* src, int64_t count, float* hi, float* lo) {
 }
 
 }  // namespace
+
+long long spin_cycles_from_env() {
+  const char* e = getenv("BAKRON_SPIN_CYCLES");
+  if (e && *e) {
+    long long v = atoll(e);
+    if (v >= 0) return v;
+  }
+  return 4000000000LL;  // ~2 s at 2 GHz
+}
 
 bool tc_band_maps(TcMaps& maps, const TcOperands& op) {
   // stage 1: A = L^B (mp x mp), B = E^T (np x mp) in 32-row boxes

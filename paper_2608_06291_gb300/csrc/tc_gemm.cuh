@@ -22,6 +22,10 @@ struct TcMaps {
 
 bool tc_band_maps(TcMaps& maps, const TcOperands& op);
 
+// Bound, in clock64 cycles, of every working device wait (BAKRON_SPIN_CYCLES,
+// default about 2 s): a wait that runs out records BAKRON_ERR_TIMEOUT.
+long long spin_cycles_from_env();
+
 // Stage 1 (M = L^B E on the band [k, h)) or stage 2 (X += M L^A^T on the
 // band [h, l)) of one Alg. 5 node, over 128 x 128 output blocks.
 int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, int h, int l,

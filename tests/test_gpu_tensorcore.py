@@ -1,6 +1,8 @@
 """The tcgen05 3xTF32 band products: the diagnostic GEMM against fp64, and the
 solve with the tensor-core path forced onto every band of width >= 2 (so that
-small, ragged problems exercise the band masks) against the oracle."""
+small, ragged problems exercise the band masks) against the oracle.  These
+tests turn the persistent subtree launches off (BAKRON_SUBTREE_MAX=0), which
+would otherwise take every narrow band of a small problem."""
 import numpy as np
 import pytest
 import torch
@@ -47,12 +49,14 @@ def test_gemm_3xtf32_structured_zeros():
 
 @pytest.mark.parametrize("m,n", [(64, 64), (97, 131), (130, 300), (257, 129), (300, 417)])
 def test_solve_with_tensor_core_bands(m, n, monkeypatch):
+    monkeypatch.setenv("BAKRON_SUBTREE_MAX", "0")
     monkeypatch.setenv("BAKRON_TC_MIN_BAND", "2")
     _assert_parity(_solve_small(m, n, 2000 + m + n, bits=4))
 
 
 @pytest.mark.parametrize("group", [32, 128])
 def test_solve_with_tensor_core_bands_groups(group, monkeypatch):
+    monkeypatch.setenv("BAKRON_SUBTREE_MAX", "0")
     monkeypatch.setenv("BAKRON_TC_MIN_BAND", "3")
     _assert_parity(_solve_small(150, 256, 33 + group, bits=3, group=group))
 
@@ -60,7 +64,7 @@ def test_solve_with_tensor_core_bands_groups(group, monkeypatch):
 def test_tensor_core_and_simt_paths_agree(monkeypatch):
     """Same inputs, band products on tcgen05 vs on CUDA cores: identical codes
     (the difference is ~1e-6 of an update, far inside the tie band)."""
-    W = None
+    monkeypatch.setenv("BAKRON_SUBTREE_MAX", "0")
     monkeypatch.setenv("BAKRON_TC_MIN_BAND", "0")
     a = _solve_small(400, 350, 91, bits=4)
     monkeypatch.setenv("BAKRON_TC_MIN_BAND", "2")
@@ -73,6 +77,7 @@ def test_tensor_core_and_simt_paths_agree(monkeypatch):
 def test_bounded_waits_report_timeout_and_recover(monkeypatch):
     """A zero wait budget makes the tensor-core waits run out: the solve returns
     BAKRON_ERR_TIMEOUT (no hang, no fault) and the next solve is correct."""
+    monkeypatch.setenv("BAKRON_SUBTREE_MAX", "0")
     monkeypatch.setenv("BAKRON_TC_MIN_BAND", "2")
     monkeypatch.setenv("BAKRON_SPIN_CYCLES", "0")
     with pytest.raises(P.BakronError) as e:
@@ -86,6 +91,7 @@ def test_bounded_waits_report_timeout_and_recover(monkeypatch):
 def test_solve_with_fused_narrow_bands(fused, monkeypatch):
     """Narrow Alg. 5 nodes with both stages fused in one launch (all widths up
     to 64 when forced) give the oracle's codes."""
+    monkeypatch.setenv("BAKRON_SUBTREE_MAX", "0")
     monkeypatch.setenv("BAKRON_FUSED_MAX_BAND", fused)
     monkeypatch.setenv("BAKRON_TC_MIN_BAND", "0")
     _assert_parity(_solve_small(160, 230, 404, bits=4))
