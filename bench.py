@@ -70,7 +70,7 @@ def _csrc_hash():
 def _traffic(family):
     """DRAM bytes per step of a kernel family from the committed ncu summary,
     or None when the kernels changed since it was taken."""
-    p = os.path.join(ROOT, "profiles", "traffic.json")
+    p = os.path.join(ROOT, "profiles", "traffic.txt")
     try:
         t = json.load(open(p))
     except Exception:
