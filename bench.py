@@ -230,6 +230,13 @@ def run_gpu(args):
     def eager_step():
         P.bakron_solve(W, fac, cfg.bits, cfg.group, workspace=work, sync=False, out=out)
 
+    # the library's own schedule autotune for this shape (outside the timed region)
+    sched = P.bakron_get_tuning(m, n)
+    sched["autotuned"] = False
+    if not args.no_autotune:
+        best = P.bakron_autotune(W, fac, cfg.bits, cfg.group, workspace=work)
+        sched = {"tc_min_band": best["tc_min_band"], "fused_max_band": best["fused_max_band"],
+                 "autotuned": True}
     for _ in range(max(3, args.warmup)):
         flush.fill_(1)
         eager_step()
@@ -400,7 +407,8 @@ def run_gpu(args):
             "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": vs, "dtype": "f32", "data": "synthetic",
             "config": dict(_config_dict(cfg), parallelism=f"replicas x{ws_n}",
-                           launch="cuda graph replay" if graph is not None else "eager"),
+                           launch="cuda graph replay" if graph is not None else "eager",
+                           schedule=sched),
             "prepare_ms": prepare_ms, "roofline": roof, "cpu_baseline": cpu_base, "e2e": e2e,
             "gpu_launches": launches, "clocks": clocks, "solve_roofline": solve_roof,
         }
@@ -422,6 +430,8 @@ def main():
     ap.add_argument("--ref-block", type=int, default=256,
                     help="side of the top-left block each reference-arm step solves")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-autotune", action="store_true",
+                    help="use the library's default schedule thresholds")
     ap.add_argument("--no-graph", action="store_true",
                     help="launch each solve's kernels eagerly instead of replaying a CUDA graph")
     args = ap.parse_args()

@@ -5,13 +5,14 @@
 #include <stdlib.h>
 
 #include "common.cuh"
+#include "tune.cuh"
 
 namespace bakron {
 int prepare_impl(const float* A, const float* B, int m, int n, float damp, void* factors,
                  void* workspace, cudaStream_t s);
 int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int bits,
                int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s);
+               void* workspace, cudaStream_t s, const Tuning* force);
 
 // Largest side accepted.  Keeps every index product inside int64 and every
 // grid dimension inside CUDA's limits (mp / 32 tiles per side).
@@ -121,7 +122,7 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw, const voi
   if (workspace_bytes < SolveLayout(m, n).bytes) return BAKRON_ERR_WORKSPACE;
   cudaStream_t s = (cudaStream_t)stream;
   int rc = solve_impl(W, wdtype, m, n, ldw, factors, bits, group_size, codes, scales, zeros,
-                      prerounding, workspace, s);
+                      prerounding, workspace, s, nullptr);
   if (rc != BAKRON_OK || !sync) return rc;
   return bakron_read_status(workspace, stream);
 }

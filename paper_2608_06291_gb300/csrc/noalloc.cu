@@ -7,11 +7,12 @@
 #include <unordered_map>
 
 #include "common.cuh"
+#include "tune.cuh"
 
 namespace bakron {
 int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int bits,
                int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s);
+               void* workspace, cudaStream_t s, const Tuning* force);
 
 // The scratch.  Every GPU that loads the library holds it until the process
 // exits.  In host code this name is only a stand-in for the device symbol:
@@ -59,7 +60,7 @@ extern "C" int bakron_solve_noalloc(const void* W, int wdtype, int m, int n, int
   if (noalloc_scratch(&scratch) != cudaSuccess) return BAKRON_ERR_CUDA;
   cudaStream_t s = (cudaStream_t)stream;
   int rc = solve_impl(W, wdtype, m, n, ldw, factors, bits, group_size, codes, scales, zeros,
-                      prerounding, scratch, s);
+                      prerounding, scratch, s, nullptr);
   if (rc != BAKRON_OK || !sync) return rc;
   return bakron_read_status(scratch, stream);
 }

@@ -20,6 +20,7 @@
 #include "common.cuh"
 #include "profile.cuh"
 #include "tc_gemm.cuh"
+#include "tune.cuh"
 #include <stdlib.h>
 
 #include <mutex>
@@ -1055,9 +1056,10 @@ static void rec(SolveArgs& a, int k, int l) {
   rec(a, h, l);
 }
 
+// `force`: thresholds to use instead of tuning_for(m, n) (the autotuner's candidates).
 int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int bits,
                int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s) {
+               void* workspace, cudaStream_t s, const Tuning* force) {
   FactorLayout fl(m, n);
   SolveLayout sl(m, n);
   char* ws = (char*)workspace;
@@ -1088,12 +1090,10 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
                   a.MH, a.ML, a.np, a.X, a.np};
   a.profiling = profiling_on();
   {
-    const char* e = getenv("BAKRON_TC_MIN_BAND");
-    a.tc_min_band = (e && *e) ? atoi(e) : 16;   // 0 or less: tensor cores off
-    const char* f2 = getenv("BAKRON_FUSED_MAX_BAND");
-    a.fused_max_band = (f2 && *f2) ? atoi(f2) : 4;
-    const char* f3 = getenv("BAKRON_SUBTREE_MAX");
-    a.subtree_max = (f3 && *f3) ? atoi(f3) : 0;   // 0 or 1: no persistent subtrees
+    const Tuning tu = force ? *force : tuning_for(m, n);
+    a.tc_min_band = tu.tc_min_band;         // 0 or less: tensor cores off
+    a.fused_max_band = tu.fused_max_band;
+    a.subtree_max = tu.subtree_max;         // 0 or 1: no persistent subtrees
     if (a.subtree_max > MAX_SUBTREE) a.subtree_max = MAX_SUBTREE;
     a.subtree_grid = 0;
     if (a.subtree_max >= 2) {
