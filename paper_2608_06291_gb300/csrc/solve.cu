@@ -539,15 +539,18 @@ constexpr int SIMT_PER = TILE * TILE / SIMT_THREADS;   // 4 elements per thread 
 
 // One operand tile, element e = t + SIMT_THREADS * k of the 32 x 32 block at
 // (row0, col0) of a hi/lo plane pair with leading dimension ld.
+// hi and lo stay separate until the tile is stored, so nothing waits on the
+// loads before the next tile product has been issued.
 struct TileRegs {
-  float v[SIMT_PER];
+  float h[SIMT_PER], l[SIMT_PER];
   __device__ void load(const float* __restrict__ hi, const float* __restrict__ lo, int64_t ld,
                        int64_t row0, int64_t col0, int t) {
 #pragma unroll
     for (int k = 0; k < SIMT_PER; ++k) {
       const int e = t + SIMT_THREADS * k;
       const int64_t o = (row0 + e / TILE) * ld + col0 + e % TILE;
-      v[k] = __ldcg(hi + o) + __ldcg(lo + o);   // L2: coherent within a persistent kernel
+      h[k] = __ldcg(hi + o);   // L2: coherent within a persistent kernel
+      l[k] = __ldcg(lo + o);
     }
   }
   // as stored (S[r][c] = tile[r][c]) or transposed (S[c][r] = tile[r][c])
@@ -555,8 +558,9 @@ struct TileRegs {
 #pragma unroll
     for (int k = 0; k < SIMT_PER; ++k) {
       const int e = t + SIMT_THREADS * k;
-      if (transpose) S[e % TILE][e / TILE] = v[k];
-      else S[e / TILE][e % TILE] = v[k];
+      const float v = h[k] + l[k];
+      if (transpose) S[e % TILE][e / TILE] = v;
+      else S[e / TILE][e % TILE] = v;
     }
   }
 };
@@ -614,20 +618,25 @@ __device__ __forceinline__ void band1_unit(const Band& bd, const BandArgs& a, in
   const int i_lo = max(0, bd.k - Jp), i_hi = min(I, bd.h - 1 - Jp);
   const int t = threadIdx.x, tr = t / 8, tc = (t % 8) * 4;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  TileRegs ra, rb;
-  // B[kk][col] = E[I'*T + kk][J'*T + col] = E^T[J'*T + col][I'*T + kk]
-  ra.load(a.LBH, a.LBL, a.ldb, (int64_t)I * TILE, (int64_t)i_lo * TILE, t);
-  rb.load(a.EtH, a.EtL, a.ldt, (int64_t)Jp * TILE, (int64_t)i_lo * TILE, t);
-  for (int Ip = i_lo; Ip <= i_hi; ++Ip) {
-    ra.store(S.As, false, t);
-    rb.store(S.Bs, true, t);
-    __syncthreads();
-    if (Ip < i_hi) {
-      ra.load(a.LBH, a.LBL, a.ldb, (int64_t)I * TILE, (int64_t)(Ip + 1) * TILE, t);
-      rb.load(a.EtH, a.EtL, a.ldt, (int64_t)Jp * TILE, (int64_t)(Ip + 1) * TILE, t);
+  // two tile pairs in flight: B[kk][col] = E[I'*T + kk][J'*T + col] = E^T[J'*T + col][I'*T + kk]
+  TileRegs ra[2], rb[2];
+  auto fetch = [&](int j, int Ip) {
+    ra[j].load(a.LBH, a.LBL, a.ldb, (int64_t)I * TILE, (int64_t)Ip * TILE, t);
+    rb[j].load(a.EtH, a.EtL, a.ldt, (int64_t)Jp * TILE, (int64_t)Ip * TILE, t);
+  };
+  fetch(0, i_lo);
+  if (i_lo + 1 <= i_hi) fetch(1, i_lo + 1);
+  for (int Ip = i_lo; Ip <= i_hi; Ip += 2) {
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      if (Ip + j > i_hi) break;
+      ra[j].store(S.As, false, t);
+      rb[j].store(S.Bs, true, t);
+      __syncthreads();
+      if (Ip + j + 2 <= i_hi) fetch(j, Ip + j + 2);
+      tile_mac(S.As, S.Bs, tr, tc, acc);
+      __syncthreads();
     }
-    tile_mac(S.As, S.Bs, tr, tc, acc);
-    __syncthreads();
   }
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
@@ -644,20 +653,25 @@ __device__ __forceinline__ void band2_unit(const Band& bd, const BandArgs& a, in
   const int j_lo = max(0, bd.k - I), j_hi = min(J, bd.h - 1);
   const int t = threadIdx.x, tr = t / 8, tc = (t % 8) * 4;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  TileRegs ra, rb;
-  // Bs[t][c] = L^A[J*T + c][J'*T + t]
-  ra.load(a.MH, a.ML, a.ldm, (int64_t)I * TILE, (int64_t)j_lo * TILE, t);
-  rb.load(a.LAH, a.LAL, a.lda, (int64_t)J * TILE, (int64_t)j_lo * TILE, t);
-  for (int Jp = j_lo; Jp <= j_hi; ++Jp) {
-    ra.store(S.As, false, t);
-    rb.store(S.Bs, true, t);
-    __syncthreads();
-    if (Jp < j_hi) {
-      ra.load(a.MH, a.ML, a.ldm, (int64_t)I * TILE, (int64_t)(Jp + 1) * TILE, t);
-      rb.load(a.LAH, a.LAL, a.lda, (int64_t)J * TILE, (int64_t)(Jp + 1) * TILE, t);
+  // two tile pairs in flight: Bs[t][c] = L^A[J*T + c][J'*T + t]
+  TileRegs ra[2], rb[2];
+  auto fetch = [&](int j, int Jp) {
+    ra[j].load(a.MH, a.ML, a.ldm, (int64_t)I * TILE, (int64_t)Jp * TILE, t);
+    rb[j].load(a.LAH, a.LAL, a.lda, (int64_t)J * TILE, (int64_t)Jp * TILE, t);
+  };
+  fetch(0, j_lo);
+  if (j_lo + 1 <= j_hi) fetch(1, j_lo + 1);
+  for (int Jp = j_lo; Jp <= j_hi; Jp += 2) {
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      if (Jp + j > j_hi) break;
+      ra[j].store(S.As, false, t);
+      rb[j].store(S.Bs, true, t);
+      __syncthreads();
+      if (Jp + j + 2 <= j_hi) fetch(j, Jp + j + 2);
+      tile_mac(S.As, S.Bs, tr, tc, acc);
+      __syncthreads();
     }
-    tile_mac(S.As, S.Bs, tr, tc, acc);
-    __syncthreads();
   }
 #pragma unroll
   for (int u = 0; u < 4; ++u) {

@@ -378,30 +378,34 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
     // number of MMAs summed in place; restarting every 32 of K bounds it.
     if (lane == 0) {
       const uint32_t idesc = idesc_tf32(BM, BN);
+      const uint64_t desc0 = smem_desc(smem_u32(smem));   // stage 0, A hi, K step 0
       for (int i = 0; i < nk; ++i) {
         const int s = i % STAGES;
         const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
         const int a = i % NACC;
-        bool ok = mbar_wait(&full[s], ph, P.spin_cycles);
         // accumulator a was last used by stage i - NACC: wait until it was read out
-        if (ok && i >= NACC)
-          ok = mbar_wait(&accE[a], (uint32_t)(i / NACC - 1) & 1u, P.spin_cycles);
-        if (!ok || *abort_flag) {
+        // (the producer's and the epilogue's aborts surface here as time-outs)
+        const bool ok = mbar_wait(&full[s], ph, P.spin_cycles) &&
+                        (i < NACC ||
+                         mbar_wait(&accE[a], (uint32_t)(i / NACC - 1) & 1u, P.spin_cycles));
+        if (!ok) {
           raise_status(P.status, BAKRON_ERR_TIMEOUT);
           *abort_flag = 1;
           break;
         }
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const uint32_t st = smem_u32(smem + s * STAGE_BYTES);
-        const uint32_t a_hi = st, a_lo = st + TILE_BYTES, b_hi = st + 2 * TILE_BYTES,
-                       b_lo = st + 3 * TILE_BYTES;
+        // descriptors of this stage's four planes; K steps of 32 bytes add 2 to
+        // the start-address field (16-byte units, no carry within a stage)
+        const uint64_t dah = desc0 + (uint64_t)((s * STAGE_BYTES) >> 4);
+        const uint64_t dal = dah + (TILE_BYTES >> 4), dbh = dah + (2 * TILE_BYTES >> 4),
+                       dbl = dah + (3 * TILE_BYTES >> 4);
         const uint32_t d = tmem + (uint32_t)(a * BN);
 #pragma unroll
         for (int kk = 0; kk < BK / 8; ++kk) {
-          const uint32_t off = kk * 32;   // 8 tf32 = 32 bytes along K inside the swizzle row
-          mma_tf32(d, smem_desc(a_hi + off), smem_desc(b_hi + off), idesc, kk > 0 ? 1u : 0u);
-          mma_tf32(d, smem_desc(a_hi + off), smem_desc(b_lo + off), idesc, 1u);
-          mma_tf32(d, smem_desc(a_lo + off), smem_desc(b_hi + off), idesc, 1u);
+          const uint64_t o = (uint64_t)(2 * kk);   // 8 tf32 = 32 bytes along K inside the swizzle row
+          mma_tf32(d, dah + o, dbh + o, idesc, kk > 0 ? 1u : 0u);
+          mma_tf32(d, dah + o, dbl + o, idesc, 1u);
+          mma_tf32(d, dal + o, dbh + o, idesc, 1u);
         }
         mma_commit(&empty[s]);    // frees the smem stage when these MMAs are done
         mma_commit(&accF[a]);     // hands the stage's sum to the epilogue
