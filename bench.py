@@ -358,6 +358,17 @@ def run_gpu(args):
     solve_roof = {"fp32_effective_tflops": p_eff, "f_alg_flops": f_alg,
                   "roofline_ms": 1e3 * t_roof, "frac": 1e3 * t_roof / ms,
                   "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained x 1.1/2.25 / 3"}
+    # context: the library's own measurement of the instruction it issues
+    # (tcgen05 kind::tf32, 128 x 128 x 8, operands resident, every SM)
+    try:
+        mr = P.bakron_diag_mma_rate(2000)
+        t_roof_mma = f_alg / (mr["fp32_effective_tflops"] * 1e12) + 17.0 * m * n / (hbm * 1e9)
+        solve_roof["measured_tf32_mma"] = {
+            "tf32_tflops": mr["tf32_tflops"], "cycles_per_mma": mr["cycles_per_mma"],
+            "fp32_effective_tflops": mr["fp32_effective_tflops"],
+            "roofline_ms": 1e3 * t_roof_mma, "frac": 1e3 * t_roof_mma / ms}
+    except Exception as exc:   # diagnostic only
+        solve_roof["measured_tf32_mma"] = {"error": str(exc)}
 
     # end to end: pinned host W in, codes/scales/zeros out, inside the timed region
     Wh = W.cpu().pin_memory()

@@ -235,6 +235,19 @@ int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C, int M,
                             int N, int K, void* workspace,
                             size_t workspace_bytes, void* stream);
 
+/*
+ * Diagnostic (no counterpart in the paper): the measured rate of the tensor
+ * core instruction the band products issue, tcgen05.mma kind::tf32 with a
+ * 128 x 128 accumulator and K = 8, from operands resident in shared memory,
+ * one CTA per SM, `stages` x 4 back-to-back MMAs each (timed with CUDA events
+ * after a warm-up launch).  *tflops receives the whole-device tf32 rate
+ * (2 * 128 * 128 * 8 flops per MMA), *cycles_per_mma (may be NULL) one SM's
+ * cycles per MMA.  The FP32-effective rate of the 3xTF32 products is a third
+ * of *tflops.  workspace >= 256 + 8 * (number of SMs) bytes.  Synchronous.
+ */
+int bakron_diag_mma_rate(int stages, void* workspace, size_t workspace_bytes,
+                         double* tflops, double* cycles_per_mma, void* stream);
+
 /* Static description of a status code. */
 const char* bakron_strerror(int status);
 

@@ -5,6 +5,7 @@ C ABI in include/bakron.h); this package is its build script and a thin
 ctypes binding with the same entry-point names.
 """
 from .bakron import (BakronError, Factors, alloc_workspace, bakron_diag_gemm_tf32x3,  # noqa: F401
+                     bakron_diag_mma_rate,
                      bakron_autotune, bakron_autotune_clear, bakron_get_factors,
                      bakron_get_tuning,
                      bakron_last_launches, bakron_prepare, bakron_profile_enable,

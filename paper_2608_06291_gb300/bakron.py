@@ -73,6 +73,9 @@ def lib() -> ctypes.CDLL:
     L.bakron_get_tuning.restype = i32
     L.bakron_autotune_clear.argtypes = []
     L.bakron_autotune_clear.restype = None
+    L.bakron_diag_mma_rate.argtypes = [i32, vp, sz, ctypes.POINTER(ctypes.c_double),
+                                       ctypes.POINTER(ctypes.c_double), vp]
+    L.bakron_diag_mma_rate.restype = i32
     L.bakron_strerror.argtypes = [i32]
     L.bakron_strerror.restype = ctypes.c_char_p
     _lib = L
@@ -311,3 +314,15 @@ def dequantize(codes, scales, zeros):
     s = scales.repeat_interleave(g, dim=1)
     z = zeros.repeat_interleave(g, dim=1)
     return s * (codes.float() - z)
+
+
+def bakron_diag_mma_rate(stages: int = 2000, stream=None) -> dict:
+    """Measured tcgen05 kind::tf32 MMA rate of the whole device (diagnostic).
+    Returns {"tf32_tflops", "cycles_per_mma", "fp32_effective_tflops"}."""
+    ws = torch.empty(256 + 8 * 1024, dtype=torch.uint8, device="cuda")
+    tf, cyc = ctypes.c_double(0.0), ctypes.c_double(0.0)
+    _check(lib().bakron_diag_mma_rate(int(stages), _ptr(ws), ws.numel(), ctypes.byref(tf),
+                                      ctypes.byref(cyc), _stream(stream)),
+           "bakron_diag_mma_rate")
+    return {"tf32_tflops": tf.value, "cycles_per_mma": cyc.value,
+            "fp32_effective_tflops": tf.value / 3.0}

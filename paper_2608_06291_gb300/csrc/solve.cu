@@ -273,21 +273,26 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, bool 
     if (e < TILE * TILE) xv[k] = __ldcg(a.X + (r0 + e / TILE) * a.ldx + c0 + e % TILE);
   }
   if (has_left || has_up) {
-    // errors of the neighbours on anti-diagonal K-1, k-major as E^T stores them
+    // errors of the neighbours on anti-diagonal K-1, k-major as E^T stores
+    // them: every load issued before any is used
+    static_assert(LEAF_PER_THREAD * LEAF_THREADS == TILE * TILE, "whole tile per pass");
+    float lh[LEAF_PER_THREAD], ll[LEAF_PER_THREAD], uh[LEAF_PER_THREAD], ul[LEAF_PER_THREAD];
 #pragma unroll
     for (int k = 0; k < LEAF_PER_THREAD; ++k) {
       const int e = t + k * LEAF_THREADS;
-      if (e < TILE * TILE) {
-        const int j = e / TILE, i = e % TILE;
-        if (has_left) {
-          const int64_t o = (c0 - TILE + j) * a.ldt + r0 + i;
-          S.u.pro.EL[j][i] = __ldcg(a.EtH + o) + __ldcg(a.EtL + o);
-        }
-        if (has_up) {
-          const int64_t o = (c0 + j) * a.ldt + r0 - TILE + i;
-          S.u.pro.EU[j][i] = __ldcg(a.EtH + o) + __ldcg(a.EtL + o);
-        }
-      }
+      const int j = e / TILE, i = e % TILE;
+      const int64_t ol = (c0 - TILE + j) * a.ldt + r0 + i, ou = (c0 + j) * a.ldt + r0 - TILE + i;
+      lh[k] = has_left ? __ldcg(a.EtH + ol) : 0.f;
+      ll[k] = has_left ? __ldcg(a.EtL + ol) : 0.f;
+      uh[k] = has_up ? __ldcg(a.EtH + ou) : 0.f;
+      ul[k] = has_up ? __ldcg(a.EtL + ou) : 0.f;
+    }
+#pragma unroll
+    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+      const int e = t + k * LEAF_THREADS;
+      const int j = e / TILE, i = e % TILE;
+      S.u.pro.EL[j][i] = lh[k] + ll[k];
+      S.u.pro.EU[j][i] = uh[k] + ul[k];
     }
   }
   leaf_sync();   // LBs, LAs and the absorbed operands complete

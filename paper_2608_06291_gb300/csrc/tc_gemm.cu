@@ -216,7 +216,9 @@ __host__ __device__ inline bool band_row_span(int mode, int k, int h, int l, int
 
 // Returns false if the block has no work at all (beyond its row's span).
 __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
-  b.rb = P.row0 + blockIdx.y;
+  // the blocks with the longest K ranges first (they sit at high rows, and
+  // in stage 2 at high columns): less of a tail when the grid runs in waves
+  b.rb = P.row0 + (P.mode == MODE_DENSE ? blockIdx.y : gridDim.y - 1 - blockIdx.y);
   if (P.mode == MODE_DENSE) {
     b.cb = blockIdx.x;
     b.k0 = 0;
@@ -225,8 +227,8 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
   }
   int cb_lo, cb_hi;
   if (!band_row_span(P.mode, P.k, P.h, P.l, P.Mt, P.Nt, b.rb, cb_lo, cb_hi)) return false;
-  b.cb = cb_lo + blockIdx.x;
-  if (b.cb > cb_hi) return false;
+  b.cb = P.mode == MODE_STAGE2 ? cb_hi - (int)blockIdx.x : cb_lo + (int)blockIdx.x;
+  if (b.cb > cb_hi || b.cb < cb_lo) return false;
   const int I0 = 4 * b.rb, Ilast = min(I0 + 3, P.Mt - 1);
   const int J0 = 4 * b.cb;
   if (P.mode == MODE_STAGE1) {

@@ -95,3 +95,12 @@ def test_solve_with_fused_narrow_bands(fused, monkeypatch):
     monkeypatch.setenv("BAKRON_FUSED_MAX_BAND", fused)
     monkeypatch.setenv("BAKRON_TC_MIN_BAND", "0")
     _assert_parity(_solve_small(160, 230, 404, bits=4))
+
+
+def test_mma_rate_diagnostic():
+    """The measured tcgen05 kind::tf32 rate is a plausible whole-GPU figure
+    (GB300 nominal dense tf32: 1.1 PFLOP/s; one MMA of 128 x 128 x 8 per SM
+    takes at least 32 cycles)."""
+    r = P.bakron_diag_mma_rate(500)
+    assert 100.0 < r["tf32_tflops"] < 3000.0, r
+    assert r["cycles_per_mma"] >= 32.0, r
