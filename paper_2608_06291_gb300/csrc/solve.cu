@@ -219,47 +219,60 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, bool 
   const int t = threadIdx.x, w = t >> 5, lane = t & 31;
   const int64_t r0 = (int64_t)I * TILE, c0 = (int64_t)J * TILE;
   const bool has_left = absorb && J > 0, has_up = absorb && I > 0;
-  if (has_left || has_up) {
-    // sub-diagonal factor blocks, transposed to k-major (read-only: before the wait)
+  // Factor blocks and the grid (read-only during the solve; the grid written
+  // by the solve's first kernel, more than one kernel ago), loaded before
+  // waiting for the previous kernel.  Each batch issues all its loads before
+  // any is used, so their latencies overlap.
+  {
+    float bh[LEAF_PER_THREAD], bl[LEAF_PER_THREAD], ah[LEAF_PER_THREAD], al[LEAF_PER_THREAD];
 #pragma unroll
     for (int k = 0; k < LEAF_PER_THREAD; ++k) {
       const int e = t + k * LEAF_THREADS;
-      if (e < TILE * TILE) {
-        const int p = e / TILE, c = e % TILE;
-        if (has_left) {
-          const int64_t o = (c0 + p) * a.lda + c0 - TILE + c;
-          S.u.pro.LAt[c][p] = a.LAH[o] + a.LAL[o];
-        }
-        if (has_up) {
-          const int64_t o = (r0 + p) * a.ldb + r0 - TILE + c;
-          S.u.pro.LBt[c][p] = a.LBH[o] + a.LBL[o];
-        }
-      }
-    }
-  }
-  float lbv[LEAF_PER_THREAD], lav[LEAF_PER_THREAD], scv[LEAF_PER_THREAD], zv[LEAF_PER_THREAD];
-#pragma unroll
-  for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-    const int e = t + k * LEAF_THREADS;
-    if (e < TILE * TILE) {
       const int p = e / TILE, c = e % TILE;
       const int64_t ob = (r0 + p) * a.ldb + r0 + c, oa = (c0 + p) * a.lda + c0 + c;
-      lbv[k] = a.LBH[ob] + a.LBL[ob];
-      lav[k] = a.LAH[oa] + a.LAL[oa];
-      const bool real = (r0 + p) < a.m && (c0 + c) < a.n;
-      const int64_t og = (r0 + p) * a.G + (c0 + c) / a.gsz;
-      scv[k] = real ? a.scales[og] : 1.f;
-      zv[k] = real ? a.zeros[og] : 0.f;
+      bh[k] = a.LBH[ob];
+      bl[k] = a.LBL[ob];
+      ah[k] = a.LAH[oa];
+      al[k] = a.LAL[oa];
+    }
+#pragma unroll
+    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+      const int e = t + k * LEAF_THREADS;
+      const int p = e / TILE, c = e % TILE;
+      S.LBs[p][c] = bh[k] + bl[k];
+      S.LAs[p][c] = ah[k] + al[k];
     }
   }
+  if (has_left || has_up) {
+    // sub-diagonal factor blocks, transposed to k-major
+    float bh[LEAF_PER_THREAD], bl[LEAF_PER_THREAD], ah[LEAF_PER_THREAD], al[LEAF_PER_THREAD];
+#pragma unroll
+    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+      const int e = t + k * LEAF_THREADS;
+      const int p = e / TILE, c = e % TILE;
+      const int64_t oa = (c0 + p) * a.lda + c0 - TILE + c, ob = (r0 + p) * a.ldb + r0 - TILE + c;
+      ah[k] = has_left ? a.LAH[oa] : 0.f;
+      al[k] = has_left ? a.LAL[oa] : 0.f;
+      bh[k] = has_up ? a.LBH[ob] : 0.f;
+      bl[k] = has_up ? a.LBL[ob] : 0.f;
+    }
+#pragma unroll
+    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+      const int e = t + k * LEAF_THREADS;
+      const int p = e / TILE, c = e % TILE;
+      S.u.pro.LAt[c][p] = ah[k] + al[k];
+      S.u.pro.LBt[c][p] = bh[k] + bl[k];
+    }
+  }
+  float scv[LEAF_PER_THREAD], zv[LEAF_PER_THREAD];
 #pragma unroll
   for (int k = 0; k < LEAF_PER_THREAD; ++k) {
     const int e = t + k * LEAF_THREADS;
-    if (e < TILE * TILE) {
-      const int p = e / TILE, c = e % TILE;
-      S.LBs[p][c] = lbv[k];
-      S.LAs[p][c] = lav[k];
-    }
+    const int p = e / TILE, c = e % TILE;
+    const bool real = (r0 + p) < a.m && (c0 + c) < a.n;
+    const int64_t og = real ? (r0 + p) * a.G + (c0 + c) / a.gsz : 0;
+    scv[k] = real ? a.scales[og] : 1.f;
+    zv[k] = real ? a.zeros[og] : 0.f;
   }
   if (t < TILE * (36 - TILE)) S.LBs[t / (36 - TILE)][TILE + t % (36 - TILE)] = 0.f;  // padding rows
   if (PDL) {
