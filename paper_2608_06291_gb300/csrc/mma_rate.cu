@@ -103,7 +103,7 @@ using namespace bakron;
 extern "C" int bakron_diag_mma_rate(int stages, void* workspace, size_t workspace_bytes,
                                     double* tflops, double* cycles_per_mma, void* stream) {
   if (stages < 1 || stages > (1 << 20) || !workspace || !tflops) return BAKRON_ERR_INVALID_ARG;
-  int dev = 0, sms = 0, khz = 0;
+  int dev = 0, sms = 0;
   BK_CUDA_OK(cudaGetDevice(&dev));
   BK_CUDA_OK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
   if (workspace_bytes < 256 + sizeof(long long) * (size_t)sms) return BAKRON_ERR_WORKSPACE;
@@ -139,6 +139,5 @@ extern "C" int bakron_diag_mma_rate(int stages, void* workspace, size_t workspac
   const double mmas = 4.0 * stages;
   *tflops = 2.0 * RM * RN * 8 * mmas * sms / (ms * 1e-3) / 1e12;
   if (cycles_per_mma) *cycles_per_mma = (double)c0 / mmas;
-  (void)khz;
   return BAKRON_OK;
 }

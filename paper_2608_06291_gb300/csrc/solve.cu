@@ -145,6 +145,22 @@ struct LeafArgs {
 
 constexpr int KM = 36;   // row stride of k-major product operands: float4 rows
 
+// A leaf absorbs the errors of at most this many earlier anti-diagonals of
+// its block (Alg. 5 ranges of up to LEAF_WINDOW + 1 anti-diagonals are run
+// as such blocks of leaves), needing the E tiles (I - dp, J - g) with
+// 1 <= dp + g <= LEAF_WINDOW.
+constexpr int LEAF_WINDOW = 3;
+constexpr int LEAF_WINDOW_TILES = (LEAF_WINDOW + 1) * (LEAF_WINDOW + 2) / 2 - 1;
+
+// Slot of E tile (I - dp, J - g) among a window-P leaf's tiles: row I first
+// (g = 1..P), then rows I - 1, I - 2, ... (g = 0..P - dp).
+__host__ __device__ constexpr int window_slot(int P, int dp, int g) {
+  return dp == 0 ? g - 1 : P + (dp - 1) * P - (dp - 1) * (dp - 2) / 2 + g;
+}
+
+// 32^3 products a window-P leaf forms before its wavefront (T1, the N_dp, U).
+__host__ __device__ constexpr int window_products(int P) { return 2 * P + P * (P + 1) / 2; }
+
 struct LeafSmem {
   float Xs[TILE][TILE];                   // W after inbound updates
   __align__(16) float LBs[TILE][36];      // stride 36: conflict-free float4 row reads
@@ -155,11 +171,11 @@ struct LeafSmem {
   float4 Lsub[TILE];                              // (L^B[p][p-1], L^B[p][p-2], L^B[p][p-3], 0)
   union {
     struct {   // prologue of an absorbing leaf: k-major product operands
-      __align__(16) float EL[TILE][KM];   // EL[j][i] = E[I, J-1][i][j]; later U[p][q]
-      __align__(16) float EU[TILE][KM];   // EU[j][i] = E[I-1, J][i][j]
-      __align__(16) float LAt[TILE][KM];  // LAt[j][q] = L^A[J, J-1][q][j]
-      __align__(16) float LBt[TILE][KM];  // LBt[i][p] = L^B[I, I-1][p][i]
-      __align__(16) float T2[TILE][KM];   // T2[i][q] = (E[I-1, J] L^A[J, J]^T)[i][q]
+      // E[I - dp, J - g] for the window's (dp, g), Et[.][j][i] = E[..][i][j];
+      // later the N_dp and U of the second round
+      __align__(16) float Et[LEAF_WINDOW_TILES][TILE][KM];
+      __align__(16) float LAt[LEAF_WINDOW][TILE][KM];   // LAt[g-1][j][q] = L^A[J, J-g][q][j]
+      __align__(16) float LBt[LEAF_WINDOW][TILE][KM];   // LBt[dp-1][i][p] = L^B[I, I-dp][p][i]
     } pro;
     struct {   // the wavefront
       union {
@@ -201,67 +217,104 @@ __device__ __forceinline__ void leaf_sync() {
   asm volatile("bar.sync 1, %0;" ::"n"(LEAF_THREADS) : "memory");
 }
 
+// Loads up to NT 32 x 32 tiles of hi/lo plane pairs into shared memory as
+// hi + lo, every load issued before the first sum.  Tile s is the block at
+// element offset base[s] of planes (hi[s], lo[s]) with row stride ld[s];
+// a tile that is not valid becomes zeros.  Element (r, c) goes to
+// dst[s][c * KM + r] (transpose) or dst[s][r * KM + c]; a null dst[s] is
+// skipped.  COHERENT: L2 loads (data written by earlier kernels or phases of
+// the solve).
+template <int NT, bool COHERENT>
+__device__ __forceinline__ void load_tiles(const float* const (&hi)[NT], const float* const (&lo)[NT],
+                                           const int64_t (&base)[NT], const int64_t (&ld)[NT],
+                                           const bool (&valid)[NT], float* const (&dst)[NT],
+                                           bool transpose, int t) {
+  float h[NT][LEAF_PER_THREAD], l[NT][LEAF_PER_THREAD];
+#pragma unroll
+  for (int s = 0; s < NT; ++s) {
+#pragma unroll
+    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+      const int e = t + k * LEAF_THREADS;
+      const int64_t o = base[s] + (int64_t)(e / TILE) * ld[s] + e % TILE;
+      h[s][k] = valid[s] ? (COHERENT ? __ldcg(hi[s] + o) : hi[s][o]) : 0.f;
+      l[s][k] = valid[s] ? (COHERENT ? __ldcg(lo[s] + o) : lo[s][o]) : 0.f;
+    }
+  }
+#pragma unroll
+  for (int s = 0; s < NT; ++s) {
+    if (dst[s] == nullptr) continue;
+#pragma unroll
+    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+      const int e = t + k * LEAF_THREADS;
+      const int r = e / TILE, c = e % TILE;
+      dst[s][transpose ? c * KM + r : r * KM + c] = h[s][k] + l[s][k];
+    }
+  }
+}
+
 // Rounds tile (I, J); run by threads 0 .. LEAF_THREADS-1 of the CTA.  With
 // PDL, the factor blocks and the grid (read-only during the solve, the grid
 // written by the solve's first kernel, more than one kernel ago) are loaded
 // before waiting for the previous kernel.
 //
-// An absorbing leaf also applies the Alg. 5 node (K-1, K, K+1) whose band
-// carries the errors of anti-diagonal K-1 into this one: for tile (I, J) that
-// is  L^B[I,I] E[I,J-1] L^A[J,J-1]^T + L^B[I,I-1] E[I-1,J] L^A[J,J]^T.  The
-// first term enters the wavefront as the initial value of G (which the
-// wavefront multiplies by L^B[I,I] anyway): T1 = E[I,J-1] L^A[J,J-1]^T.  The
-// second, U = L^B[I,I-1] (E[I-1,J] L^A[J,J]^T), is added to X before the
-// wavefront.
-template <bool PDL>
-__device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, bool absorb,
-                                          LeafSmem& S) {
+// A window-P leaf (1 <= P <= LEAF_WINDOW) also applies everything the P
+// anti-diagonals before it in its block send to it, i.e. the Alg. 5 nodes
+// inside the block: for tile (I, J) that is the sum over the E tiles
+// (I - dp, J - g), 1 <= dp + g <= P, of L^B[I,I-dp] E[I-dp,J-g] L^A[J,J-g]^T.
+// The terms of row I (dp = 0) enter the wavefront as the initial value of G
+// (which the wavefront multiplies by L^B[I,I] anyway):
+//     T1 = sum_g E[I,J-g] L^A[J,J-g]^T.
+// The others are added to X before the wavefront:
+//     U = sum_dp L^B[I,I-dp] N_dp,   N_dp = sum_g E[I-dp,J-g] L^A[J,J-g]^T.
+// Tiles outside the matrix (I - dp < 0 or J - g < 0) are zeros.
+template <bool PDL, int P>
+__device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafSmem& S) {
+  static_assert(P >= 0 && P <= LEAF_WINDOW, "window");
+  static_assert(LEAF_PER_THREAD * LEAF_THREADS == TILE * TILE, "whole tile per pass");
   const int t = threadIdx.x, w = t >> 5, lane = t & 31;
   const int64_t r0 = (int64_t)I * TILE, c0 = (int64_t)J * TILE;
-  const bool has_left = absorb && J > 0, has_up = absorb && I > 0;
   // Factor blocks and the grid (read-only during the solve; the grid written
   // by the solve's first kernel, more than one kernel ago), loaded before
   // waiting for the previous kernel.  Each batch issues all its loads before
   // any is used, so their latencies overlap.
   {
-    float bh[LEAF_PER_THREAD], bl[LEAF_PER_THREAD], ah[LEAF_PER_THREAD], al[LEAF_PER_THREAD];
-#pragma unroll
-    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-      const int e = t + k * LEAF_THREADS;
-      const int p = e / TILE, c = e % TILE;
-      const int64_t ob = (r0 + p) * a.ldb + r0 + c, oa = (c0 + p) * a.lda + c0 + c;
-      bh[k] = a.LBH[ob];
-      bl[k] = a.LBL[ob];
-      ah[k] = a.LAH[oa];
-      al[k] = a.LAL[oa];
-    }
-#pragma unroll
-    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-      const int e = t + k * LEAF_THREADS;
-      const int p = e / TILE, c = e % TILE;
-      S.LBs[p][c] = bh[k] + bl[k];
-      S.LAs[p][c] = ah[k] + al[k];
-    }
+    const float* const hi[2] = {a.LBH, a.LAH};
+    const float* const lo[2] = {a.LBL, a.LAL};
+    const int64_t base[2] = {r0 * a.ldb + r0, c0 * a.lda + c0};
+    const int64_t ld[2] = {a.ldb, a.lda};
+    const bool valid[2] = {true, true};
+    // LBs has row stride 36 = KM, LAs 33: the second tile is stored by hand below
+    float* const dst[2] = {&S.LBs[0][0], &S.u.pro.Et[0][0][0]};
+    load_tiles<2, false>(hi, lo, base, ld, valid, dst, false, t);
   }
-  if (has_left || has_up) {
-    // sub-diagonal factor blocks, transposed to k-major
-    float bh[LEAF_PER_THREAD], bl[LEAF_PER_THREAD], ah[LEAF_PER_THREAD], al[LEAF_PER_THREAD];
+  if (P >= 1) {
+    // sub-diagonal factor blocks L^A[J, J-g], L^B[I, I-dp], transposed to k-major
 #pragma unroll
-    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-      const int e = t + k * LEAF_THREADS;
-      const int p = e / TILE, c = e % TILE;
-      const int64_t oa = (c0 + p) * a.lda + c0 - TILE + c, ob = (r0 + p) * a.ldb + r0 - TILE + c;
-      ah[k] = has_left ? a.LAH[oa] : 0.f;
-      al[k] = has_left ? a.LAL[oa] : 0.f;
-      bh[k] = has_up ? a.LBH[ob] : 0.f;
-      bl[k] = has_up ? a.LBL[ob] : 0.f;
-    }
+    for (int g0 = 1; g0 <= P; g0 += 3) {
+      constexpr int NB = 3;
+      const float* hi[NB];
+      const float* lo[NB];
+      int64_t base[NB], ld[NB];
+      bool valid[NB];
+      float* dst[NB];
 #pragma unroll
-    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-      const int e = t + k * LEAF_THREADS;
-      const int p = e / TILE, c = e % TILE;
-      S.u.pro.LAt[c][p] = ah[k] + al[k];
-      S.u.pro.LBt[c][p] = bh[k] + bl[k];
+      for (int s = 0; s < NB; ++s) {
+        const int g = g0 + s;
+        hi[s] = a.LAH; lo[s] = a.LAL; ld[s] = a.lda;
+        valid[s] = g <= P && J - g >= 0;
+        base[s] = valid[s] ? c0 * a.lda + c0 - (int64_t)TILE * g : 0;
+        dst[s] = g <= P ? &S.u.pro.LAt[g - 1][0][0] : nullptr;
+      }
+      load_tiles<NB, false>(hi, lo, base, ld, valid, dst, true, t);
+#pragma unroll
+      for (int s = 0; s < NB; ++s) {
+        const int dp = g0 + s;
+        hi[s] = a.LBH; lo[s] = a.LBL; ld[s] = a.ldb;
+        valid[s] = dp <= P && I - dp >= 0;
+        base[s] = valid[s] ? r0 * a.ldb + r0 - (int64_t)TILE * dp : 0;
+        dst[s] = dp <= P ? &S.u.pro.LBt[dp - 1][0][0] : nullptr;
+      }
+      load_tiles<NB, false>(hi, lo, base, ld, valid, dst, true, t);
     }
   }
   float scv[LEAF_PER_THREAD], zv[LEAF_PER_THREAD];
@@ -283,72 +336,127 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, bool 
 #pragma unroll
   for (int k = 0; k < LEAF_PER_THREAD; ++k) {
     const int e = t + k * LEAF_THREADS;
-    if (e < TILE * TILE) xv[k] = __ldcg(a.X + (r0 + e / TILE) * a.ldx + c0 + e % TILE);
+    xv[k] = __ldcg(a.X + (r0 + e / TILE) * a.ldx + c0 + e % TILE);
   }
-  if (has_left || has_up) {
-    // errors of the neighbours on anti-diagonal K-1, k-major as E^T stores
-    // them: every load issued before any is used
-    static_assert(LEAF_PER_THREAD * LEAF_THREADS == TILE * TILE, "whole tile per pass");
-    float lh[LEAF_PER_THREAD], ll[LEAF_PER_THREAD], uh[LEAF_PER_THREAD], ul[LEAF_PER_THREAD];
+  leaf_sync();   // LAs staged in Et[0]
 #pragma unroll
-    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-      const int e = t + k * LEAF_THREADS;
-      const int j = e / TILE, i = e % TILE;
-      const int64_t ol = (c0 - TILE + j) * a.ldt + r0 + i, ou = (c0 + j) * a.ldt + r0 - TILE + i;
-      lh[k] = has_left ? __ldcg(a.EtH + ol) : 0.f;
-      ll[k] = has_left ? __ldcg(a.EtL + ol) : 0.f;
-      uh[k] = has_up ? __ldcg(a.EtH + ou) : 0.f;
-      ul[k] = has_up ? __ldcg(a.EtL + ou) : 0.f;
-    }
-#pragma unroll
-    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-      const int e = t + k * LEAF_THREADS;
-      const int j = e / TILE, i = e % TILE;
-      S.u.pro.EL[j][i] = lh[k] + ll[k];
-      S.u.pro.EU[j][i] = uh[k] + ul[k];
-    }
+  for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+    const int e = t + k * LEAF_THREADS;
+    S.LAs[e / TILE][e % TILE] = S.u.pro.Et[0][e / TILE][e % TILE];
   }
-  leaf_sync();   // LBs, LAs and the absorbed operands complete
-  if (has_left || has_up) {
+  if (P >= 1) {
+    leaf_sync();   // Et[0] free again
+    // errors of the window's tiles, k-major as E^T stores them, three at a time
+    constexpr int NE = (P + 1) * (P + 2) / 2 - 1;   // E tiles of the window
+#pragma unroll
+    for (int s0 = 0; s0 < NE; s0 += 3) {
+      constexpr int NB = 3;
+      const float* const hi[NB] = {a.EtH, a.EtH, a.EtH};
+      const float* const lo[NB] = {a.EtL, a.EtL, a.EtL};
+      int64_t base[NB];
+      const int64_t ld[NB] = {a.ldt, a.ldt, a.ldt};
+      bool valid[NB];
+      float* dst[NB];
+#pragma unroll
+      for (int s = 0; s < NB; ++s) {
+        // slot s0 + s -> (dp, g)
+        int dp = 0, g = 0, idx = s0 + s;
+        if (idx < P) { dp = 0; g = idx + 1; }
+        else {
+          idx -= P;
+#pragma unroll
+          for (int d = 1; d <= LEAF_WINDOW; ++d) {
+            const int cnt = P - d + 1;
+            if (d <= P && dp == 0 && idx < cnt) { dp = d; g = idx; }
+            else if (d <= P && dp == 0) idx -= cnt;
+          }
+        }
+        valid[s] = s0 + s < NE && dp + g >= 1 && I - dp >= 0 && J - g >= 0;
+        // E[I - dp, J - g] k-major: row j of the tile is E^T row c0 - 32 g + j
+        base[s] = valid[s] ? (c0 - (int64_t)TILE * g) * a.ldt + r0 - (int64_t)TILE * dp : 0;
+        dst[s] = s0 + s < NE ? &S.u.pro.Et[s0 + s][0][0] : nullptr;
+      }
+      load_tiles<NB, true>(hi, lo, base, ld, valid, dst, false, t);
+    }
+    leaf_sync();
+    // round 1: T1 and N_1 .. N_P in one pass over K (their terms interleave)
     const int pr = 4 * (t >> 4), pc = 2 * (t & 15);
-    float acc[4][2];
-    if (t < 128) {
-      if (has_left) {   // T1[i][q] = sum_j E[I,J-1][i][j] L^A[J,J-1][q][j]
-        mm_4x2(&S.u.pro.EL[0][0], &S.u.pro.LAt[0][0], KM, 1, t, acc);
+    float acc[P + 1][4][2];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          S.T1s[pr + i][pc] = acc[i][0];
-          S.T1s[pr + i][pc + 1] = acc[i][1];
+    for (int o = 0; o <= P; ++o)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) acc[o][i][0] = acc[o][i][1] = 0.f;
+#pragma unroll 2
+    for (int k = 0; k < TILE; ++k) {
+      float b[P + 1][2];   // L^A[J, J-g][c][k] for this thread's two columns
+      b[0][0] = S.LAs[pc][k];
+      b[0][1] = S.LAs[pc + 1][k];
+#pragma unroll
+      for (int g = 1; g <= P; ++g) {
+        b[g][0] = S.u.pro.LAt[g - 1][k][pc];
+        b[g][1] = S.u.pro.LAt[g - 1][k][pc + 1];
+      }
+#pragma unroll
+      for (int dp = 0; dp <= P; ++dp) {
+#pragma unroll
+        for (int g = (dp == 0 ? 1 : 0); g + dp <= P; ++g) {
+          const float4 av = *reinterpret_cast<const float4*>(&S.u.pro.Et[window_slot(P, dp, g)][k][pr]);
+          acc[dp][0][0] = fmaf(av.x, b[g][0], acc[dp][0][0]);
+          acc[dp][0][1] = fmaf(av.x, b[g][1], acc[dp][0][1]);
+          acc[dp][1][0] = fmaf(av.y, b[g][0], acc[dp][1][0]);
+          acc[dp][1][1] = fmaf(av.y, b[g][1], acc[dp][1][1]);
+          acc[dp][2][0] = fmaf(av.z, b[g][0], acc[dp][2][0]);
+          acc[dp][2][1] = fmaf(av.z, b[g][1], acc[dp][2][1]);
+          acc[dp][3][0] = fmaf(av.w, b[g][0], acc[dp][3][0]);
+          acc[dp][3][1] = fmaf(av.w, b[g][1], acc[dp][3][1]);
         }
       }
-      if (has_up) {     // T2[i][q] = sum_j E[I-1,J][i][j] L^A[J,J][q][j]
-        mm_4x2(&S.u.pro.EU[0][0], &S.LAs[0][0], 1, TILE + 1, t, acc);
+    }
+    leaf_sync();   // the E tiles are read: their slots take N_dp and U
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          S.u.pro.T2[pr + i][pc] = acc[i][0];
-          S.u.pro.T2[pr + i][pc + 1] = acc[i][1];
-        }
+    for (int i = 0; i < 4; ++i) {
+      S.T1s[pr + i][pc] = acc[0][i][0];
+      S.T1s[pr + i][pc + 1] = acc[0][i][1];
+#pragma unroll
+      for (int dp = 1; dp <= P; ++dp) {
+        S.u.pro.Et[dp - 1][pr + i][pc] = acc[dp][i][0];
+        S.u.pro.Et[dp - 1][pr + i][pc + 1] = acc[dp][i][1];
       }
     }
     leaf_sync();
-    if (has_up) {
-      if (t < 128) {    // U[p][q] = sum_i L^B[I,I-1][p][i] T2[i][q], into EL's place
-        mm_4x2(&S.u.pro.LBt[0][0], &S.u.pro.T2[0][0], KM, 1, t, acc);
+    // round 2: U[p][q] = sum_dp sum_i L^B[I,I-dp][p][i] N_dp[i][q], into slot P
+    float u[4][2];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          S.u.pro.EL[pr + i][pc] = acc[i][0];
-          S.u.pro.EL[pr + i][pc + 1] = acc[i][1];
-        }
-      }
-      leaf_sync();
+    for (int i = 0; i < 4; ++i) u[i][0] = u[i][1] = 0.f;
+#pragma unroll 2
+    for (int k = 0; k < TILE; ++k) {
 #pragma unroll
-      for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-        const int e = t + k * LEAF_THREADS;
-        if (e < TILE * TILE) xv[k] += S.u.pro.EL[e / TILE][e % TILE];
+      for (int dp = 1; dp <= P; ++dp) {
+        const float4 av = *reinterpret_cast<const float4*>(&S.u.pro.LBt[dp - 1][k][pr]);
+        const float b0 = S.u.pro.Et[dp - 1][k][pc], b1 = S.u.pro.Et[dp - 1][k][pc + 1];
+        u[0][0] = fmaf(av.x, b0, u[0][0]);
+        u[0][1] = fmaf(av.x, b1, u[0][1]);
+        u[1][0] = fmaf(av.y, b0, u[1][0]);
+        u[1][1] = fmaf(av.y, b1, u[1][1]);
+        u[2][0] = fmaf(av.z, b0, u[2][0]);
+        u[2][1] = fmaf(av.z, b1, u[2][1]);
+        u[3][0] = fmaf(av.w, b0, u[3][0]);
+        u[3][1] = fmaf(av.w, b1, u[3][1]);
       }
-      leaf_sync();   // the wavefront's arrays overlay the prologue's
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      S.u.pro.Et[P][pr + i][pc] = u[i][0];
+      S.u.pro.Et[P][pr + i][pc + 1] = u[i][1];
+    }
+    leaf_sync();
+#pragma unroll
+    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+      const int e = t + k * LEAF_THREADS;
+      xv[k] += S.u.pro.Et[P][e / TILE][e % TILE];
     }
   }
+  leaf_sync();   // the wavefront's arrays overlay the prologue's
 #pragma unroll
   for (int k = 0; k < LEAF_PER_THREAD; ++k) {
     const int e = t + k * LEAF_THREADS;
@@ -449,7 +557,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, bool 
     float Gg[LEAF_ROWS_PER_HELPER];
 #pragma unroll
     for (int r = 0; r < LEAF_ROWS_PER_HELPER; ++r)
-      Gg[r] = (has_left && i0 + r < TILE) ? S.T1s[i0 + r][q] : 0.f;
+      Gg[r] = (P >= 1 && i0 + r < TILE) ? S.T1s[i0 + r][q] : 0.f;
     // partial pre of step d's entry (row d - q) over these rows
     auto dot = [&](int d) {
       const int pn = d - q;
@@ -532,11 +640,13 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, bool 
   leaf_sync();   // shared memory free for the next tile of this CTA
 }
 
-// One CTA per tile of tile anti-diagonal K.
-__global__ void __launch_bounds__(LEAF_THREADS) k_leaf(int K, int absorb, LeafArgs a) {
-  __shared__ LeafSmem S;
+// One CTA per tile of tile anti-diagonal K; P: the leaf's window.
+template <int P>
+__global__ void __launch_bounds__(LEAF_THREADS) k_leaf(int K, LeafArgs a) {
+  extern __shared__ __align__(16) unsigned char leaf_smem[];
+  LeafSmem& S = *reinterpret_cast<LeafSmem*>(leaf_smem);
   const int I = max(0, K - (a.Nt - 1)) + blockIdx.x;
-  leaf_tile<true>(a, I, K - I, absorb != 0, S);
+  leaf_tile<true, P>(a, I, K - I, S);
 }
 
 // ------------------------------------------------------- band products (SIMT)
@@ -790,9 +900,9 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_band_fused_simt(Band bd, BandA
 // kernel boundaries.  Each phase spreads its units (tiles of a leaf, output
 // or M tiles of a band stage) over the CTAs; a CTA runs a leaf with its first
 // five warps and a band unit with all eight.
-enum PhaseType { PH_LEAF = 0, PH_FUSED = 1, PH_STAGE1 = 2, PH_STAGE2 = 3, PH_LEAF_ABSORB = 4 };
+enum PhaseType { PH_LEAF = 0, PH_FUSED = 1, PH_STAGE1 = 2, PH_STAGE2 = 3 };
 struct Phase {
-  int type, k, h, l;
+  int type, k, h, l;   // a leaf: k its anti-diagonal, h its window
 };
 constexpr int MAX_SUBTREE = 32;  // widest range run as one subtree (anti-diagonals)
 constexpr int MAX_PHASES = 128;  // >= MAX_SUBTREE leaves + 2 phases per band node
@@ -855,11 +965,15 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_subtree(const __grid_constant_
   const int Mt = A.leaf.Mt, Nt = A.leaf.Nt;
   for (int ph = 0; ph < A.nph; ++ph) {
     const Phase P = A.ph[ph];
-    if (P.type == PH_LEAF || P.type == PH_LEAF_ABSORB) {
+    if (P.type == PH_LEAF) {
       const int ilo = max(0, P.k - (Nt - 1)), ihi = min(P.k, Mt - 1);
       if (threadIdx.x < LEAF_THREADS)
-        for (int I = ilo + (int)blockIdx.x; I <= ihi; I += gridDim.x)
-          leaf_tile<false>(A.leaf, I, P.k - I, P.type == PH_LEAF_ABSORB, S.leaf);
+        for (int I = ilo + (int)blockIdx.x; I <= ihi; I += gridDim.x) {
+          if (P.h == 0) leaf_tile<false, 0>(A.leaf, I, P.k - I, S.leaf);
+          else if (P.h == 1) leaf_tile<false, 1>(A.leaf, I, P.k - I, S.leaf);
+          else if (P.h == 2) leaf_tile<false, 2>(A.leaf, I, P.k - I, S.leaf);
+          else leaf_tile<false, 3>(A.leaf, I, P.k - I, S.leaf);
+        }
     } else {
       const int row_lo = max(0, P.h - (Nt - 1)), row_hi = min(Mt - 1, P.l - 1);
       const Band bd{P.k, P.h, P.l, Mt, Nt, row_lo};
@@ -946,17 +1060,42 @@ static void note(SolveArgs& a, cudaError_t e) {
   if (e != cudaSuccess) a.rc = BAKRON_ERR_CUDA;
 }
 
-// Leaf of anti-diagonal K; `absorb`: it also applies the node (K-1, K, K+1).
-static void leaf(SolveArgs& a, int K, int absorb) {
+// Leaf of anti-diagonal K; `window`: how many anti-diagonals before it (in
+// its block) it absorbs.  Flops: the in-tile feedback and the window's
+// products, 2 * 32^3 each, per tile.
+static void leaf(SolveArgs& a, int K, int window) {
   const int ilo = max(0, K - (a.Nt - 1)), ihi = min(K, a.Mt - 1);
-  double flops = 2.0 * TILE * TILE * TILE * (ihi - ilo + 1);
-  if (absorb && a.profiling) {
-    double p1, p2;
-    band_tile_products(a, K - 1, K, K + 1, p1, p2);
-    flops += 2.0 * TILE * TILE * TILE * (p1 + p2);
+  LaunchScope ls(kFamLeaf, a.s,
+                 2.0 * TILE * TILE * TILE * (1 + window_products(window)) * (ihi - ilo + 1));
+  const dim3 grid(ihi - ilo + 1), block(LEAF_THREADS);
+  const size_t sm = sizeof(LeafSmem);
+  switch (window) {
+    case 0: note(a, launch_pdl(k_leaf<0>, grid, block, sm, a.s, K, a.la)); break;
+    case 1: note(a, launch_pdl(k_leaf<1>, grid, block, sm, a.s, K, a.la)); break;
+    case 2: note(a, launch_pdl(k_leaf<2>, grid, block, sm, a.s, K, a.la)); break;
+    default: note(a, launch_pdl(k_leaf<3>, grid, block, sm, a.s, K, a.la)); break;
   }
-  LaunchScope ls(kFamLeaf, a.s, flops);
-  note(a, launch_pdl(k_leaf, dim3(ihi - ilo + 1), dim3(LEAF_THREADS), 0, a.s, K, absorb, a.la));
+}
+
+// Dynamic shared memory of the leaf and subtree kernels above the 48 KB
+// default, set once per process.
+static cudaError_t ensure_leaf_attrs() {
+  static std::mutex mu;
+  static bool done = false;
+  std::lock_guard<std::mutex> lk(mu);
+  if (done) return cudaSuccess;
+  const int sm = (int)sizeof(LeafSmem), ss = (int)sizeof(SubtreeSmem);
+  cudaError_t e = cudaFuncSetAttribute(k_leaf<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_leaf<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_leaf<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_leaf<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_subtree, cudaFuncAttributeMaxDynamicSharedMemorySize, ss);
+  if (e == cudaSuccess) done = true;
+  return e;
 }
 
 static void band(SolveArgs& a, int k, int h, int l) {
@@ -999,13 +1138,8 @@ static void band(SolveArgs& a, int k, int h, int l) {
 
 // Phases of rec(k, l) in the order rec enqueues them.
 static void subtree_phases(const SolveArgs& a, int k, int l, SubtreeArgs& A) {
-  if (l == k + 1) {
-    A.ph[A.nph++] = Phase{PH_LEAF, k, k, l};
-    return;
-  }
-  if (l == k + 2) {   // the node (k, k+1, k+2) is applied by its second leaf
-    A.ph[A.nph++] = Phase{PH_LEAF, k, k, k + 1};
-    A.ph[A.nph++] = Phase{PH_LEAF_ABSORB, k + 1, k + 1, l};
+  if (l - k <= LEAF_WINDOW + 1) {   // a block of leaves, each absorbing the ones before it
+    for (int K = k; K < l; ++K) A.ph[A.nph++] = Phase{PH_LEAF, K, K - k, K + 1};
     return;
   }
   const int h = (k + l) / 2;
@@ -1039,14 +1173,9 @@ static void subtree(SolveArgs& a, int k, int l) {
   if (a.profiling) {
     for (int i = 0; i < A.nph; ++i) {
       const Phase& P = A.ph[i];
-      if (P.type == PH_LEAF || P.type == PH_LEAF_ABSORB) {
-        flops += 2.0 * TILE * TILE * TILE *
+      if (P.type == PH_LEAF) {
+        flops += 2.0 * TILE * TILE * TILE * (1 + window_products(P.h)) *
                  (min(P.k, a.Mt - 1) - max(0, P.k - (a.Nt - 1)) + 1);
-        if (P.type == PH_LEAF_ABSORB) {
-          double p1, p2;
-          band_tile_products(a, P.k - 1, P.k, P.k + 1, p1, p2);
-          flops += 2.0 * TILE * TILE * TILE * (p1 + p2);
-        }
       } else if (P.type != PH_STAGE2) {
         double p1, p2;
         band_tile_products(a, P.k, P.h, P.l, p1, p2);
@@ -1069,13 +1198,10 @@ static void subtree(SolveArgs& a, int k, int l) {
 }
 
 static void rec(SolveArgs& a, int k, int l) {
-  if (l == k + 1) {
-    leaf(a, k, 0);
-    return;
-  }
-  if (l == k + 2) {   // the node (k, k+1, k+2) is applied by its second leaf
-    leaf(a, k, 0);
-    leaf(a, k + 1, 1);
+  if (l - k <= LEAF_WINDOW + 1) {
+    // a block of leaves: leaf K applies what anti-diagonals k .. K-1 send it
+    // (the Alg. 5 nodes inside [k, l)), so no band launch is needed here
+    for (int K = k; K < l; ++K) leaf(a, K, K - k);
     return;
   }
   if (l - k <= a.subtree_max && a.subtree_grid > 0) {
@@ -1122,6 +1248,7 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
                   a.MH, a.ML, a.np, a.X, a.np};
   a.profiling = profiling_on();
   {
+    if (ensure_leaf_attrs() != cudaSuccess) return BAKRON_ERR_CUDA;
     const Tuning tu = force ? *force : tuning_for(m, n);
     a.tc_min_band = tu.tc_min_band;         // 0 or less: tensor cores off
     a.fused_max_band = tu.fused_max_band;
