@@ -251,6 +251,7 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
 __global__ void __launch_bounds__(THREADS, 1)
 k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUtensorMap mapAl,
           const __grid_constant__ CUtensorMap mapBh, const __grid_constant__ CUtensorMap mapBl,
+          const __grid_constant__ CUtensorMap mapBh4, const __grid_constant__ CUtensorMap mapBl4,
           const TcParams P) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // 1024-byte alignment for the 128-byte swizzle atoms
@@ -273,6 +274,14 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
     return;
   }
 
+  if (threadIdx.x == 32) {   // descriptors into the cache while the previous kernel runs
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapAh)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapAl)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBh)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBl)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBh4)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBl4)) : "memory");
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
@@ -349,7 +358,10 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
         mbar_expect_tx(&full[s], bytes);
         tma_load_2d(a_hi, &mapAh, &full[s], kt * BK, blk.rb * BM);
         tma_load_2d(a_lo, &mapAl, &full[s], kt * BK, blk.rb * BM);
-        if (P.mode == MODE_STAGE1) {
+        if (P.mode == MODE_STAGE1 && valid == 0xFu) {   // inside the band: one box per plane
+          tma_load_2d(b_hi, &mapBh4, &full[s], kt * BK, blk.cb * BN);
+          tma_load_2d(b_lo, &mapBl4, &full[s], kt * BK, blk.cb * BN);
+        } else if (P.mode == MODE_STAGE1) {
           for (int sub = 0; sub < 4; ++sub) {
             if (!(valid & (1u << sub))) continue;
             const int y = (4 * blk.cb + sub) * 32;
@@ -574,6 +586,8 @@ bool tc_band_maps(TcMaps& maps, const TcOperands& op) {
   ok &= make_map(&maps.LBl, op.LBL, op.mp, op.mp, op.mp, BM);
   ok &= make_map(&maps.Eth, op.EtH, op.np, op.mp, op.mp, 32);
   ok &= make_map(&maps.Etl, op.EtL, op.np, op.mp, op.mp, 32);
+  ok &= make_map(&maps.Eth4, op.EtH, op.np, op.mp, op.mp, BN);
+  ok &= make_map(&maps.Etl4, op.EtL, op.np, op.mp, op.mp, BN);
   ok &= make_map(&maps.Mh, op.MH, op.mp, op.np, op.np, BM);
   ok &= make_map(&maps.Ml, op.ML, op.mp, op.np, op.np, BM);
   ok &= make_map(&maps.LAh, op.LAH, op.np, op.np, op.np, BN);
@@ -609,10 +623,10 @@ int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, in
   cudaError_t e;
   if (stage == 1)
     e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.LBh, maps.LBl, maps.Eth,
-                   maps.Etl, P);
+                   maps.Etl, maps.Eth4, maps.Etl4, P);
   else
     e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.Mh, maps.Ml, maps.LAh,
-                   maps.LAl, P);
+                   maps.LAl, maps.LAh, maps.LAl, P);
   return e == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
 }
 
@@ -651,7 +665,7 @@ extern "C" int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C,
   P.status = status;
   P.spin_cycles = spin_cycles_from_env();
   dim3 grid(N / BN, M / BM);
-  k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(mA, mAl, mB, mBl, P);
+  k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(mA, mAl, mB, mBl, mB, mBl, P);
   BK_CUDA_OK(cudaGetLastError());
   return bakron_read_status(workspace, stream);
 }

@@ -18,6 +18,7 @@ struct TcOperands {
 // TMA descriptors of every operand plane (built on the host per solve call).
 struct TcMaps {
   CUtensorMap LBh, LBl, Eth, Etl, Mh, Ml, LAh, LAl;
+  CUtensorMap Eth4, Etl4;   // E^T planes in 128-row boxes (whole stage-1 B operand)
 };
 
 bool tc_band_maps(TcMaps& maps, const TcOperands& op);
