@@ -103,16 +103,16 @@ __global__ void k_copy_out(const float* X, int64_t np, int m, int n, float* out)
 //     form the partial pre of later steps, sum_i L^B[p][i] G_q[i] (+ X_pq),
 //     which they leave in shared memory.
 // The two sides hand over once per two steps (one barrier); see the
-// wavefront below for the exact lag.  A step is latency bound (a dependent
-// chain of a shuffle and about eight floating-point operations), and every
-// warp of the leaf issues from a scheduler of its own: errors are broadcast
-// indexed by row (every row written every step, zero when off the tile), a
-// helper keeps its L^A values in registers rotated by 8 every 8 steps
-// (compile-time slots), and codes are staged in shared memory and stored
-// coalesced at the end.
-// x / s is evaluated as x * fl(1/s); it can differ from the correctly rounded
-// quotient by one ulp, which only matters within 1e-6 grid units of a
-// rounding boundary.
+// wavefront below for the exact lag.  A step is latency bound (a shuffle and
+// about seven dependent floating-point operations), and every warp of the
+// leaf issues from a scheduler of its own: errors are broadcast indexed by
+// row (every row written every step, zero when off the tile), a helper keeps
+// its L^A values in registers rotated by 8 every 8 steps (compile-time slots)
+// and loads the L^B rows of its dot products one interval ahead, and codes
+// are staged in shared memory and stored coalesced at the end.
+// x / s is evaluated as the exact product x * fl(1/s), rounded once to an
+// integer; fl(1/s) can differ from 1/s by half an ulp, which only matters
+// within 1e-6 grid units of a rounding boundary.
 // Outputs: codes, X (pre-rounding values) and E^T as a tf32 hi/lo pair.
 // Three helper warps, so that each of the SM's four schedulers runs one warp
 // of the leaf (warp w issues from scheduler w mod 4) and the chain shares its
@@ -492,57 +492,74 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     const float la2 = q >= 2 ? S.LAs[q][q - 2] : 0.f;
     const float la3 = q >= 3 ? S.LAs[q][q - 3] : 0.f;
     const float fq = (float)a.qmax;
+    // Rounding to the nearest integer (ties to even) by the shift R = 1.5 * 2^23:
+    // for |v| < 2^22, fl(v + R) - R is v rounded to an integer, and the clamp
+    // to integer bounds commutes with it, so
+    //     c - z = clamp(fl(x * fl(1/s) + R), R - z, R + qmax - z) - R
+    // (one fused multiply-add: the product x * fl(1/s) is rounded once, to
+    // the integer).  Larger |v| fall outside the bounds and are clamped.
+    constexpr float R = 12582912.f;
     float E1 = 0.f, E2 = 0.f, E3 = 0.f;
     float L1_1 = 0.f, L1_2 = 0.f, L1_3 = 0.f, L2_2 = 0.f, L2_3 = 0.f, L3_3 = 0.f;
-    // one step: explicit terms of the last two (ODD: three) steps, then round
+    // One step.  Of the explicit terms only E1 (own column, last step) and
+    // L1_1 (left neighbour, last step, still in flight from its shuffle) are
+    // new; the sum of the older ones is formed first so that these two enter
+    // last.  The shuffles the next step needs are issued as soon as their
+    // inputs exist.  Entries off the tile or outside W get a zero error (the
+    // factor mk).
     auto step = [&](int d, bool odd, float pre, const float4& g, const float4& lb) {
       const int p = d - q;
-      const bool act = p >= 0 && p < TILE;
-      // age the left columns' errors by one step, then fetch the new ones
+      const bool on_tile = p >= 0 && p < TILE;
+      float A = fmaf(la2, L2_2, pre);
+      const float A2 = fmaf(lb.y, E2, (lb.x * la1) * L1_2);
+      if (odd) {
+        const float o1 = fmaf(la3, L3_3, (lb.x * la2) * L2_3);
+        const float o2 = fmaf(lb.y * la1, L1_3, lb.z * E3);
+        A = A + (o1 + o2);
+      }
+      A = A + A2;
+      const float nL3_3 = __shfl_up_sync(0xffffffffu, L2_2, 1);   // column q-3, this step's d-2
+      const float x = fmaf(la1, L1_1, fmaf(lb.x, E1, A));
+      const float nL2_2 = __shfl_up_sync(0xffffffffu, L1_1, 1);   // column q-2, step d-1
+      const float tc = fminf(fmaxf(fmaf(x, g.y, R), R + g.z), R + fq + g.z);
+      const float mk = (on_tile && p < rows_real && col_real) ? 1.f : 0.f;
+      const float e = fmaf(g.x * mk, tc - R, x * -mk);   // s (c - z) - x, rounded once
       L1_3 = L1_2;
       L1_2 = L1_1;
       L2_3 = L2_2;
-      L2_2 = __shfl_up_sync(0xffffffffu, L1_2, 1);   // column q-2, step d-2
-      L3_3 = __shfl_up_sync(0xffffffffu, L2_3, 1);   // column q-3, step d-3
-      L1_1 = __shfl_up_sync(0xffffffffu, E1, 1);     // column q-1, step d-1
-      float r = fmaf(lb.x, fmaf(la1, L1_2, E1), fmaf(la2, L2_2, pre));
-      r = fmaf(lb.y, E2, r);
-      if (odd) {
-        r = fmaf(la3, L3_3, r);
-        r = fmaf(lb.x, la2 * L2_3, r);
-        r = fmaf(lb.y, la1 * L1_3, r);
-        r = fmaf(lb.z, E3, r);
-      }
-      const float x = fmaf(la1, L1_1, r);
-      // code c = clamp(rint(x / s) + z, 0, qmax); with the integer z the
-      // clamp moves before the rounding and the offset after it:
-      // c - z = rint(clamp(x / s, -z, qmax - z)), exactly
-      const float cz = rintf(fminf(fmaxf(x * g.y, g.z), fq + g.z));
-      float e = fmaf(g.x, cz, -x);         // s (c - z) - x, rounded once
-      if (!(act && p < rows_real && col_real)) e = 0.f;
-      if (act) {
-        S.u.w.XE[p][q] = make_float2(x, e);
-        S.u.w.Cs[p][q] = (uint8_t)(cz - g.z);
-      }
-      S.Ebr[d & 3][p & (TILE - 1)] = e;    // rows off the tile get a zero
+      L2_2 = nL2_2;
+      L3_3 = nL3_3;
       E3 = E2;
       E2 = E1;
       E1 = e;
+      L1_1 = __shfl_up_sync(0xffffffffu, e, 1);                    // column q-1, step d
+      if (on_tile) {
+        S.u.w.XE[p][q] = make_float2(x, e);
+        S.u.w.Cs[p][q] = (uint8_t)(int)(tc - (R + g.z));
+      }
+      S.Ebr[d & 3][p & (TILE - 1)] = e;    // rows off the tile get a zero
     };
+    // (s, 1/s, -z) and the sub-diagonal L^B of the next interval's entries are
+    // loaded one interval ahead
+    float4 g0 = S.u.w.Srzl[(0 - q) & (TILE - 1)][q], g1 = S.u.w.Srzl[(1 - q) & (TILE - 1)][q];
+    float4 lb0 = S.Lsub[(0 - q) & (TILE - 1)], lb1 = S.Lsub[(1 - q) & (TILE - 1)];
     leaf_sync();   // the helpers' pre of steps 0 and 1
 #pragma unroll 1
     for (int k = 0; k < TILE; ++k) {
       const int d0 = 2 * k, d1 = 2 * k + 1;
-      const int p0 = (d0 - q) & (TILE - 1), p1 = (d1 - q) & (TILE - 1);
       const float* pa = &S.Part[d0 & 3][0][q];
       const float* pb = &S.Part[d1 & 3][0][q];
       static_assert(LEAF_HELPERS == 3, "the chain sums three partials");
       const float pre0 = (pa[0] + pa[TILE]) + pa[2 * TILE];
       const float pre1 = (pb[0] + pb[TILE]) + pb[2 * TILE];
-      const float4 g0 = S.u.w.Srzl[p0][q], g1 = S.u.w.Srzl[p1][q];
-      const float4 lb0 = S.Lsub[p0], lb1 = S.Lsub[p1];
-      step(d0, false, pre0, g0, lb0);
-      if (d1 < 2 * TILE - 1) step(d1, true, pre1, g1, lb1);
+      const float4 g0c = g0, g1c = g1, lb0c = lb0, lb1c = lb1;
+      const int n0 = (d0 + 2 - q) & (TILE - 1), n1 = (d1 + 2 - q) & (TILE - 1);
+      g0 = S.u.w.Srzl[n0][q];
+      g1 = S.u.w.Srzl[n1][q];
+      lb0 = S.Lsub[n0];
+      lb1 = S.Lsub[n1];
+      step(d0, false, pre0, g0c, lb0c);
+      if (d1 < 2 * TILE - 1) step(d1, true, pre1, g1c, lb1c);
       leaf_sync();
     }
   } else {
@@ -558,23 +575,36 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
 #pragma unroll
     for (int r = 0; r < LEAF_ROWS_PER_HELPER; ++r)
       Gg[r] = (P >= 1 && i0 + r < TILE) ? S.T1s[i0 + r][q] : 0.f;
-    // partial pre of step d's entry (row d - q) over these rows
-    auto dot = [&](int d) {
+    // The L^B row (and, for helper 0, X) of step d's entry (row d - q), zero
+    // off the tile; loaded one interval before use into one of four slots
+    // (slots 2, 3 serve even intervals, 0, 1 odd ones).
+    float LBv[4][LEAF_ROWS_PER_HELPER], Xv[4];
+    auto fetch = [&](int d, int slot) {
       const int pn = d - q;
-      float acc = 0.f;
-      if (pn >= 0 && pn < TILE) {
-        float a4[LEAF_ROWS_PER_HELPER / 4];
+      const bool on_tile = pn >= 0 && pn < TILE;
+      const int pr = on_tile ? pn : 0;
 #pragma unroll
-        for (int v = 0; v < LEAF_ROWS_PER_HELPER / 4; ++v) {
-          const float4 l = *reinterpret_cast<const float4*>(&S.LBs[pn][i0 + 4 * v]);
-          a4[v] = fmaf(l.x, Gg[4 * v],
-                       fmaf(l.y, Gg[4 * v + 1], fmaf(l.z, Gg[4 * v + 2], l.w * Gg[4 * v + 3])));
-        }
-        static_assert(LEAF_ROWS_PER_HELPER == 12, "three float4 groups per helper");
-        acc = (a4[0] + a4[1]) + a4[2];
-        if (g == 0) acc += S.Xs[pn][q];
+      for (int v = 0; v < LEAF_ROWS_PER_HELPER / 4; ++v) {
+        float4 l = *reinterpret_cast<const float4*>(&S.LBs[pr][i0 + 4 * v]);
+        if (!on_tile) l = make_float4(0.f, 0.f, 0.f, 0.f);
+        LBv[slot][4 * v] = l.x;
+        LBv[slot][4 * v + 1] = l.y;
+        LBv[slot][4 * v + 2] = l.z;
+        LBv[slot][4 * v + 3] = l.w;
       }
-      S.Part[d & 3][g][q] = acc;
+      Xv[slot] = (g == 0 && on_tile) ? S.Xs[pr][q] : 0.f;
+    };
+    // partial pre of step d's entry over these rows (zero off the tile)
+    auto dot = [&](int d, int slot) {
+      float a4[LEAF_ROWS_PER_HELPER / 4];
+#pragma unroll
+      for (int v = 0; v < LEAF_ROWS_PER_HELPER / 4; ++v)
+        a4[v] = fmaf(LBv[slot][4 * v], Gg[4 * v],
+                     fmaf(LBv[slot][4 * v + 1], Gg[4 * v + 1],
+                          fmaf(LBv[slot][4 * v + 2], Gg[4 * v + 2],
+                               fmaf(LBv[slot][4 * v + 3], Gg[4 * v + 3], v == 0 ? Xv[slot] : 0.f))));
+      static_assert(LEAF_ROWS_PER_HELPER == 12, "three float4 groups per helper");
+      S.Part[d & 3][g][q] = (a4[0] + a4[1]) + a4[2];
     };
     // fold the errors of step sidx (its row i0 + r came from column sidx - i0 - r)
     auto fold = [&](int sidx, int slot0) {
@@ -592,20 +622,27 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
         Gg[r] = fmaf(ev[r], LAr[(slot0 - r) & (TILE - 1)], Gg[r]);
     };
     // the pre of steps 0 and 1: nothing folded yet
-    dot(0);
-    dot(1);
+    fetch(0, 0);
+    fetch(1, 1);
+    dot(0, 0);
+    dot(1, 1);
+    fetch(2, 2);
+    fetch(3, 3);
     leaf_sync();   // the chain's interval 0 may start
 #pragma unroll 1
     for (int b = 0; b < TILE / 4; ++b) {
 #pragma unroll
       for (int v = 0; v < 4; ++v) {
         const int k = 4 * b + v;
+        const int cur = (v & 1) ? 0 : 2, nxt = (v & 1) ? 2 : 0;
+        fetch(2 * k + 4, nxt);    // rows of the next interval, ahead of their use
+        fetch(2 * k + 5, nxt + 1);
         if (k >= 1) {             // steps 2k-2 and 2k-1 were published at the last barrier
           fold(2 * k - 2, 2 * v);
           fold(2 * k - 1, 2 * v + 1);
         }
-        if (2 * k + 2 < 2 * TILE - 1) dot(2 * k + 2);
-        if (2 * k + 3 < 2 * TILE - 1) dot(2 * k + 3);
+        if (2 * k + 2 < 2 * TILE - 1) dot(2 * k + 2, cur);
+        if (2 * k + 3 < 2 * TILE - 1) dot(2 * k + 3, cur + 1);
         leaf_sync();
       }
       // next block: the slot of every column drops by 8, i.e. new slot s = old slot s + 8
