@@ -89,7 +89,7 @@ int bakron_set_factors(const float* LA, const float* LB, const float* rA, const 
   k_import_diag<<<nblocks(fl.np, 256), 256, 0, s>>>(rA, n, (float*)(f + fl.off_rA), fl.np);
   k_import_diag<<<nblocks(fl.mp, 256), 256, 0, s>>>(rB, m, (float*)(f + fl.off_rB), fl.mp);
   BK_CUDA_OK(cudaGetLastError());
-  return BAKRON_OK;
+  return build_leaf_blocks(fl, f, s);
 }
 
 int bakron_get_factors(const void* factors, int m, int n, float* LA, float* LB, float* rA,

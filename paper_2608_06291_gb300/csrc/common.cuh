@@ -46,28 +46,47 @@ __host__ __device__ inline float tf32_hi(float x) {
 // [rB mp][rA np], fp32, sections 256-byte aligned.  L^X = hi + lo exactly;
 // stored dense row-major with exact zeros above the diagonal, ones on it and
 // an identity extension over the padding.
+// Then the leaf blocks: per tile row I of L^B, the diagonal block and the
+// LEAF_BLOCKS - 1 blocks left of it, L^B[I, I - d]; per tile column J of L^A,
+// L^A[J, J - g]; fp32 (hi + lo), TILE rows of LEAF_BLOCK_LD floats each (the
+// columns past TILE zero), laid out as the leaf kernel keeps them in shared
+// memory (see build_leaf_blocks), so that it copies them as they are.
+constexpr int LEAF_BLOCKS = 4;
+constexpr int LEAF_BLOCK_LD = 36;
+constexpr int LEAF_BLOCK_FLOATS = TILE * LEAF_BLOCK_LD;
+
 struct FactorLayout {
   int m, n;
-  int64_t mp, np;
-  size_t off_LBH, off_LBL, off_LAH, off_LAL, off_rB, off_rA, bytes;
+  int64_t mp, np, Mt, Nt;
+  size_t off_LBH, off_LBL, off_LAH, off_LAL, off_rB, off_rA, off_LBblk, off_LAblk, bytes;
   explicit FactorLayout(int m_, int n_) : m(m_), n(n_) {
     mp = round_up(m, PAD);
     np = round_up(n, PAD);
+    Mt = mp / TILE;
+    Nt = np / TILE;
     off_LBH = 0;
     off_LBL = align256(off_LBH + size_t(mp * mp) * 4);
     off_LAH = align256(off_LBL + size_t(mp * mp) * 4);
     off_LAL = align256(off_LAH + size_t(np * np) * 4);
     off_rB = align256(off_LAL + size_t(np * np) * 4);
     off_rA = align256(off_rB + size_t(mp) * 4);
-    bytes = align256(off_rA + size_t(np) * 4);
+    off_LBblk = align256(off_rA + size_t(np) * 4);
+    off_LAblk = align256(off_LBblk + size_t(Mt) * LEAF_BLOCKS * LEAF_BLOCK_FLOATS * 4);
+    bytes = align256(off_LAblk + size_t(Nt) * LEAF_BLOCKS * LEAF_BLOCK_FLOATS * 4);
   }
 };
+
+// Fills the leaf blocks of a factor buffer from its L^B and L^A planes
+// (solve.cu); run after every write of the planes.
+int build_leaf_blocks(const FactorLayout& fl, char* factors, cudaStream_t s);
 
 // Solve workspace: [status 256 B][X mp x np][E^T hi, lo: np x mp each]
 // [M hi, lo: mp x np each], fp32.  X holds W widened and, once an entry is
 // rounded, the value it was rounded at.  E^T is the error matrix transposed
 // (row = column index of W) so that it is K-major as the second operand of
-// M = L^B E; M is the stage-1 band product.
+// M = L^B E; M is the stage-1 band product.  The M hi plane doubles as E^T in
+// fp32 for the leaves: a leaf block reads back only E tiles written inside the
+// block, and M is written only by band products, which run between blocks.
 struct SolveLayout {
   int64_t mp, np;
   size_t off_status, off_X, off_EtH, off_EtL, off_MH, off_ML, bytes;

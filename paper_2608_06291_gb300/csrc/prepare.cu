@@ -303,6 +303,7 @@ int prepare_impl(const float* A, const float* B, int m, int n, float damp, void*
       rc = factor_one<double>(B, m, damp, (float*)(f + fl.off_LBH), (float*)(f + fl.off_LBL),
                               fl.mp, (float*)(f + fl.off_rB), workspace, pl, s);
   }
+  if (rc == BAKRON_OK) rc = build_leaf_blocks(fl, f, s);
   return rc;
 }
 

@@ -83,6 +83,41 @@ __global__ void k_copy_out(const float* X, int64_t np, int m, int n, float* out)
   out[idx] = X[r * np + c];
 }
 
+// Leaf blocks of a factor buffer (FactorLayout), one thread per stored float:
+// block d of tile row I of L^B is L^B[I, I-d], row-major for d = 0
+// (element (p, i) at p * LD + i) and k-major for d >= 1 (at i * LD + p); block
+// g of tile column J of L^A is L^A[J, J-g], k-major (element (q, j) at
+// j * LD + q).  Zero outside the matrix (I - d < 0) and in columns TILE..LD-1.
+__global__ void k_leaf_blocks(const float* hi, const float* lo, int64_t ld, int64_t T,
+                              bool row_major_diag, float* out) {
+  const int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (idx >= T * LEAF_BLOCKS * LEAF_BLOCK_FLOATS) return;
+  const int c = (int)(idx % LEAF_BLOCK_LD);
+  const int r = (int)((idx / LEAF_BLOCK_LD) % TILE);
+  const int d = (int)((idx / LEAF_BLOCK_FLOATS) % LEAF_BLOCKS);
+  const int64_t I = idx / ((int64_t)LEAF_BLOCK_FLOATS * LEAF_BLOCKS);
+  float v = 0.f;
+  if (c < TILE && I - d >= 0) {
+    const bool rm = row_major_diag && d == 0;
+    const int p = rm ? r : c, i = rm ? c : r;   // element (p, i) of the block
+    const int64_t o = (TILE * I + p) * ld + TILE * (I - d) + i;
+    v = hi[o] + lo[o];
+  }
+  out[idx] = v;
+}
+
+int build_leaf_blocks(const FactorLayout& fl, char* f, cudaStream_t s) {
+  const int64_t nb = fl.Mt * LEAF_BLOCKS * LEAF_BLOCK_FLOATS, na = fl.Nt * LEAF_BLOCKS * LEAF_BLOCK_FLOATS;
+  k_leaf_blocks<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(
+      (const float*)(f + fl.off_LBH), (const float*)(f + fl.off_LBL), fl.mp, fl.Mt, true,
+      (float*)(f + fl.off_LBblk));
+  k_leaf_blocks<<<(unsigned)((na + 255) / 256), 256, 0, s>>>(
+      (const float*)(f + fl.off_LAH), (const float*)(f + fl.off_LAL), fl.np, fl.Nt, false,
+      (float*)(f + fl.off_LAblk));
+  BK_CUDA_OK(cudaGetLastError());
+  return BAKRON_OK;
+}
+
 // ------------------------------------------------------------------ leaf
 // One CTA rounds one TILE x TILE tile whose inbound updates from all earlier
 // tiles are already in X (paper, the parallel anti-diagonal loop of Sec. 3.3,
@@ -132,11 +167,9 @@ struct LeafArgs {
   float* X;
   int64_t ldx;
   float *EtH, *EtL;
+  float* EtF;                  // E^T in fp32 (the leaves' own copy), same layout
   int64_t ldt;
-  const float *LBH, *LBL;
-  int64_t ldb;
-  const float *LAH, *LAL;
-  int64_t lda;
+  const float *LBblk, *LAblk;  // the factor buffer's leaf blocks
   const float *scales, *zeros;
   int G, gsz, qmax;
   uint8_t* codes;
@@ -144,12 +177,14 @@ struct LeafArgs {
 };
 
 constexpr int KM = 36;   // row stride of k-major product operands: float4 rows
+static_assert(KM == LEAF_BLOCK_LD, "the factor buffer's leaf blocks are copied as they are");
 
 // A leaf absorbs the errors of at most this many earlier anti-diagonals of
 // its block (Alg. 5 ranges of up to LEAF_WINDOW + 1 anti-diagonals are run
 // as such blocks of leaves), needing the E tiles (I - dp, J - g) with
 // 1 <= dp + g <= LEAF_WINDOW.
 constexpr int LEAF_WINDOW = 3;
+static_assert(LEAF_WINDOW + 1 == LEAF_BLOCKS, "a window needs the blocks L[I, I-1 .. I-LEAF_WINDOW]");
 constexpr int LEAF_WINDOW_TILES = (LEAF_WINDOW + 1) * (LEAF_WINDOW + 2) / 2 - 1;
 
 // Slot of E tile (I - dp, J - g) among a window-P leaf's tiles: row I first
@@ -158,13 +193,21 @@ __host__ __device__ constexpr int window_slot(int P, int dp, int g) {
   return dp == 0 ? g - 1 : P + (dp - 1) * P - (dp - 1) * (dp - 2) / 2 + g;
 }
 
+// (dp, g) of slot s (the inverse of window_slot).
+__host__ __device__ constexpr int window_dp(int P, int s) {
+  return s < P ? 0 : (s < 2 * P ? 1 : (s < 3 * P - 1 ? 2 : 3));
+}
+__host__ __device__ constexpr int window_g(int P, int s) {
+  return window_dp(P, s) == 0 ? s + 1 : s - window_slot(P, window_dp(P, s), 0);
+}
+
 // 32^3 products a window-P leaf forms before its wavefront (T1, the N_dp, U).
 __host__ __device__ constexpr int window_products(int P) { return 2 * P + P * (P + 1) / 2; }
 
 struct LeafSmem {
   float Xs[TILE][TILE];                   // W after inbound updates
   __align__(16) float LBs[TILE][36];      // stride 36: conflict-free float4 row reads
-  float LAs[TILE][TILE + 1];
+  __align__(16) float LA0[TILE][KM];      // LA0[j][q] = L^A[J,J][q][j]
   float T1s[TILE][TILE + 1];              // left neighbour's feedback: initial G (absorbing leaf)
   __align__(16) float Ebr[4][LEAF_ROWS_PADDED];   // errors of a step, by row (ring of 4 steps)
   float Part[4][LEAF_HELPERS][TILE];              // partial pre of a step (ring of 4 steps)
@@ -217,39 +260,23 @@ __device__ __forceinline__ void leaf_sync() {
   asm volatile("bar.sync 1, %0;" ::"n"(LEAF_THREADS) : "memory");
 }
 
-// Loads up to NT 32 x 32 tiles of hi/lo plane pairs into shared memory as
-// hi + lo, every load issued before the first sum.  Tile s is the block at
-// element offset base[s] of planes (hi[s], lo[s]) with row stride ld[s];
-// a tile that is not valid becomes zeros.  Element (r, c) goes to
-// dst[s][c * KM + r] (transpose) or dst[s][r * KM + c]; a null dst[s] is
-// skipped.  COHERENT: L2 loads (data written by earlier kernels or phases of
-// the solve).
-template <int NT, bool COHERENT>
-__device__ __forceinline__ void load_tiles(const float* const (&hi)[NT], const float* const (&lo)[NT],
-                                           const int64_t (&base)[NT], const int64_t (&ld)[NT],
-                                           const bool (&valid)[NT], float* const (&dst)[NT],
-                                           bool transpose, int t) {
-  float h[NT][LEAF_PER_THREAD], l[NT][LEAF_PER_THREAD];
+// 16-byte asynchronous copy global -> shared (L2 only); !valid writes zeros
+// and reads nothing.
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool valid) {
+  const unsigned d = (unsigned)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src),
+               "r"(valid ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
+// Copies one leaf block (TILE rows of KM floats) as it is; thread t of the leaf.
+__device__ __forceinline__ void copy_block(float* dst, const float* src, int t) {
+  constexpr int CHUNKS = TILE * KM / 4;
 #pragma unroll
-  for (int s = 0; s < NT; ++s) {
-#pragma unroll
-    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-      const int e = t + k * LEAF_THREADS;
-      const int64_t o = base[s] + (int64_t)(e / TILE) * ld[s] + e % TILE;
-      h[s][k] = valid[s] ? (COHERENT ? __ldcg(hi[s] + o) : hi[s][o]) : 0.f;
-      l[s][k] = valid[s] ? (COHERENT ? __ldcg(lo[s] + o) : lo[s][o]) : 0.f;
-    }
-  }
-#pragma unroll
-  for (int s = 0; s < NT; ++s) {
-    if (dst[s] == nullptr) continue;
-#pragma unroll
-    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-      const int e = t + k * LEAF_THREADS;
-      const int r = e / TILE, c = e % TILE;
-      dst[s][transpose ? c * KM + r : r * KM + c] = h[s][k] + l[s][k];
-    }
-  }
+  for (int c = t; c < CHUNKS; c += LEAF_THREADS) cp_async16(dst + 4 * c, src + 4 * c, true);
 }
 
 // Rounds tile (I, J); run by threads 0 .. LEAF_THREADS-1 of the CTA.  With
@@ -275,46 +302,18 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
   const int64_t r0 = (int64_t)I * TILE, c0 = (int64_t)J * TILE;
   // Factor blocks and the grid (read-only during the solve; the grid written
   // by the solve's first kernel, more than one kernel ago), loaded before
-  // waiting for the previous kernel.  Each batch issues all its loads before
-  // any is used, so their latencies overlap.
+  // waiting for the previous kernel; the factor blocks as asynchronous copies
+  // of the factor buffer's leaf blocks, which hold them in the layouts used
+  // here (LBs row-major, the others k-major, rows padded to KM).
   {
-    const float* const hi[2] = {a.LBH, a.LAH};
-    const float* const lo[2] = {a.LBL, a.LAL};
-    const int64_t base[2] = {r0 * a.ldb + r0, c0 * a.lda + c0};
-    const int64_t ld[2] = {a.ldb, a.lda};
-    const bool valid[2] = {true, true};
-    // LBs has row stride 36 = KM, LAs 33: the second tile is stored by hand below
-    float* const dst[2] = {&S.LBs[0][0], &S.u.pro.Et[0][0][0]};
-    load_tiles<2, false>(hi, lo, base, ld, valid, dst, false, t);
-  }
-  if (P >= 1) {
-    // sub-diagonal factor blocks L^A[J, J-g], L^B[I, I-dp], transposed to k-major
+    const float* lb = a.LBblk + (int64_t)I * LEAF_BLOCKS * LEAF_BLOCK_FLOATS;
+    const float* la = a.LAblk + (int64_t)J * LEAF_BLOCKS * LEAF_BLOCK_FLOATS;
+    copy_block(&S.LBs[0][0], lb, t);
+    copy_block(&S.LA0[0][0], la, t);
 #pragma unroll
-    for (int g0 = 1; g0 <= P; g0 += 3) {
-      constexpr int NB = 3;
-      const float* hi[NB];
-      const float* lo[NB];
-      int64_t base[NB], ld[NB];
-      bool valid[NB];
-      float* dst[NB];
-#pragma unroll
-      for (int s = 0; s < NB; ++s) {
-        const int g = g0 + s;
-        hi[s] = a.LAH; lo[s] = a.LAL; ld[s] = a.lda;
-        valid[s] = g <= P && J - g >= 0;
-        base[s] = valid[s] ? c0 * a.lda + c0 - (int64_t)TILE * g : 0;
-        dst[s] = g <= P ? &S.u.pro.LAt[g - 1][0][0] : nullptr;
-      }
-      load_tiles<NB, false>(hi, lo, base, ld, valid, dst, true, t);
-#pragma unroll
-      for (int s = 0; s < NB; ++s) {
-        const int dp = g0 + s;
-        hi[s] = a.LBH; lo[s] = a.LBL; ld[s] = a.ldb;
-        valid[s] = dp <= P && I - dp >= 0;
-        base[s] = valid[s] ? r0 * a.ldb + r0 - (int64_t)TILE * dp : 0;
-        dst[s] = dp <= P ? &S.u.pro.LBt[dp - 1][0][0] : nullptr;
-      }
-      load_tiles<NB, false>(hi, lo, base, ld, valid, dst, true, t);
+    for (int d = 1; d <= P; ++d) {
+      copy_block(&S.u.pro.LBt[d - 1][0][0], lb + d * LEAF_BLOCK_FLOATS, t);
+      copy_block(&S.u.pro.LAt[d - 1][0][0], la + d * LEAF_BLOCK_FLOATS, t);
     }
   }
   float scv[LEAF_PER_THREAD], zv[LEAF_PER_THREAD];
@@ -327,7 +326,6 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     scv[k] = real ? a.scales[og] : 1.f;
     zv[k] = real ? a.zeros[og] : 0.f;
   }
-  if (t < TILE * (36 - TILE)) S.LBs[t / (36 - TILE)][TILE + t % (36 - TILE)] = 0.f;  // padding rows
   if (PDL) {
     pdl_wait();
     pdl_trigger();
@@ -338,47 +336,29 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     const int e = t + k * LEAF_THREADS;
     xv[k] = __ldcg(a.X + (r0 + e / TILE) * a.ldx + c0 + e % TILE);
   }
-  leaf_sync();   // LAs staged in Et[0]
-#pragma unroll
-  for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-    const int e = t + k * LEAF_THREADS;
-    S.LAs[e / TILE][e % TILE] = S.u.pro.Et[0][e / TILE][e % TILE];
-  }
   if (P >= 1) {
-    leaf_sync();   // Et[0] free again
-    // errors of the window's tiles, k-major as E^T stores them, three at a time
+    // errors of the window's tiles (written by the leaves before this one in
+    // its block), k-major as E^T stores them: row j of slot s is the E^T row
+    // c0 - 32 g + j, columns r0 - 32 dp ..; tiles outside the matrix are zeros
     constexpr int NE = (P + 1) * (P + 2) / 2 - 1;   // E tiles of the window
+    constexpr int CH = TILE * TILE / 4;              // 16-byte chunks of a tile
+    static_assert(CH == 2 * LEAF_THREADS, "two chunks of every tile per thread");
 #pragma unroll
-    for (int s0 = 0; s0 < NE; s0 += 3) {
-      constexpr int NB = 3;
-      const float* const hi[NB] = {a.EtH, a.EtH, a.EtH};
-      const float* const lo[NB] = {a.EtL, a.EtL, a.EtL};
-      int64_t base[NB];
-      const int64_t ld[NB] = {a.ldt, a.ldt, a.ldt};
-      bool valid[NB];
-      float* dst[NB];
+    for (int sl = 0; sl < NE; ++sl) {
+      const int dp = window_dp(P, sl), g = window_g(P, sl);
+      const bool valid = I - dp >= 0 && J - g >= 0;
 #pragma unroll
-      for (int s = 0; s < NB; ++s) {
-        // slot s0 + s -> (dp, g)
-        int dp = 0, g = 0, idx = s0 + s;
-        if (idx < P) { dp = 0; g = idx + 1; }
-        else {
-          idx -= P;
-#pragma unroll
-          for (int d = 1; d <= LEAF_WINDOW; ++d) {
-            const int cnt = P - d + 1;
-            if (d <= P && dp == 0 && idx < cnt) { dp = d; g = idx; }
-            else if (d <= P && dp == 0) idx -= cnt;
-          }
-        }
-        valid[s] = s0 + s < NE && dp + g >= 1 && I - dp >= 0 && J - g >= 0;
-        // E[I - dp, J - g] k-major: row j of the tile is E^T row c0 - 32 g + j
-        base[s] = valid[s] ? (c0 - (int64_t)TILE * g) * a.ldt + r0 - (int64_t)TILE * dp : 0;
-        dst[s] = s0 + s < NE ? &S.u.pro.Et[s0 + s][0][0] : nullptr;
+      for (int h = 0; h < 2; ++h) {
+        const int c = t + LEAF_THREADS * h, j = c / (TILE / 4), i4 = 4 * (c % (TILE / 4));
+        const float* src =
+            valid ? a.EtF + (c0 - (int64_t)TILE * g + j) * a.ldt + r0 - (int64_t)TILE * dp + i4 : a.EtF;
+        cp_async16(&S.u.pro.Et[sl][j][i4], src, valid);
       }
-      load_tiles<NB, true>(hi, lo, base, ld, valid, dst, false, t);
     }
-    leaf_sync();
+  }
+  cp_async_wait_all();
+  leaf_sync();   // factor blocks and window tiles in shared memory
+  if (P >= 1) {
     // round 1: T1 and N_1 .. N_P in one pass over K (their terms interleave)
     const int pr = 4 * (t >> 4), pc = 2 * (t & 15);
     float acc[P + 1][4][2];
@@ -389,8 +369,8 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
 #pragma unroll 2
     for (int k = 0; k < TILE; ++k) {
       float b[P + 1][2];   // L^A[J, J-g][c][k] for this thread's two columns
-      b[0][0] = S.LAs[pc][k];
-      b[0][1] = S.LAs[pc + 1][k];
+      b[0][0] = S.LA0[k][pc];
+      b[0][1] = S.LA0[k][pc + 1];
 #pragma unroll
       for (int g = 1; g <= P; ++g) {
         b[g][0] = S.u.pro.LAt[g - 1][k][pc];
@@ -488,9 +468,9 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     // ------------------------------------------------ the chain
     const bool col_real = (c0 + q) < a.n;
     const int rows_real = a.m - (int)r0;     // rows p < rows_real are inside W
-    const float la1 = q >= 1 ? S.LAs[q][q - 1] : 0.f;
-    const float la2 = q >= 2 ? S.LAs[q][q - 2] : 0.f;
-    const float la3 = q >= 3 ? S.LAs[q][q - 3] : 0.f;
+    const float la1 = q >= 1 ? S.LA0[q - 1][q] : 0.f;
+    const float la2 = q >= 2 ? S.LA0[q - 2][q] : 0.f;
+    const float la3 = q >= 3 ? S.LA0[q - 3][q] : 0.f;
     const float fq = (float)a.qmax;
     // Rounding to the nearest integer (ties to even) by the shift R = 1.5 * 2^23:
     // for |v| < 2^22, fl(v + R) - R is v rounded to an integer, and the clamp
@@ -570,7 +550,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     // step s = 8b + 2v - 2 (+1) brings is in slot 2v - r (+1) mod 32
     float LAr[TILE];
 #pragma unroll
-    for (int sl = 0; sl < TILE; ++sl) LAr[sl] = S.LAs[q][(sl - 2 - i0) & (TILE - 1)];
+    for (int sl = 0; sl < TILE; ++sl) LAr[sl] = S.LA0[(sl - 2 - i0) & (TILE - 1)][q];
     float Gg[LEAF_ROWS_PER_HELPER];
 #pragma unroll
     for (int r = 0; r < LEAF_ROWS_PER_HELPER; ++r)
@@ -672,6 +652,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     const int64_t o = (c0 + r) * a.ldt + r0 + c;
     a.EtH[o] = hi;
     a.EtL[o] = ev - hi;
+    a.EtF[o] = ev;
   }
   if (bad) raise_status(a.status, BAKRON_ERR_NONFINITE);
   leaf_sync();   // shared memory free for the next tile of this CTA
@@ -1279,8 +1260,10 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
   a.status = (int*)(ws + sl.off_status);
   a.s = s;
   a.rc = BAKRON_OK;
-  a.la = LeafArgs{a.Mt, a.Nt, m, n, a.X, a.np, a.EtH, a.EtL, a.mp, a.LBH, a.LBL, a.mp,
-                  a.LAH, a.LAL, a.np, scales, zeros, a.G, a.gsz, a.qmax, codes, a.status};
+  // the leaves' fp32 E^T shares the M hi plane (see SolveLayout)
+  a.la = LeafArgs{a.Mt, a.Nt, m, n, a.X, a.np, a.EtH, a.EtL, a.MH, a.mp,
+                  (const float*)(f + fl.off_LBblk), (const float*)(f + fl.off_LAblk),
+                  scales, zeros, a.G, a.gsz, a.qmax, codes, a.status};
   a.ba = BandArgs{a.LBH, a.LBL, a.mp, a.EtH, a.EtL, a.mp, a.LAH, a.LAL, a.np,
                   a.MH, a.ML, a.np, a.X, a.np};
   a.profiling = profiling_on();
