@@ -23,6 +23,8 @@
 #include "tune.cuh"
 #include <stdlib.h>
 
+#include <type_traits>
+
 #include <mutex>
 
 namespace bakron {
@@ -326,46 +328,40 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     scv[k] = real ? a.scales[og] : 1.f;
     zv[k] = real ? a.zeros[og] : 0.f;
   }
-  if (PDL) {
-    pdl_wait();
-    pdl_trigger();
-  }
-  float xv[LEAF_PER_THREAD];
+  // The window's products.  Thread t forms rows pr .. pr+3, columns pc,
+  // pc+1 of each output.  Round 1 accumulates acc[dp] = N_dp (acc[0] = T1)
+  // over the window's E tiles; round 2 u = U = sum_dp L^B[I,I-dp] N_dp, with
+  // N_dp kept in slot dp - 1.  E tiles of anti-diagonals K-2 and before
+  // (dp + g >= 2) were written by kernels that had completed when this one
+  // was launched, so their part runs before the wait for the previous kernel
+  // (overlapping it); only E[I, J-1] and E[I-1, J] come after.
+  const int pr = 4 * (t >> 4), pc = 2 * (t & 15);
+  float acc[P + 1][4][2];
+  float u[4][2];
 #pragma unroll
-  for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-    const int e = t + k * LEAF_THREADS;
-    xv[k] = __ldcg(a.X + (r0 + e / TILE) * a.ldx + c0 + e % TILE);
-  }
-  if (P >= 1) {
-    // errors of the window's tiles (written by the leaves before this one in
-    // its block), k-major as E^T stores them: row j of slot s is the E^T row
-    // c0 - 32 g + j, columns r0 - 32 dp ..; tiles outside the matrix are zeros
-    constexpr int NE = (P + 1) * (P + 2) / 2 - 1;   // E tiles of the window
-    constexpr int CH = TILE * TILE / 4;              // 16-byte chunks of a tile
+  for (int o = 0; o <= P; ++o)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) acc[o][i][0] = acc[o][i][1] = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) u[i][0] = u[i][1] = 0.f;
+  // copies E[I-dp, J-g] into slot sl (k-major as E^T stores it: row j of the
+  // slot is the E^T row c0 - 32 g + j, columns r0 - 32 dp ..); zeros outside
+  // the matrix
+  auto fetch_e = [&](int sl, int dp, int g) {
+    constexpr int CH = TILE * TILE / 4;   // 16-byte chunks of a tile
     static_assert(CH == 2 * LEAF_THREADS, "two chunks of every tile per thread");
+    const bool valid = I - dp >= 0 && J - g >= 0;
 #pragma unroll
-    for (int sl = 0; sl < NE; ++sl) {
-      const int dp = window_dp(P, sl), g = window_g(P, sl);
-      const bool valid = I - dp >= 0 && J - g >= 0;
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int c = t + LEAF_THREADS * h, j = c / (TILE / 4), i4 = 4 * (c % (TILE / 4));
-        const float* src =
-            valid ? a.EtF + (c0 - (int64_t)TILE * g + j) * a.ldt + r0 - (int64_t)TILE * dp + i4 : a.EtF;
-        cp_async16(&S.u.pro.Et[sl][j][i4], src, valid);
-      }
+    for (int h = 0; h < 2; ++h) {
+      const int c = t + LEAF_THREADS * h, j = c / (TILE / 4), i4 = 4 * (c % (TILE / 4));
+      const float* src =
+          valid ? a.EtF + (c0 - (int64_t)TILE * g + j) * a.ldt + r0 - (int64_t)TILE * dp + i4 : a.EtF;
+      cp_async16(&S.u.pro.Et[sl][j][i4], src, valid);
     }
-  }
-  cp_async_wait_all();
-  leaf_sync();   // factor blocks and window tiles in shared memory
-  if (P >= 1) {
-    // round 1: T1 and N_1 .. N_P in one pass over K (their terms interleave)
-    const int pr = 4 * (t >> 4), pc = 2 * (t & 15);
-    float acc[P + 1][4][2];
-#pragma unroll
-    for (int o = 0; o <= P; ++o)
-#pragma unroll
-      for (int i = 0; i < 4; ++i) acc[o][i][0] = acc[o][i][1] = 0.f;
+  };
+  // round 1 over the window's tiles with (dp + g >= 2) == OLD
+  auto round1 = [&](auto old_tag) {
+    constexpr bool OLD = decltype(old_tag)::value;
 #pragma unroll 2
     for (int k = 0; k < TILE; ++k) {
       float b[P + 1][2];   // L^A[J, J-g][c][k] for this thread's two columns
@@ -380,6 +376,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
       for (int dp = 0; dp <= P; ++dp) {
 #pragma unroll
         for (int g = (dp == 0 ? 1 : 0); g + dp <= P; ++g) {
+          if ((dp + g >= 2) != OLD) continue;
           const float4 av = *reinterpret_cast<const float4*>(&S.u.pro.Et[window_slot(P, dp, g)][k][pr]);
           acc[dp][0][0] = fmaf(av.x, b[g][0], acc[dp][0][0]);
           acc[dp][0][1] = fmaf(av.x, b[g][1], acc[dp][0][1]);
@@ -392,26 +389,14 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
         }
       }
     }
-    leaf_sync();   // the E tiles are read: their slots take N_dp and U
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      S.T1s[pr + i][pc] = acc[0][i][0];
-      S.T1s[pr + i][pc + 1] = acc[0][i][1];
-#pragma unroll
-      for (int dp = 1; dp <= P; ++dp) {
-        S.u.pro.Et[dp - 1][pr + i][pc] = acc[dp][i][0];
-        S.u.pro.Et[dp - 1][pr + i][pc + 1] = acc[dp][i][1];
-      }
-    }
-    leaf_sync();
-    // round 2: U[p][q] = sum_dp sum_i L^B[I,I-dp][p][i] N_dp[i][q], into slot P
-    float u[4][2];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) u[i][0] = u[i][1] = 0.f;
+  };
+  // round 2 over N_dp, dp in [d_lo, d_hi]
+  auto round2 = [&](int d_lo, int d_hi) {
 #pragma unroll 2
     for (int k = 0; k < TILE; ++k) {
 #pragma unroll
       for (int dp = 1; dp <= P; ++dp) {
+        if (dp < d_lo || dp > d_hi) continue;
         const float4 av = *reinterpret_cast<const float4*>(&S.u.pro.LBt[dp - 1][k][pr]);
         const float b0 = S.u.pro.Et[dp - 1][k][pc], b1 = S.u.pro.Et[dp - 1][k][pc + 1];
         u[0][0] = fmaf(av.x, b0, u[0][0]);
@@ -424,6 +409,60 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
         u[3][1] = fmaf(av.w, b1, u[3][1]);
       }
     }
+  };
+  // stores acc[dp] (N_dp) into slot dp - 1
+  auto store_n = [&](int dp) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      S.u.pro.Et[dp - 1][pr + i][pc] = acc[dp][i][0];
+      S.u.pro.Et[dp - 1][pr + i][pc + 1] = acc[dp][i][1];
+    }
+  };
+  if (P >= 2) {
+    // the part of the older tiles: N_2 .. N_P are complete after it
+#pragma unroll
+    for (int sl = 0; sl < (P + 1) * (P + 2) / 2 - 1; ++sl)
+      if (window_dp(P, sl) + window_g(P, sl) >= 2) fetch_e(sl, window_dp(P, sl), window_g(P, sl));
+    cp_async_wait_all();
+    leaf_sync();
+    round1(std::true_type());
+    leaf_sync();   // older tiles read: slots 1 .. P-1 take N_2 .. N_P
+#pragma unroll
+    for (int dp = 2; dp <= P; ++dp) store_n(dp);
+    leaf_sync();
+    round2(2, P);
+  }
+  if (PDL) {
+    pdl_wait();
+    pdl_trigger();
+  }
+  float xv[LEAF_PER_THREAD];
+#pragma unroll
+  for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+    const int e = t + k * LEAF_THREADS;
+    xv[k] = __ldcg(a.X + (r0 + e / TILE) * a.ldx + c0 + e % TILE);
+  }
+  if (P >= 1) {
+    // the newest tiles, E[I, J-1] (slot 0) and E[I-1, J] (slot P); slots 1 ..
+    // P-1 hold N_2 .. N_P, which round 2 has read
+    fetch_e(window_slot(P, 0, 1), 0, 1);
+    fetch_e(window_slot(P, 1, 0), 1, 0);
+  }
+  cp_async_wait_all();
+  leaf_sync();   // factor blocks and window tiles in shared memory
+  if (P >= 1) {
+    static_assert(window_slot(1, 0, 1) == 0 && window_slot(2, 1, 0) == 2 && window_slot(3, 1, 0) == 3,
+                  "newest tiles in slots 0 and P");
+    round1(std::false_type());
+    leaf_sync();   // the newest tiles are read: slot 0 takes N_1, slot P takes U
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      S.T1s[pr + i][pc] = acc[0][i][0];
+      S.T1s[pr + i][pc + 1] = acc[0][i][1];
+    }
+    store_n(1);
+    leaf_sync();
+    round2(1, 1);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       S.u.pro.Et[P][pr + i][pc] = u[i][0];
