@@ -26,7 +26,10 @@
 // stages: each 32-wide stage is accumulated afresh in one of four TMEM
 // accumulators and added, in fp32 round-to-nearest, into registers by the two
 // warps that own its 32-lane quarter (64 columns each, tcgen05.ld), while the
-// MMAs of the next stages run.  One 128 x 128 output block per CTA, K staged
+// MMAs of the next stages run.  The finished block goes out through shared
+// memory (the freed ring, in the tensor maps' 128-byte swizzled layout) by
+// TMA: stage 1 stores M as hi/lo planes, stage 2 adds into X with a TMA
+// reduction, one 32 x 32 tile of S2 at a time.  One 128 x 128 output block per CTA, K staged
 // 32 at a time through a 3-deep shared-memory ring.  The grid covers exactly
 // the bounding box of the output blocks that have work (rows from row0).
 // Every wait is bounded: a timed-out wait records BAKRON_ERR_TIMEOUT and the
@@ -128,6 +131,26 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
 
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
 // 128 bytes, 8-row core groups 1024 bytes apart (SBO), version 1.
+// TMA store of a box from shared memory, and TMA reduce-add of a box into
+// global memory (fp32 add at L2), both tracked as a bulk group of the thread.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(smem_u32(src))
+               : "memory");
+}
+__device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* map, const void* src, int x, int y) {
+  asm volatile(
+      "cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(x), "r"(y), "r"(smem_u32(src))
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit_and_wait() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
   uint64_t d = 0;
   d |= (uint64_t)((addr & 0x3FFFF) >> 4);            // start address
@@ -252,6 +275,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUtensorMap mapAl,
           const __grid_constant__ CUtensorMap mapBh, const __grid_constant__ CUtensorMap mapBl,
           const __grid_constant__ CUtensorMap mapBh4, const __grid_constant__ CUtensorMap mapBl4,
+          const __grid_constant__ CUtensorMap mapOh, const __grid_constant__ CUtensorMap mapOl,
           const TcParams P) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // 1024-byte alignment for the 128-byte swizzle atoms
@@ -281,6 +305,8 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBl)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBh4)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBl4)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapOh)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapOl)) : "memory");
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -445,7 +471,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
       int ok = 1;
       if (lane == 0) {
         ok = mbar_wait(&accF[a], (uint32_t)(i / NACC) & 1u, P.spin_cycles) ? 1 : 0;
-        if (!ok) raise_status(P.status, BAKRON_ERR_TIMEOUT);
+        if (!ok) { raise_status(P.status, BAKRON_ERR_TIMEOUT); *abort_flag = 1; }
         if (*abort_flag) ok = 0;
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -465,44 +491,70 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
       __syncwarp();
       if (lane == 0) mbar_arrive(&accE[a]);
     }
-    const int64_t gi = (int64_t)blk.rb * BM + row;
+    if (P.mode == MODE_DENSE) {
+      const int64_t gi = (int64_t)blk.rb * BM + row;
 #pragma unroll
-    for (int c = 0; c < EPI_COLS / 32; ++c) {
-      if (!write) break;
-      const float* v = &acc[c * 32];
-      const int64_t gj = (int64_t)blk.cb * BN + c0 + c * 32;
-      if (P.mode == MODE_DENSE) {
+      for (int c = 0; c < EPI_COLS / 32; ++c) {
+        if (!write) break;
+        const float* v = &acc[c * 32];
+        const int64_t gj = (int64_t)blk.cb * BN + c0 + c * 32;
         float4* o = reinterpret_cast<float4*>(P.out_hi + gi * P.ldo + gj);
 #pragma unroll
         for (int u = 0; u < 8; ++u) o[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
-      } else if (P.mode == MODE_STAGE1) {
-        float4* oh = reinterpret_cast<float4*>(P.out_hi + gi * P.ldo + gj);
-        float4* ol = reinterpret_cast<float4*>(P.out_lo + gi * P.ldo + gj);
+      }
+    } else {
+      // Every MMA has completed (the last accumulator was committed after
+      // them), so the ring is free: stage the block as 32-column boxes of 128
+      // rows, box (plane, c) at smem + (plane * 4 + c) * 16 KiB, 16-byte chunk
+      // u of row r at chunk u ^ (r & 7) (the 128-byte swizzle of the maps).
+      if (write) {
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          float hi[4], lo[4];
+        for (int c = 0; c < EPI_COLS / 32; ++c) {
+          const int cb32 = (c0 >> 5) + c;     // 32-column box of this chunk
+          const float* v = &acc[c * 32];
+          unsigned char* rowh = smem + cb32 * TILE_BYTES + row * 128;
+          unsigned char* rowl = rowh + 4 * TILE_BYTES;
 #pragma unroll
-          for (int w2 = 0; w2 < 4; ++w2) {
-            hi[w2] = tf32_hi(v[4 * u + w2]);
-            lo[w2] = v[4 * u + w2] - hi[w2];
+          for (int u = 0; u < 8; ++u) {
+            const int off = ((u ^ (row & 7)) << 4);
+            if (P.mode == MODE_STAGE1) {
+              float hi[4], lo[4];
+#pragma unroll
+              for (int w2 = 0; w2 < 4; ++w2) {
+                hi[w2] = tf32_hi(v[4 * u + w2]);
+                lo[w2] = v[4 * u + w2] - hi[w2];
+              }
+              *reinterpret_cast<float4*>(rowh + off) = make_float4(hi[0], hi[1], hi[2], hi[3]);
+              *reinterpret_cast<float4*>(rowl + off) = make_float4(lo[0], lo[1], lo[2], lo[3]);
+            } else {
+              *reinterpret_cast<float4*>(rowh + off) =
+                  make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+            }
           }
-          oh[u] = make_float4(hi[0], hi[1], hi[2], hi[3]);
-          ol[u] = make_float4(lo[0], lo[1], lo[2], lo[3]);
         }
-      } else {
-        // stage 2: add into X only on tiles of the band S2
-        const int I = (int)(gi / 32), J = (int)(gj / 32);
-        if (nk == 0 || I >= P.Mt || J >= P.Nt || I + J < P.h || I + J >= P.l) continue;
-        float4* o = reinterpret_cast<float4*>(P.X + gi * P.ldo + gj);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // visible to the TMA unit
+      }
+      asm volatile("bar.sync 2, %0;" ::"n"(EPI_WARPS * 32) : "memory");   // the epilogue warps
+      if (warp == 2 && lane == 0 && !*abort_flag) {
+        const int x0 = blk.cb * BN, y0 = blk.rb * BM;
+        if (P.mode == MODE_STAGE1) {
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          float4 x = o[u];
-          x.x += v[4 * u];
-          x.y += v[4 * u + 1];
-          x.z += v[4 * u + 2];
-          x.w += v[4 * u + 3];
-          o[u] = x;
+          for (int c = 0; c < 4; ++c) {
+            tma_store_2d(&mapOh, smem + c * TILE_BYTES, x0 + 32 * c, y0);
+            tma_store_2d(&mapOl, smem + (4 + c) * TILE_BYTES, x0 + 32 * c, y0);
+          }
+        } else if (nk > 0) {
+          // X += the block's tiles that lie in S2 (32 x 32 boxes: rows 32 ti
+          // .. of box c start 4 KiB apart, whole swizzle periods)
+          for (int ti = 0; ti < 4; ++ti) {
+            for (int c = 0; c < 4; ++c) {
+              const int I = 4 * blk.rb + ti, J = 4 * blk.cb + c;
+              if (I >= P.Mt || J >= P.Nt || I + J < P.h || I + J >= P.l) continue;
+              tma_reduce_add_2d(&mapOh, smem + c * TILE_BYTES + ti * 4096, 32 * J, 32 * I);
+            }
+          }
         }
+        bulk_commit_and_wait();   // complete before the CTA (and its shared memory) goes
       }
     }
   }
@@ -592,6 +644,7 @@ bool tc_band_maps(TcMaps& maps, const TcOperands& op) {
   ok &= make_map(&maps.Ml, op.ML, op.mp, op.np, op.np, BM);
   ok &= make_map(&maps.LAh, op.LAH, op.np, op.np, op.np, BN);
   ok &= make_map(&maps.LAl, op.LAL, op.np, op.np, op.np, BN);
+  ok &= make_map(&maps.X32, op.X, op.mp, op.np, op.np, 32);   // stage-2 reduce target
   return ok;
 }
 
@@ -623,10 +676,10 @@ int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, in
   cudaError_t e;
   if (stage == 1)
     e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.LBh, maps.LBl, maps.Eth,
-                   maps.Etl, maps.Eth4, maps.Etl4, P);
+                   maps.Etl, maps.Eth4, maps.Etl4, maps.Mh, maps.Ml, P);
   else
     e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.Mh, maps.Ml, maps.LAh,
-                   maps.LAl, maps.LAh, maps.LAl, P);
+                   maps.LAl, maps.LAh, maps.LAl, maps.X32, maps.X32, P);
   return e == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
 }
 
@@ -665,7 +718,7 @@ extern "C" int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C,
   P.status = status;
   P.spin_cycles = spin_cycles_from_env();
   dim3 grid(N / BN, M / BM);
-  k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(mA, mAl, mB, mBl, mB, mBl, P);
+  k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(mA, mAl, mB, mBl, mB, mBl, mB, mBl, P);
   BK_CUDA_OK(cudaGetLastError());
   return bakron_read_status(workspace, stream);
 }

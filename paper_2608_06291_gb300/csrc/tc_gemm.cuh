@@ -19,6 +19,7 @@ struct TcOperands {
 struct TcMaps {
   CUtensorMap LBh, LBl, Eth, Etl, Mh, Ml, LAh, LAl;
   CUtensorMap Eth4, Etl4;   // E^T planes in 128-row boxes (whole stage-1 B operand)
+  CUtensorMap X32;          // X in 32 x 32 boxes: stage-2 TMA reduce-add target
 };
 
 bool tc_band_maps(TcMaps& maps, const TcOperands& op);
