@@ -93,6 +93,13 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
                : "memory");
 }
 
+// Adds to the bytes the current phase waits for, without arriving.
+__device__ __forceinline__ void mbar_expect_tx_only(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
@@ -332,7 +339,26 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = *tmem_slot;
-  // everything above touched no global memory: now wait for the previous kernel
+  // The factor operand (stage 1: A = L^B; stage 2: B = L^A) is read-only
+  // during the solve: its part of the first ring slots is loaded before the
+  // wait for the previous kernel, whose output (E^T or M) is the other one.
+  const int npre = blk.nk < STAGES ? blk.nk : STAGES;
+  const bool a_static = P.mode != MODE_STAGE2;
+  if (warp == 0 && lane == 0) {
+    for (int i = 0; i < npre; ++i) {
+      unsigned char* st = smem + i * STAGE_BYTES;
+      const int kt = blk.k0 + i;
+      mbar_expect_tx_only(&full[i], 2 * TILE_BYTES);
+      if (a_static) {
+        tma_load_2d(st, &mapAh, &full[i], kt * BK, blk.rb * BM);
+        tma_load_2d(st + TILE_BYTES, &mapAl, &full[i], kt * BK, blk.rb * BM);
+      } else {
+        tma_load_2d(st + 2 * TILE_BYTES, &mapBh, &full[i], kt * BK, blk.cb * BN);
+        tma_load_2d(st + 3 * TILE_BYTES, &mapBl, &full[i], kt * BK, blk.cb * BN);
+      }
+    }
+  }
+  // the rest waits for the previous kernel
   pdl_wait();
   pdl_trigger();
   const long long drain = 4000000000LL;   // ~2 s at 2 GHz: wind-down bound
@@ -349,13 +375,19 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok || *abort_flag) {
         if (lane == 0 && !ok) { raise_status(P.status, BAKRON_ERR_TIMEOUT); *abort_flag = 1; }
+        // slots loaded in part before the wait: arrive, so that their phase
+        // completes once those copies land (the drain below waits for them)
+        if (lane == 0)
+          for (int j = i; j < npre; ++j) mbar_arrive(&full[j]);
         break;
       }
       unsigned char* st = smem + s * STAGE_BYTES;
       unsigned char *a_hi = st, *a_lo = st + TILE_BYTES, *b_hi = st + 2 * TILE_BYTES,
                     *b_lo = st + 3 * TILE_BYTES;
       const int kt = blk.k0 + i;            // K tile index (32 wide)
-      uint32_t bytes = 2 * TILE_BYTES;      // A hi + A lo always loaded
+      const bool pre = i < npre;            // the factor operand is already on its way
+      const bool load_a = !(pre && a_static), load_b = !(pre && !a_static);
+      uint32_t bytes = load_a ? 2 * TILE_BYTES : 0u;   // A hi + A lo
       unsigned valid = 0xF;                 // stage 1: B sub-tiles in the band
       if (P.mode == MODE_STAGE1) {
         valid = 0;
@@ -377,14 +409,17 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();
         bytes += 2u * 4096u * (uint32_t)__popc(valid);
-      } else {
+      } else if (load_b) {
         bytes += 2 * TILE_BYTES;
       }
       if (lane == 0) {
         mbar_expect_tx(&full[s], bytes);
-        tma_load_2d(a_hi, &mapAh, &full[s], kt * BK, blk.rb * BM);
-        tma_load_2d(a_lo, &mapAl, &full[s], kt * BK, blk.rb * BM);
-        if (P.mode == MODE_STAGE1 && valid == 0xFu) {   // inside the band: one box per plane
+        if (load_a) {
+          tma_load_2d(a_hi, &mapAh, &full[s], kt * BK, blk.rb * BM);
+          tma_load_2d(a_lo, &mapAl, &full[s], kt * BK, blk.rb * BM);
+        }
+        if (!load_b) {
+        } else if (P.mode == MODE_STAGE1 && valid == 0xFu) {   // inside the band: one box per plane
           tma_load_2d(b_hi, &mapBh4, &full[s], kt * BK, blk.cb * BN);
           tma_load_2d(b_lo, &mapBl4, &full[s], kt * BK, blk.cb * BN);
         } else if (P.mode == MODE_STAGE1) {
@@ -404,8 +439,9 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
     }
     // drain: every copy this warp issued has landed before the CTA winds down
     if (lane == 0) {
-      const int first = issued > STAGES ? issued - STAGES : 0;
-      for (int i = first; i < issued; ++i) {
+      const int last = issued > npre ? issued : npre;
+      const int first = last > STAGES ? last - STAGES : 0;
+      for (int i = first; i < last; ++i) {
         if (!mbar_wait(&full[i % STAGES], (uint32_t)(i / STAGES) & 1u, drain))
           raise_status(P.status, BAKRON_ERR_TIMEOUT);
       }
