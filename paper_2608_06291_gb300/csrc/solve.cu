@@ -170,6 +170,7 @@ struct LeafArgs {
   int64_t ldx;
   float *EtH, *EtL;
   float* EtF;                  // E^T in fp32 (the leaves' own copy), same layout
+  float* Gout;                 // final G of every tile, X's layout (row i, column q)
   int64_t ldt;
   const float *LBblk, *LAblk;  // the factor buffer's leaf blocks
   const float *scales, *zeros;
@@ -183,28 +184,14 @@ static_assert(KM == LEAF_BLOCK_LD, "the factor buffer's leaf blocks are copied a
 
 // A leaf absorbs the errors of at most this many earlier anti-diagonals of
 // its block (Alg. 5 ranges of up to LEAF_WINDOW + 1 anti-diagonals are run
-// as such blocks of leaves), needing the E tiles (I - dp, J - g) with
-// 1 <= dp + g <= LEAF_WINDOW.
+// as such blocks of leaves), through the E tiles (I, J - g) and the final G
+// of the tiles (I - dp, J), 1 <= g, dp <= LEAF_WINDOW.
 constexpr int LEAF_WINDOW = 3;
 static_assert(LEAF_WINDOW + 1 == LEAF_BLOCKS, "a window needs the blocks L[I, I-1 .. I-LEAF_WINDOW]");
-constexpr int LEAF_WINDOW_TILES = (LEAF_WINDOW + 1) * (LEAF_WINDOW + 2) / 2 - 1;
+constexpr int LEAF_WINDOW_TILES = 2 * LEAF_WINDOW;   // E[I, J-g] and G[I-dp, J]
 
-// Slot of E tile (I - dp, J - g) among a window-P leaf's tiles: row I first
-// (g = 1..P), then rows I - 1, I - 2, ... (g = 0..P - dp).
-__host__ __device__ constexpr int window_slot(int P, int dp, int g) {
-  return dp == 0 ? g - 1 : P + (dp - 1) * P - (dp - 1) * (dp - 2) / 2 + g;
-}
-
-// (dp, g) of slot s (the inverse of window_slot).
-__host__ __device__ constexpr int window_dp(int P, int s) {
-  return s < P ? 0 : (s < 2 * P ? 1 : (s < 3 * P - 1 ? 2 : 3));
-}
-__host__ __device__ constexpr int window_g(int P, int s) {
-  return window_dp(P, s) == 0 ? s + 1 : s - window_slot(P, window_dp(P, s), 0);
-}
-
-// 32^3 products a window-P leaf forms before its wavefront (T1, the N_dp, U).
-__host__ __device__ constexpr int window_products(int P) { return 2 * P + P * (P + 1) / 2; }
+// 32^3 products a window-P leaf forms before its wavefront (T1 and U).
+__host__ __device__ constexpr int window_products(int P) { return 2 * P; }
 
 struct LeafSmem {
   float Xs[TILE][TILE];                   // W after inbound updates
@@ -216,8 +203,8 @@ struct LeafSmem {
   float4 Lsub[TILE];                              // (L^B[p][p-1], L^B[p][p-2], L^B[p][p-3], 0)
   union {
     struct {   // prologue of an absorbing leaf: k-major product operands
-      // E[I - dp, J - g] for the window's (dp, g), Et[.][j][i] = E[..][i][j];
-      // later the N_dp and U of the second round
+      // slots 0 .. LEAF_WINDOW-1: E[I, J-g] k-major, Et[g-1][j][i] = E[..][i][j];
+      // slots LEAF_WINDOW ..: G[I-dp, J] as stored, Et[LEAF_WINDOW+dp-1][i][q]
       __align__(16) float Et[LEAF_WINDOW_TILES][TILE][KM];
       __align__(16) float LAt[LEAF_WINDOW][TILE][KM];   // LAt[g-1][j][q] = L^A[J, J-g][q][j]
       __align__(16) float LBt[LEAF_WINDOW][TILE][KM];   // LBt[dp-1][i][p] = L^B[I, I-dp][p][i]
@@ -294,8 +281,9 @@ __device__ __forceinline__ void copy_block(float* dst, const float* src, int t) 
 // (which the wavefront multiplies by L^B[I,I] anyway):
 //     T1 = sum_g E[I,J-g] L^A[J,J-g]^T.
 // The others are added to X before the wavefront:
-//     U = sum_dp L^B[I,I-dp] N_dp,   N_dp = sum_g E[I-dp,J-g] L^A[J,J-g]^T.
-// Tiles outside the matrix (I - dp < 0 or J - g < 0) are zeros.
+//     U = sum_dp L^B[I,I-dp] N_dp,   N_dp = sum_g E[I-dp,J-g] L^A[J,J-g]^T,
+// and N_dp is the final G of tile (I - dp, J), which that tile's leaf leaves
+// behind (its window is P - dp).  Tiles outside the matrix are zeros.
 template <bool PDL, int P>
 __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafSmem& S) {
   static_assert(P >= 0 && P <= LEAF_WINDOW, "window");
@@ -328,162 +316,112 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     scv[k] = real ? a.scales[og] : 1.f;
     zv[k] = real ? a.zeros[og] : 0.f;
   }
-  // The window's products.  Thread t forms rows pr .. pr+3, columns pc,
-  // pc+1 of each output.  Round 1 accumulates acc[dp] = N_dp (acc[0] = T1)
-  // over the window's E tiles; round 2 u = U = sum_dp L^B[I,I-dp] N_dp, with
-  // N_dp kept in slot dp - 1.  E tiles of anti-diagonals K-2 and before
-  // (dp + g >= 2) were written by kernels that had completed when this one
-  // was launched, so their part runs before the wait for the previous kernel
-  // (overlapping it); only E[I, J-1] and E[I-1, J] come after.
+  // The window.  N_dp of this tile (the errors of row I - dp of the window
+  // seen from column block J) equals the final G of tile (I - dp, J), which
+  // sits at position P - dp of the same block: every leaf leaves its final G
+  // in the Gout plane.  So
+  //     T1 = sum_{g=1..P} E[I, J-g] L^A[J, J-g]^T,
+  //     U  = sum_{dp=1..P} L^B[I, I-dp] G[I-dp, J],
+  // 2P products of 32^3.  Terms of tiles two or more anti-diagonals back
+  // (g >= 2, dp >= 2) were written by kernels that had completed when this
+  // one was launched: they run before the wait for the previous kernel
+  // (overlapping it); E[I, J-1] and G[I-1, J] come after.  Thread t forms
+  // rows pr .. pr+3, columns pc, pc+1 of T1 and U.
   const int pr = 4 * (t >> 4), pc = 2 * (t & 15);
-  float acc[P + 1][4][2];
-  float u[4][2];
+  float t1[4][2], u[4][2];
 #pragma unroll
-  for (int o = 0; o <= P; ++o)
-#pragma unroll
-    for (int i = 0; i < 4; ++i) acc[o][i][0] = acc[o][i][1] = 0.f;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) u[i][0] = u[i][1] = 0.f;
-  // copies E[I-dp, J-g] into slot sl (k-major as E^T stores it: row j of the
-  // slot is the E^T row c0 - 32 g + j, columns r0 - 32 dp ..); zeros outside
-  // the matrix
-  auto fetch_e = [&](int sl, int dp, int g) {
+  for (int i = 0; i < 4; ++i) t1[i][0] = t1[i][1] = u[i][0] = u[i][1] = 0.f;
+  // E[I, J-g] into slot g - 1, k-major as E^T stores it (row j of the slot is
+  // the E^T row c0 - 32 g + j, columns r0 ..); G[I-dp, J] into slot
+  // LEAF_WINDOW + dp - 1 as stored (row i, columns c0 ..); zeros outside the
+  // matrix
+  auto fetch = [&](bool is_e, int d) {
     constexpr int CH = TILE * TILE / 4;   // 16-byte chunks of a tile
     static_assert(CH == 2 * LEAF_THREADS, "two chunks of every tile per thread");
-    const bool valid = I - dp >= 0 && J - g >= 0;
+    const bool valid = is_e ? J - d >= 0 : I - d >= 0;
+    const int sl = is_e ? d - 1 : LEAF_WINDOW + d - 1;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       const int c = t + LEAF_THREADS * h, j = c / (TILE / 4), i4 = 4 * (c % (TILE / 4));
       const float* src =
-          valid ? a.EtF + (c0 - (int64_t)TILE * g + j) * a.ldt + r0 - (int64_t)TILE * dp + i4 : a.EtF;
+          !valid ? a.EtF
+          : is_e ? a.EtF + (c0 - (int64_t)TILE * d + j) * a.ldt + r0 + i4
+                 : a.Gout + (r0 - (int64_t)TILE * d + j) * a.ldx + c0 + i4;
       cp_async16(&S.u.pro.Et[sl][j][i4], src, valid);
     }
   };
-  // round 1 over the window's tiles with (dp + g >= 2) == OLD
-  auto round1 = [&](auto old_tag) {
-    constexpr bool OLD = decltype(old_tag)::value;
+  // T1 over g in [g_lo, g_hi] and U over dp in [g_lo, g_hi], one pass over K
+  auto products = [&](int g_lo, int g_hi) {
 #pragma unroll 2
     for (int k = 0; k < TILE; ++k) {
-      float b[P + 1][2];   // L^A[J, J-g][c][k] for this thread's two columns
-      b[0][0] = S.LA0[k][pc];
-      b[0][1] = S.LA0[k][pc + 1];
 #pragma unroll
-      for (int g = 1; g <= P; ++g) {
-        b[g][0] = S.u.pro.LAt[g - 1][k][pc];
-        b[g][1] = S.u.pro.LAt[g - 1][k][pc + 1];
-      }
+      for (int d = 1; d <= P; ++d) {
+        if (d < g_lo || d > g_hi) continue;
+        const float4 ae = *reinterpret_cast<const float4*>(&S.u.pro.Et[d - 1][k][pr]);
+        const float be0 = S.u.pro.LAt[d - 1][k][pc], be1 = S.u.pro.LAt[d - 1][k][pc + 1];
+        const float4 ab = *reinterpret_cast<const float4*>(&S.u.pro.LBt[d - 1][k][pr]);
+        const float bn0 = S.u.pro.Et[LEAF_WINDOW + d - 1][k][pc];
+        const float bn1 = S.u.pro.Et[LEAF_WINDOW + d - 1][k][pc + 1];
+        const float ea[4] = {ae.x, ae.y, ae.z, ae.w}, ba[4] = {ab.x, ab.y, ab.z, ab.w};
 #pragma unroll
-      for (int dp = 0; dp <= P; ++dp) {
-#pragma unroll
-        for (int g = (dp == 0 ? 1 : 0); g + dp <= P; ++g) {
-          if ((dp + g >= 2) != OLD) continue;
-          const float4 av = *reinterpret_cast<const float4*>(&S.u.pro.Et[window_slot(P, dp, g)][k][pr]);
-          acc[dp][0][0] = fmaf(av.x, b[g][0], acc[dp][0][0]);
-          acc[dp][0][1] = fmaf(av.x, b[g][1], acc[dp][0][1]);
-          acc[dp][1][0] = fmaf(av.y, b[g][0], acc[dp][1][0]);
-          acc[dp][1][1] = fmaf(av.y, b[g][1], acc[dp][1][1]);
-          acc[dp][2][0] = fmaf(av.z, b[g][0], acc[dp][2][0]);
-          acc[dp][2][1] = fmaf(av.z, b[g][1], acc[dp][2][1]);
-          acc[dp][3][0] = fmaf(av.w, b[g][0], acc[dp][3][0]);
-          acc[dp][3][1] = fmaf(av.w, b[g][1], acc[dp][3][1]);
+        for (int i = 0; i < 4; ++i) {
+          t1[i][0] = fmaf(ea[i], be0, t1[i][0]);
+          t1[i][1] = fmaf(ea[i], be1, t1[i][1]);
+          u[i][0] = fmaf(ba[i], bn0, u[i][0]);
+          u[i][1] = fmaf(ba[i], bn1, u[i][1]);
         }
       }
     }
   };
-  // round 2 over N_dp, dp in [d_lo, d_hi]
-  auto round2 = [&](int d_lo, int d_hi) {
-#pragma unroll 2
-    for (int k = 0; k < TILE; ++k) {
-#pragma unroll
-      for (int dp = 1; dp <= P; ++dp) {
-        if (dp < d_lo || dp > d_hi) continue;
-        const float4 av = *reinterpret_cast<const float4*>(&S.u.pro.LBt[dp - 1][k][pr]);
-        const float b0 = S.u.pro.Et[dp - 1][k][pc], b1 = S.u.pro.Et[dp - 1][k][pc + 1];
-        u[0][0] = fmaf(av.x, b0, u[0][0]);
-        u[0][1] = fmaf(av.x, b1, u[0][1]);
-        u[1][0] = fmaf(av.y, b0, u[1][0]);
-        u[1][1] = fmaf(av.y, b1, u[1][1]);
-        u[2][0] = fmaf(av.z, b0, u[2][0]);
-        u[2][1] = fmaf(av.z, b1, u[2][1]);
-        u[3][0] = fmaf(av.w, b0, u[3][0]);
-        u[3][1] = fmaf(av.w, b1, u[3][1]);
-      }
-    }
-  };
-  // stores acc[dp] (N_dp) into slot dp - 1
-  auto store_n = [&](int dp) {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      S.u.pro.Et[dp - 1][pr + i][pc] = acc[dp][i][0];
-      S.u.pro.Et[dp - 1][pr + i][pc + 1] = acc[dp][i][1];
-    }
-  };
   if (P >= 2) {
-    // the part of the older tiles: N_2 .. N_P are complete after it
 #pragma unroll
-    for (int sl = 0; sl < (P + 1) * (P + 2) / 2 - 1; ++sl)
-      if (window_dp(P, sl) + window_g(P, sl) >= 2) fetch_e(sl, window_dp(P, sl), window_g(P, sl));
+    for (int d = 2; d <= P; ++d) {
+      fetch(true, d);
+      fetch(false, d);
+    }
     cp_async_wait_all();
     leaf_sync();
-    round1(std::true_type());
-    leaf_sync();   // older tiles read: slots 1 .. P-1 take N_2 .. N_P
-#pragma unroll
-    for (int dp = 2; dp <= P; ++dp) store_n(dp);
-    leaf_sync();
-    round2(2, P);
+    products(2, P);
   }
   if (PDL) {
     pdl_wait();
     pdl_trigger();
   }
-  float xv[LEAF_PER_THREAD];
+  // X at this thread's product positions: rows pr .. pr+3, columns pc, pc+1
+  float xv[4][2];
 #pragma unroll
-  for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-    const int e = t + k * LEAF_THREADS;
-    xv[k] = __ldcg(a.X + (r0 + e / TILE) * a.ldx + c0 + e % TILE);
+  for (int i = 0; i < 4; ++i) {
+    const float2 x2 = __ldcg(reinterpret_cast<const float2*>(a.X + (r0 + pr + i) * a.ldx + c0 + pc));
+    xv[i][0] = x2.x;
+    xv[i][1] = x2.y;
   }
   if (P >= 1) {
-    // the newest tiles, E[I, J-1] (slot 0) and E[I-1, J] (slot P); slots 1 ..
-    // P-1 hold N_2 .. N_P, which round 2 has read
-    fetch_e(window_slot(P, 0, 1), 0, 1);
-    fetch_e(window_slot(P, 1, 0), 1, 0);
+    fetch(true, 1);
+    fetch(false, 1);
   }
   cp_async_wait_all();
   leaf_sync();   // factor blocks and window tiles in shared memory
   if (P >= 1) {
-    static_assert(window_slot(1, 0, 1) == 0 && window_slot(2, 1, 0) == 2 && window_slot(3, 1, 0) == 3,
-                  "newest tiles in slots 0 and P");
-    round1(std::false_type());
-    leaf_sync();   // the newest tiles are read: slot 0 takes N_1, slot P takes U
+    products(1, 1);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      S.T1s[pr + i][pc] = acc[0][i][0];
-      S.T1s[pr + i][pc + 1] = acc[0][i][1];
-    }
-    store_n(1);
-    leaf_sync();
-    round2(1, 1);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      S.u.pro.Et[P][pr + i][pc] = u[i][0];
-      S.u.pro.Et[P][pr + i][pc + 1] = u[i][1];
-    }
-    leaf_sync();
-#pragma unroll
-    for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-      const int e = t + k * LEAF_THREADS;
-      xv[k] += S.u.pro.Et[P][e / TILE][e % TILE];
+      S.T1s[pr + i][pc] = t1[i][0];
+      S.T1s[pr + i][pc + 1] = t1[i][1];
+      xv[i][0] += u[i][0];
+      xv[i][1] += u[i][1];
     }
   }
   leaf_sync();   // the wavefront's arrays overlay the prologue's
 #pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    S.Xs[pr + i][pc] = xv[i][0];
+    S.Xs[pr + i][pc + 1] = xv[i][1];
+  }
+#pragma unroll
   for (int k = 0; k < LEAF_PER_THREAD; ++k) {
     const int e = t + k * LEAF_THREADS;
-    if (e < TILE * TILE) {
-      const int p = e / TILE, c = e % TILE;
-      S.Xs[p][c] = xv[k];
-      S.u.w.Srzl[p][c] = make_float4(scv[k], 1.f / scv[k], -zv[k], 0.f);
-    }
+    const int p = e / TILE, c = e % TILE;
+    S.u.w.Srzl[p][c] = make_float4(scv[k], 1.f / scv[k], -zv[k], 0.f);
   }
   if (t < TILE)
     S.Lsub[t] = make_float4(t >= 1 ? S.LBs[t][t - 1] : 0.f, t >= 2 ? S.LBs[t][t - 2] : 0.f,
@@ -670,6 +608,15 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
       for (int j = 0; j < TILE; ++j) tmp[j] = LAr[(j + 8) & (TILE - 1)];
 #pragma unroll
       for (int j = 0; j < TILE; ++j) LAr[j] = tmp[j];
+    }
+    if (P < LEAF_WINDOW) {
+      // the final G (the last step's errors, published at the last barrier,
+      // folded too; LAr is back at its first rotation) for the tiles below
+      // in this block: G[i][q] = T1[i][q] + sum_{j <= q} E[i][j] L^A[J,J][q][j]
+      fold(2 * TILE - 2, 0);
+#pragma unroll
+      for (int r = 0; r < LEAF_ROWS_PER_HELPER; ++r)
+        if (i0 + r < TILE) a.Gout[(r0 + i0 + r) * a.ldx + c0 + q] = Gg[r];
     }
   }
   leaf_sync();   // the wavefront is done: its arrays are free
@@ -1299,8 +1246,8 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
   a.status = (int*)(ws + sl.off_status);
   a.s = s;
   a.rc = BAKRON_OK;
-  // the leaves' fp32 E^T shares the M hi plane (see SolveLayout)
-  a.la = LeafArgs{a.Mt, a.Nt, m, n, a.X, a.np, a.EtH, a.EtL, a.MH, a.mp,
+  // the leaves' fp32 E^T and final G share the M planes (see SolveLayout)
+  a.la = LeafArgs{a.Mt, a.Nt, m, n, a.X, a.np, a.EtH, a.EtL, a.MH, a.ML, a.mp,
                   (const float*)(f + fl.off_LBblk), (const float*)(f + fl.off_LAblk),
                   scales, zeros, a.G, a.gsz, a.qmax, codes, a.status};
   a.ba = BandArgs{a.LBH, a.LBL, a.mp, a.EtH, a.EtL, a.mp, a.LAH, a.LAL, a.np,
