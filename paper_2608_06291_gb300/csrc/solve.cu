@@ -186,9 +186,8 @@ static_assert(KM == LEAF_BLOCK_LD, "the factor buffer's leaf blocks are copied a
 // its block (Alg. 5 ranges of up to LEAF_WINDOW + 1 anti-diagonals are run
 // as such blocks of leaves), through the E tiles (I, J - g) and the final G
 // of the tiles (I - dp, J), 1 <= g, dp <= LEAF_WINDOW.
-constexpr int LEAF_WINDOW = 3;
+constexpr int LEAF_WINDOW = 7;
 static_assert(LEAF_WINDOW + 1 == LEAF_BLOCKS, "a window needs the blocks L[I, I-1 .. I-LEAF_WINDOW]");
-constexpr int LEAF_WINDOW_TILES = 2 * LEAF_WINDOW;   // E[I, J-g] and G[I-dp, J]
 
 // 32^3 products a window-P leaf forms before its wavefront (T1 and U).
 __host__ __device__ constexpr int window_products(int P) { return 2 * P; }
@@ -202,12 +201,12 @@ struct LeafSmem {
   float Part[4][LEAF_HELPERS][TILE];              // partial pre of a step (ring of 4 steps)
   float4 Lsub[TILE];                              // (L^B[p][p-1], L^B[p][p-2], L^B[p][p-3], 0)
   union {
-    struct {   // prologue of an absorbing leaf: k-major product operands
-      // slots 0 .. LEAF_WINDOW-1: E[I, J-g] k-major, Et[g-1][j][i] = E[..][i][j];
-      // slots LEAF_WINDOW ..: G[I-dp, J] as stored, Et[LEAF_WINDOW+dp-1][i][q]
-      __align__(16) float Et[LEAF_WINDOW_TILES][TILE][KM];
-      __align__(16) float LAt[LEAF_WINDOW][TILE][KM];   // LAt[g-1][j][q] = L^A[J, J-g][q][j]
-      __align__(16) float LBt[LEAF_WINDOW][TILE][KM];   // LBt[dp-1][i][p] = L^B[I, I-dp][p][i]
+    struct {   // prologue of a window-P leaf: its window, staged one d at a time
+      // buffer b holds the operands of one d: [0] E[I, J-d] k-major
+      // (Et[j][i] = E[i][j]), [1] G[I-d, J] (row i, column q), [2] L^A[J, J-d]
+      // k-major ([j][q] = L^A[q][j]), [3] L^B[I, I-d] k-major ([i][p] =
+      // L^B[p][i]).  Buffers 0, 1 alternate before the PDL wait, 2 is d = 1.
+      __align__(16) float B[3][4][TILE][KM];
     } pro;
     struct {   // the wavefront
       union {
@@ -257,8 +256,13 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, bool vali
                "r"(valid ? 16 : 0)
                : "memory");
 }
-__device__ __forceinline__ void cp_async_wait_all() {
-  asm volatile("cp.async.wait_all;" ::: "memory");
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+// waits until at most N of this thread's committed groups are in flight
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
 // Copies one leaf block (TILE rows of KM floats) as it is; thread t of the leaf.
@@ -295,17 +299,65 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
   // waiting for the previous kernel; the factor blocks as asynchronous copies
   // of the factor buffer's leaf blocks, which hold them in the layouts used
   // here (LBs row-major, the others k-major, rows padded to KM).
-  {
-    const float* lb = a.LBblk + (int64_t)I * LEAF_BLOCKS * LEAF_BLOCK_FLOATS;
-    const float* la = a.LAblk + (int64_t)J * LEAF_BLOCKS * LEAF_BLOCK_FLOATS;
-    copy_block(&S.LBs[0][0], lb, t);
-    copy_block(&S.LA0[0][0], la, t);
+  const float* lbk = a.LBblk + (int64_t)I * LEAF_BLOCKS * LEAF_BLOCK_FLOATS;
+  const float* lak = a.LAblk + (int64_t)J * LEAF_BLOCKS * LEAF_BLOCK_FLOATS;
+  copy_block(&S.LBs[0][0], lbk, t);
+  copy_block(&S.LA0[0][0], lak, t);
+  // The window.  N_d of this tile (the errors of row I - d of the window
+  // seen from column block J) equals the final G of tile (I - d, J), which
+  // sits at position P - d of the same block: every leaf leaves its final G
+  // in the Gout plane.  So
+  //     T1 = sum_{d=1..P} E[I, J-d] L^A[J, J-d]^T,
+  //     U  = sum_{d=1..P} L^B[I, I-d] G[I-d, J],
+  // 2P products of 32^3, taken one d at a time.  For d >= 2 the tiles were
+  // written by kernels that had completed when this one was launched: their
+  // part runs before the wait for the previous kernel (overlapping it), its
+  // operands double-buffered; E[I, J-1] and G[I-1, J] come after.  Thread t
+  // forms rows pr .. pr+3, columns pc, pc+1 of T1 and U.
+  const int pr = 4 * (t >> 4), pc = 2 * (t & 15);
+  float t1[4][2], u[4][2];
 #pragma unroll
-    for (int d = 1; d <= P; ++d) {
-      copy_block(&S.u.pro.LBt[d - 1][0][0], lb + d * LEAF_BLOCK_FLOATS, t);
-      copy_block(&S.u.pro.LAt[d - 1][0][0], la + d * LEAF_BLOCK_FLOATS, t);
+  for (int i = 0; i < 4; ++i) t1[i][0] = t1[i][1] = u[i][0] = u[i][1] = 0.f;
+  auto fetch_factors = [&](int d, int b) {
+    copy_block(&S.u.pro.B[b][2][0][0], lak + d * LEAF_BLOCK_FLOATS, t);
+    copy_block(&S.u.pro.B[b][3][0][0], lbk + d * LEAF_BLOCK_FLOATS, t);
+  };
+  // E[I, J-d] (row j of the buffer is the E^T row c0 - 32 d + j, columns
+  // r0 ..) and G[I-d, J] (row i is the Gout row r0 - 32 d + i, columns c0 ..);
+  // zeros outside the matrix
+  auto fetch_tiles = [&](int d, int b) {
+    constexpr int CH = TILE * TILE / 4;   // 16-byte chunks of a tile
+    static_assert(CH == 2 * LEAF_THREADS, "two chunks of every tile per thread");
+    const bool ve = J - d >= 0, vg = I - d >= 0;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int c = t + LEAF_THREADS * h, j = c / (TILE / 4), i4 = 4 * (c % (TILE / 4));
+      cp_async16(&S.u.pro.B[b][0][j][i4],
+                 ve ? a.EtF + (c0 - (int64_t)TILE * d + j) * a.ldt + r0 + i4 : a.EtF, ve);
+      cp_async16(&S.u.pro.B[b][1][j][i4],
+                 vg ? a.Gout + (r0 - (int64_t)TILE * d + j) * a.ldx + c0 + i4 : a.Gout, vg);
     }
-  }
+  };
+  // T1 += E[I, J-d] L^A[J, J-d]^T and U += L^B[I, I-d] G[I-d, J] from buffer b
+  auto products = [&](int b) {
+#pragma unroll 2
+    for (int k = 0; k < TILE; ++k) {
+      const float4 ae = *reinterpret_cast<const float4*>(&S.u.pro.B[b][0][k][pr]);
+      const float be0 = S.u.pro.B[b][2][k][pc], be1 = S.u.pro.B[b][2][k][pc + 1];
+      const float4 ab = *reinterpret_cast<const float4*>(&S.u.pro.B[b][3][k][pr]);
+      const float bn0 = S.u.pro.B[b][1][k][pc], bn1 = S.u.pro.B[b][1][k][pc + 1];
+      const float ea[4] = {ae.x, ae.y, ae.z, ae.w}, ba[4] = {ab.x, ab.y, ab.z, ab.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        t1[i][0] = fmaf(ea[i], be0, t1[i][0]);
+        t1[i][1] = fmaf(ea[i], be1, t1[i][1]);
+        u[i][0] = fmaf(ba[i], bn0, u[i][0]);
+        u[i][1] = fmaf(ba[i], bn1, u[i][1]);
+      }
+    }
+  };
+  if (P >= 1) fetch_factors(1, 2);
+  cp_async_commit();
   float scv[LEAF_PER_THREAD], zv[LEAF_PER_THREAD];
 #pragma unroll
   for (int k = 0; k < LEAF_PER_THREAD; ++k) {
@@ -316,72 +368,26 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     scv[k] = real ? a.scales[og] : 1.f;
     zv[k] = real ? a.zeros[og] : 0.f;
   }
-  // The window.  N_dp of this tile (the errors of row I - dp of the window
-  // seen from column block J) equals the final G of tile (I - dp, J), which
-  // sits at position P - dp of the same block: every leaf leaves its final G
-  // in the Gout plane.  So
-  //     T1 = sum_{g=1..P} E[I, J-g] L^A[J, J-g]^T,
-  //     U  = sum_{dp=1..P} L^B[I, I-dp] G[I-dp, J],
-  // 2P products of 32^3.  Terms of tiles two or more anti-diagonals back
-  // (g >= 2, dp >= 2) were written by kernels that had completed when this
-  // one was launched: they run before the wait for the previous kernel
-  // (overlapping it); E[I, J-1] and G[I-1, J] come after.  Thread t forms
-  // rows pr .. pr+3, columns pc, pc+1 of T1 and U.
-  const int pr = 4 * (t >> 4), pc = 2 * (t & 15);
-  float t1[4][2], u[4][2];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) t1[i][0] = t1[i][1] = u[i][0] = u[i][1] = 0.f;
-  // E[I, J-g] into slot g - 1, k-major as E^T stores it (row j of the slot is
-  // the E^T row c0 - 32 g + j, columns r0 ..); G[I-dp, J] into slot
-  // LEAF_WINDOW + dp - 1 as stored (row i, columns c0 ..); zeros outside the
-  // matrix
-  auto fetch = [&](bool is_e, int d) {
-    constexpr int CH = TILE * TILE / 4;   // 16-byte chunks of a tile
-    static_assert(CH == 2 * LEAF_THREADS, "two chunks of every tile per thread");
-    const bool valid = is_e ? J - d >= 0 : I - d >= 0;
-    const int sl = is_e ? d - 1 : LEAF_WINDOW + d - 1;
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int c = t + LEAF_THREADS * h, j = c / (TILE / 4), i4 = 4 * (c % (TILE / 4));
-      const float* src =
-          !valid ? a.EtF
-          : is_e ? a.EtF + (c0 - (int64_t)TILE * d + j) * a.ldt + r0 + i4
-                 : a.Gout + (r0 - (int64_t)TILE * d + j) * a.ldx + c0 + i4;
-      cp_async16(&S.u.pro.Et[sl][j][i4], src, valid);
-    }
-  };
-  // T1 over g in [g_lo, g_hi] and U over dp in [g_lo, g_hi], one pass over K
-  auto products = [&](int g_lo, int g_hi) {
-#pragma unroll 2
-    for (int k = 0; k < TILE; ++k) {
-#pragma unroll
-      for (int d = 1; d <= P; ++d) {
-        if (d < g_lo || d > g_hi) continue;
-        const float4 ae = *reinterpret_cast<const float4*>(&S.u.pro.Et[d - 1][k][pr]);
-        const float be0 = S.u.pro.LAt[d - 1][k][pc], be1 = S.u.pro.LAt[d - 1][k][pc + 1];
-        const float4 ab = *reinterpret_cast<const float4*>(&S.u.pro.LBt[d - 1][k][pr]);
-        const float bn0 = S.u.pro.Et[LEAF_WINDOW + d - 1][k][pc];
-        const float bn1 = S.u.pro.Et[LEAF_WINDOW + d - 1][k][pc + 1];
-        const float ea[4] = {ae.x, ae.y, ae.z, ae.w}, ba[4] = {ab.x, ab.y, ab.z, ab.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          t1[i][0] = fmaf(ea[i], be0, t1[i][0]);
-          t1[i][1] = fmaf(ea[i], be1, t1[i][1]);
-          u[i][0] = fmaf(ba[i], bn0, u[i][0]);
-          u[i][1] = fmaf(ba[i], bn1, u[i][1]);
-        }
-      }
-    }
-  };
   if (P >= 2) {
 #pragma unroll
-    for (int d = 2; d <= P; ++d) {
-      fetch(true, d);
-      fetch(false, d);
+    for (int d = 2; d <= P && d <= 3; ++d) {
+      fetch_factors(d, d & 1);
+      fetch_tiles(d, d & 1);
+      cp_async_commit();
     }
-    cp_async_wait_all();
-    leaf_sync();
-    products(2, P);
+#pragma unroll
+    for (int d = 2; d <= P; ++d) {
+      if (d < P) cp_async_wait_group<1>();   // the copies of d + 1 may still fly
+      else cp_async_wait_group<0>();
+      leaf_sync();
+      products(d & 1);
+      if (d + 2 <= P) {
+        leaf_sync();   // buffer d & 1 is read: it takes d + 2
+        fetch_factors(d + 2, d & 1);
+        fetch_tiles(d + 2, d & 1);
+        cp_async_commit();
+      }
+    }
   }
   if (PDL) {
     pdl_wait();
@@ -395,14 +401,12 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     xv[i][0] = x2.x;
     xv[i][1] = x2.y;
   }
+  if (P >= 1) fetch_tiles(1, 2);
+  cp_async_commit();
+  cp_async_wait_group<0>();
+  leaf_sync();   // factor blocks and the last window tiles in shared memory
   if (P >= 1) {
-    fetch(true, 1);
-    fetch(false, 1);
-  }
-  cp_async_wait_all();
-  leaf_sync();   // factor blocks and window tiles in shared memory
-  if (P >= 1) {
-    products(1, 1);
+    products(2);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       S.T1s[pr + i][pc] = t1[i][0];
@@ -642,6 +646,16 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
   }
   if (bad) raise_status(a.status, BAKRON_ERR_NONFINITE);
   leaf_sync();   // shared memory free for the next tile of this CTA
+}
+
+// leaf_tile<false, P> for a window known at run time (0 <= h <= LEAF_WINDOW)
+template <int P>
+__device__ __forceinline__ void leaf_tile_window(int h, const LeafArgs& a, int I, int J, LeafSmem& S) {
+  if (h == P || P == LEAF_WINDOW) {
+    leaf_tile<false, P>(a, I, J, S);
+    return;
+  }
+  if constexpr (P < LEAF_WINDOW) leaf_tile_window<P + 1>(h, a, I, J, S);
 }
 
 // One CTA per tile of tile anti-diagonal K; P: the leaf's window.
@@ -973,10 +987,7 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_subtree(const __grid_constant_
       const int ilo = max(0, P.k - (Nt - 1)), ihi = min(P.k, Mt - 1);
       if (threadIdx.x < LEAF_THREADS)
         for (int I = ilo + (int)blockIdx.x; I <= ihi; I += gridDim.x) {
-          if (P.h == 0) leaf_tile<false, 0>(A.leaf, I, P.k - I, S.leaf);
-          else if (P.h == 1) leaf_tile<false, 1>(A.leaf, I, P.k - I, S.leaf);
-          else if (P.h == 2) leaf_tile<false, 2>(A.leaf, I, P.k - I, S.leaf);
-          else leaf_tile<false, 3>(A.leaf, I, P.k - I, S.leaf);
+          leaf_tile_window<0>(P.h, A.leaf, I, P.k - I, S.leaf);
         }
     } else {
       const int row_lo = max(0, P.h - (Nt - 1)), row_hi = min(Mt - 1, P.l - 1);
@@ -1067,18 +1078,35 @@ static void note(SolveArgs& a, cudaError_t e) {
 // Leaf of anti-diagonal K; `window`: how many anti-diagonals before it (in
 // its block) it absorbs.  Flops: the in-tile feedback and the window's
 // products, 2 * 32^3 each, per tile.
+// k_leaf<P> for a window known at run time (0 <= window <= LEAF_WINDOW)
+template <int P>
+static cudaError_t launch_leaf_window(int window, dim3 grid, dim3 block, size_t sm, cudaStream_t s,
+                                     int K, const LeafArgs& la) {
+  if (window == P || P == LEAF_WINDOW) return launch_pdl(k_leaf<P>, grid, block, sm, s, K, la);
+  if constexpr (P < LEAF_WINDOW) return launch_leaf_window<P + 1>(window, grid, block, sm, s, K, la);
+  return cudaErrorInvalidValue;
+}
+static cudaError_t launch_leaf_window(int window, dim3 grid, dim3 block, size_t sm, cudaStream_t s,
+                                      int K, const LeafArgs& la) {
+  return launch_leaf_window<0>(window, grid, block, sm, s, K, la);
+}
+
+// dynamic shared memory of k_leaf<P> .. k_leaf<LEAF_WINDOW>
+template <int P>
+static cudaError_t set_leaf_smem(int bytes) {
+  cudaError_t e = cudaFuncSetAttribute(k_leaf<P>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if constexpr (P < LEAF_WINDOW)
+    if (e == cudaSuccess) e = set_leaf_smem<P + 1>(bytes);
+  return e;
+}
+
 static void leaf(SolveArgs& a, int K, int window) {
   const int ilo = max(0, K - (a.Nt - 1)), ihi = min(K, a.Mt - 1);
   LaunchScope ls(kFamLeaf, a.s,
                  2.0 * TILE * TILE * TILE * (1 + window_products(window)) * (ihi - ilo + 1));
   const dim3 grid(ihi - ilo + 1), block(LEAF_THREADS);
   const size_t sm = sizeof(LeafSmem);
-  switch (window) {
-    case 0: note(a, launch_pdl(k_leaf<0>, grid, block, sm, a.s, K, a.la)); break;
-    case 1: note(a, launch_pdl(k_leaf<1>, grid, block, sm, a.s, K, a.la)); break;
-    case 2: note(a, launch_pdl(k_leaf<2>, grid, block, sm, a.s, K, a.la)); break;
-    default: note(a, launch_pdl(k_leaf<3>, grid, block, sm, a.s, K, a.la)); break;
-  }
+  note(a, launch_leaf_window(window, grid, block, sm, a.s, K, a.la));
 }
 
 // Dynamic shared memory of the leaf and subtree kernels above the 48 KB
@@ -1089,13 +1117,7 @@ static cudaError_t ensure_leaf_attrs() {
   std::lock_guard<std::mutex> lk(mu);
   if (done) return cudaSuccess;
   const int sm = (int)sizeof(LeafSmem), ss = (int)sizeof(SubtreeSmem);
-  cudaError_t e = cudaFuncSetAttribute(k_leaf<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(k_leaf<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(k_leaf<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(k_leaf<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+  cudaError_t e = set_leaf_smem<0>(sm);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(k_subtree, cudaFuncAttributeMaxDynamicSharedMemorySize, ss);
   if (e == cudaSuccess) done = true;
