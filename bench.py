@@ -236,7 +236,7 @@ def run_gpu(args):
     if not args.no_autotune:
         best = P.bakron_autotune(W, fac, cfg.bits, cfg.group, workspace=work)
         sched = {"tc_min_band": best["tc_min_band"], "fused_max_band": best["fused_max_band"],
-                 "autotuned": True}
+                 "leaf_block": best["leaf_block"], "autotuned": True}
     for _ in range(max(3, args.warmup)):
         flush.fill_(1)
         eager_step()

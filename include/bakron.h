@@ -133,34 +133,40 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw,
  * No counterpart in the paper: Alg. 5 fixes the recursion (halving of the
  * anti-diagonal range, Sec. 3.5) and its result, not how a node's band
  * product is evaluated; only that is tuned, so every choice rounds W the same
- * way up to fp32 summation order.  Two thresholds, in tile anti-diagonals
- * (32 x 32 tiles) spanned by a node:
- *   tc_min_band     nodes spanning at least this many run their two band
- *                   products on the tensor cores (3xTF32); 0: never
+ * way up to fp32 summation order.  Three settings, in tile anti-diagonals
+ * (32 x 32 tiles) spanned by a range of the recursion:
+ *   leaf_block      ranges spanning at most this many (1 .. 16) run as a
+ *                   block of leaves, each leaf applying what the earlier
+ *                   anti-diagonals of its block send it (the nodes inside)
+ *   tc_min_band     wider nodes spanning at least this many run their two
+ *                   band products on the tensor cores (3xTF32); 0: never
  *   fused_max_band  narrower nodes spanning at most this many run both
  *                   products in one CUDA-core launch, wider ones in two
  * Candidates: tc_min_band in {0, 4, 6, 8, 12, 16, 24} x fused_max_band in
- * {2, 4}; each is solved three times (one warm-up) and timed with CUDA events
- * on `stream`.  The fastest is stored in a process-wide table keyed by the
- * current device and (m, n), which later bakron_solve calls of that shape
- * use; the environment variables BAKRON_TC_MIN_BAND and BAKRON_FUSED_MAX_BAND
- * override the table.  Untuned shapes use tc_min_band = 6, fused_max_band = 2.
- * Arguments as bakron_solve (codes, scales and zeros are overwritten; no
- * pre-rounding output); tc_min_band, fused_max_band (host, may be NULL)
- * receive the choice and best_ms (host, may be NULL) its time.  Synchronous:
- * it synchronises `stream` after every candidate, so it cannot be captured in
- * a CUDA graph.  Returns the first nonzero status of a candidate solve.
+ * {2, 4} x leaf_block in {4, 8, 16}; each is solved three times (one warm-up)
+ * and timed with CUDA events on `stream`.  The fastest is stored in a
+ * process-wide table keyed by the current device and (m, n), which later
+ * bakron_solve calls of that shape use; the environment variables
+ * BAKRON_TC_MIN_BAND, BAKRON_FUSED_MAX_BAND and BAKRON_LEAF_BLOCK override
+ * the table.  Untuned shapes use tc_min_band = 6, fused_max_band = 2,
+ * leaf_block = 8.  Arguments as bakron_solve (codes, scales and zeros are
+ * overwritten; no pre-rounding output); tc_min_band, fused_max_band,
+ * leaf_block (host, may be NULL) receive the choice and best_ms (host, may
+ * be NULL) its time.  Synchronous: it synchronises `stream` after every
+ * candidate, so it cannot be captured in a CUDA graph.  Returns the first
+ * nonzero status of a candidate solve.
  */
 int bakron_autotune(const void* W, int wdtype, int m, int n, int64_t ldw,
                     const void* factors, int bits, int group_size,
                     uint8_t* codes, float* scales, float* zeros,
                     void* workspace, size_t workspace_bytes,
-                    int* tc_min_band, int* fused_max_band, float* best_ms,
-                    void* stream);
+                    int* tc_min_band, int* fused_max_band, int* leaf_block,
+                    float* best_ms, void* stream);
 
-/* bakron_get_tuning -- the thresholds a bakron_solve of shape m x n would use
+/* bakron_get_tuning -- the settings a bakron_solve of shape m x n would use
  * now (table entry or default, environment applied).  Host only. */
-int bakron_get_tuning(int m, int n, int* tc_min_band, int* fused_max_band);
+int bakron_get_tuning(int m, int n, int* tc_min_band, int* fused_max_band,
+                      int* leaf_block);
 
 /* bakron_autotune_clear -- forget every tuned shape. */
 void bakron_autotune_clear(void);

@@ -66,10 +66,11 @@ def lib() -> ctypes.CDLL:
     L.bakron_diag_gemm_tf32x3.argtypes = [vp, vp, vp, i32, i32, i32, vp, sz, vp]
     L.bakron_diag_gemm_tf32x3.restype = i32
     L.bakron_autotune.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, sz,
-                                  ctypes.POINTER(i32), ctypes.POINTER(i32),
+                                  ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32),
                                   ctypes.POINTER(ctypes.c_float), vp]
     L.bakron_autotune.restype = i32
-    L.bakron_get_tuning.argtypes = [i32, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)]
+    L.bakron_get_tuning.argtypes = [i32, i32, ctypes.POINTER(i32), ctypes.POINTER(i32),
+                                    ctypes.POINTER(i32)]
     L.bakron_get_tuning.restype = i32
     L.bakron_autotune_clear.argtypes = []
     L.bakron_autotune_clear.restype = None
@@ -199,7 +200,8 @@ def bakron_autotune(W, f: Factors, bits: int, group_size: int = 0, workspace=Non
                     stream=None) -> dict:
     """Time the candidate schedules of an m x n solve on W and remember the
     fastest for later solves of that shape.  Returns {"tc_min_band",
-    "fused_max_band", "ms"}.  Synchronous; overwrites scratch outputs only."""
+    "fused_max_band", "leaf_block", "ms"}.  Synchronous; overwrites scratch
+    outputs only."""
     if not W.is_cuda or W.dim() != 2 or W.stride(1) != 1:
         raise ValueError("W must be a 2-D CUDA tensor with unit column stride")
     dt = {torch.float32: F32, torch.bfloat16: BF16}.get(W.dtype)
@@ -214,21 +216,22 @@ def bakron_autotune(W, f: Factors, bits: int, group_size: int = 0, workspace=Non
     scales = torch.empty(m, G, dtype=torch.float32, device=dev)
     zeros = torch.empty(m, G, dtype=torch.float32, device=dev)
     ws = workspace if workspace is not None else alloc_workspace(m, n, dev)
-    tc, fu, ms = ctypes.c_int(0), ctypes.c_int(0), ctypes.c_float(0.0)
+    tc, fu, lb, ms = ctypes.c_int(0), ctypes.c_int(0), ctypes.c_int(0), ctypes.c_float(0.0)
     rc = lib().bakron_autotune(_ptr(W), dt, m, n, W.stride(0), _ptr(f.buf), int(bits),
                                int(group_size), _ptr(codes), _ptr(scales), _ptr(zeros), _ptr(ws),
-                               ws.numel(), ctypes.byref(tc), ctypes.byref(fu), ctypes.byref(ms),
-                               _stream(stream))
+                               ws.numel(), ctypes.byref(tc), ctypes.byref(fu), ctypes.byref(lb),
+                               ctypes.byref(ms), _stream(stream))
     _check(rc, "bakron_autotune")
-    return {"tc_min_band": tc.value, "fused_max_band": fu.value, "ms": ms.value}
+    return {"tc_min_band": tc.value, "fused_max_band": fu.value, "leaf_block": lb.value,
+            "ms": ms.value}
 
 
 def bakron_get_tuning(m: int, n: int) -> dict:
-    """The schedule thresholds an m x n solve would use now."""
-    tc, fu = ctypes.c_int(0), ctypes.c_int(0)
-    _check(lib().bakron_get_tuning(int(m), int(n), ctypes.byref(tc), ctypes.byref(fu)),
-           "bakron_get_tuning")
-    return {"tc_min_band": tc.value, "fused_max_band": fu.value}
+    """The schedule settings an m x n solve would use now."""
+    tc, fu, lb = ctypes.c_int(0), ctypes.c_int(0), ctypes.c_int(0)
+    _check(lib().bakron_get_tuning(int(m), int(n), ctypes.byref(tc), ctypes.byref(fu),
+                                   ctypes.byref(lb)), "bakron_get_tuning")
+    return {"tc_min_band": tc.value, "fused_max_band": fu.value, "leaf_block": lb.value}
 
 
 def bakron_autotune_clear() -> None:

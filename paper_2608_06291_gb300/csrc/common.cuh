@@ -51,7 +51,7 @@ __host__ __device__ inline float tf32_hi(float x) {
 // L^A[J, J - g]; fp32 (hi + lo), TILE rows of LEAF_BLOCK_LD floats each (the
 // columns past TILE zero), laid out as the leaf kernel keeps them in shared
 // memory (see build_leaf_blocks), so that it copies them as they are.
-constexpr int LEAF_BLOCKS = 8;
+constexpr int LEAF_BLOCKS = 16;
 constexpr int LEAF_BLOCK_LD = 36;
 constexpr int LEAF_BLOCK_FLOATS = TILE * LEAF_BLOCK_LD;
 

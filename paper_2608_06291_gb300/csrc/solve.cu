@@ -25,6 +25,7 @@
 
 #include <type_traits>
 
+#include <algorithm>
 #include <mutex>
 
 namespace bakron {
@@ -186,7 +187,7 @@ static_assert(KM == LEAF_BLOCK_LD, "the factor buffer's leaf blocks are copied a
 // its block (Alg. 5 ranges of up to LEAF_WINDOW + 1 anti-diagonals are run
 // as such blocks of leaves), through the E tiles (I, J - g) and the final G
 // of the tiles (I - dp, J), 1 <= g, dp <= LEAF_WINDOW.
-constexpr int LEAF_WINDOW = 7;
+constexpr int LEAF_WINDOW = 15;
 static_assert(LEAF_WINDOW + 1 == LEAF_BLOCKS, "a window needs the blocks L[I, I-1 .. I-LEAF_WINDOW]");
 
 // 32^3 products a window-P leaf forms before its wavefront (T1 and U).
@@ -375,7 +376,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
       fetch_tiles(d, d & 1);
       cp_async_commit();
     }
-#pragma unroll
+#pragma unroll 1
     for (int d = 2; d <= P; ++d) {
       if (d < P) cp_async_wait_group<1>();   // the copies of d + 1 may still fly
       else cp_async_wait_group<0>();
@@ -1047,6 +1048,7 @@ struct SolveArgs {
   int tc_min_band;
   int fused_max_band;   // nodes spanning <= this many tile anti-diagonals: one fused launch
   int subtree_max;      // ranges spanning <= this many: one persistent cooperative launch
+  int leaf_block;       // ranges spanning <= this many: a block of leaves (1 .. LEAF_WINDOW + 1)
   int subtree_grid;     // CTAs a cooperative launch may hold (resident at once)
   long long spin_cycles;
   bool tc_ready;
@@ -1164,7 +1166,7 @@ static void band(SolveArgs& a, int k, int h, int l) {
 
 // Phases of rec(k, l) in the order rec enqueues them.
 static void subtree_phases(const SolveArgs& a, int k, int l, SubtreeArgs& A) {
-  if (l - k <= LEAF_WINDOW + 1) {   // a block of leaves, each absorbing the ones before it
+  if (l - k <= a.leaf_block) {   // a block of leaves, each absorbing the ones before it
     for (int K = k; K < l; ++K) A.ph[A.nph++] = Phase{PH_LEAF, K, K - k, K + 1};
     return;
   }
@@ -1224,7 +1226,7 @@ static void subtree(SolveArgs& a, int k, int l) {
 }
 
 static void rec(SolveArgs& a, int k, int l) {
-  if (l - k <= LEAF_WINDOW + 1) {
+  if (l - k <= a.leaf_block) {
     // a block of leaves: leaf K applies what anti-diagonals k .. K-1 send it
     // (the Alg. 5 nodes inside [k, l)), so no band launch is needed here
     for (int K = k; K < l; ++K) leaf(a, K, K - k);
@@ -1281,6 +1283,7 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
     a.tc_min_band = tu.tc_min_band;         // 0 or less: tensor cores off
     a.fused_max_band = tu.fused_max_band;
     a.subtree_max = tu.subtree_max;         // 0 or 1: no persistent subtrees
+    a.leaf_block = std::min(std::max(tu.leaf_block, 1), LEAF_WINDOW + 1);
     if (a.subtree_max > MAX_SUBTREE) a.subtree_max = MAX_SUBTREE;
     a.subtree_grid = 0;
     if (a.subtree_max >= 2) {

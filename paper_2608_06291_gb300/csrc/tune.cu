@@ -44,6 +44,7 @@ Tuning tuning_for(int m, int n) {
   env_override("BAKRON_TC_MIN_BAND", t.tc_min_band);
   env_override("BAKRON_FUSED_MAX_BAND", t.fused_max_band);
   env_override("BAKRON_SUBTREE_MAX", t.subtree_max);
+  env_override("BAKRON_LEAF_BLOCK", t.leaf_block);
   return t;
 }
 
@@ -56,7 +57,7 @@ extern "C" {
 int bakron_autotune(const void* W, int wdtype, int m, int n, int64_t ldw, const void* factors,
                     int bits, int group_size, uint8_t* codes, float* scales, float* zeros,
                     void* workspace, size_t workspace_bytes, int* tc_min_band,
-                    int* fused_max_band, float* best_ms, void* stream) {
+                    int* fused_max_band, int* leaf_block, float* best_ms, void* stream) {
   if (!W || !factors || !codes || !scales || !zeros || !workspace || m < 1 || n < 1)
     return BAKRON_ERR_INVALID_ARG;
   if (wdtype != BAKRON_F32 && wdtype != BAKRON_BF16) return BAKRON_ERR_INVALID_ARG;
@@ -66,6 +67,7 @@ int bakron_autotune(const void* W, int wdtype, int m, int n, int64_t ldw, const 
   cudaStream_t s = (cudaStream_t)stream;
   static const int kTc[] = {0, 4, 6, 8, 12, 16, 24};
   static const int kFused[] = {2, 4};
+  static const int kBlock[] = {4, 8, 16};
   cudaEvent_t e0, e1;
   BK_CUDA_OK(cudaEventCreate(&e0));
   if (cudaEventCreate(&e1) != cudaSuccess) {
@@ -77,7 +79,8 @@ int bakron_autotune(const void* W, int wdtype, int m, int n, int64_t ldw, const 
   int rc = BAKRON_OK;
   for (int tc : kTc) {
     for (int fu : kFused) {
-      const Tuning cand{tc, fu, 0};
+     for (int lb : kBlock) {
+      const Tuning cand{tc, fu, 0, lb};
       float t_min = -1.f;
       for (int rep = 0; rep < 3 && rc == BAKRON_OK; ++rep) {   // rep 0 warms up
         if (cudaEventRecord(e0, s) != cudaSuccess) { rc = BAKRON_ERR_CUDA; break; }
@@ -96,6 +99,8 @@ int bakron_autotune(const void* W, int wdtype, int m, int n, int64_t ldw, const 
         best_t = t_min;
         best = cand;
       }
+     }
+     if (rc != BAKRON_OK) break;
     }
     if (rc != BAKRON_OK) break;
   }
@@ -108,15 +113,17 @@ int bakron_autotune(const void* W, int wdtype, int m, int n, int64_t ldw, const 
   }
   if (tc_min_band) *tc_min_band = best.tc_min_band;
   if (fused_max_band) *fused_max_band = best.fused_max_band;
+  if (leaf_block) *leaf_block = best.leaf_block;
   if (best_ms) *best_ms = best_t;
   return BAKRON_OK;
 }
 
-int bakron_get_tuning(int m, int n, int* tc_min_band, int* fused_max_band) {
+int bakron_get_tuning(int m, int n, int* tc_min_band, int* fused_max_band, int* leaf_block) {
   if (m < 1 || n < 1) return BAKRON_ERR_INVALID_ARG;
   const Tuning t = tuning_for(m, n);
   if (tc_min_band) *tc_min_band = t.tc_min_band;
   if (fused_max_band) *fused_max_band = t.fused_max_band;
+  if (leaf_block) *leaf_block = t.leaf_block;
   return BAKRON_OK;
 }
 

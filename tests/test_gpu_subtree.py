@@ -22,6 +22,13 @@ def _lib():
     P.lib()
 
 
+@pytest.fixture(autouse=True)
+def _small_leaf_blocks(monkeypatch):
+    """Blocks of at most 4 leaves, so that these small problems still have
+    band nodes of every width (the default blocks of 8 leave none below 9)."""
+    monkeypatch.setenv("BAKRON_LEAF_BLOCK", "4")
+
+
 @pytest.mark.parametrize("width", ["2", "3", "8", "16", "32"])
 @pytest.mark.parametrize("m,n", [(97, 131), (300, 417), (640, 96)])
 def test_subtree_widths(width, m, n, monkeypatch):
@@ -66,8 +73,10 @@ def test_subtree_barrier_timeout_and_recover(monkeypatch):
     monkeypatch.setenv("BAKRON_TC_MIN_BAND", "0")
     monkeypatch.setenv("BAKRON_SUBTREE_MAX", "32")
     monkeypatch.setenv("BAKRON_SPIN_CYCLES", "0")
+    # 19 x 14 tiles, 32 tile anti-diagonals: one subtree of two leaf blocks
+    # and the band between them, up to 14 CTAs per phase
     with pytest.raises(P.BakronError) as e:
-        _solve_small(256, 256, 5, bits=4)
+        _solve_small(600, 420, 5, bits=4)
     assert e.value.status == 4
     monkeypatch.delenv("BAKRON_SPIN_CYCLES")
-    _assert_parity(_solve_small(256, 256, 5, bits=4))
+    _assert_parity(_solve_small(600, 420, 5, bits=4))

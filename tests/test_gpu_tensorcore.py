@@ -25,6 +25,13 @@ def _lib():
     P.lib()
 
 
+@pytest.fixture(autouse=True)
+def _small_leaf_blocks(monkeypatch):
+    """Blocks of at most 4 leaves, so that these small problems still have
+    band nodes of every width (the default blocks of 8 leave none below 9)."""
+    monkeypatch.setenv("BAKRON_LEAF_BLOCK", "4")
+
+
 @pytest.mark.parametrize("M,N,K", [(128, 128, 32), (256, 384, 512), (384, 128, 1024)])
 def test_gemm_3xtf32_matches_fp64(M, N, K):
     g = torch.Generator(device="cuda").manual_seed(M + N + K)

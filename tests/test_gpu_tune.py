@@ -36,23 +36,26 @@ def _problem(m, n, seed):
 
 
 def test_autotune_choice_is_used_and_cleared(monkeypatch):
-    for v in ("BAKRON_TC_MIN_BAND", "BAKRON_FUSED_MAX_BAND"):
+    for v in ("BAKRON_TC_MIN_BAND", "BAKRON_FUSED_MAX_BAND", "BAKRON_LEAF_BLOCK"):
         monkeypatch.delenv(v, raising=False)
     P.bakron_autotune_clear()
     m, n = 520, 610
-    assert P.bakron_get_tuning(m, n) == {"tc_min_band": 6, "fused_max_band": 2}
+    default = {"tc_min_band": 6, "fused_max_band": 2, "leaf_block": 8}
+    assert P.bakron_get_tuning(m, n) == default
     W, fac = _problem(m, n, 3)
     best = P.bakron_autotune(W, fac, 4, 0)
     assert best["tc_min_band"] in (0, 4, 6, 8, 12, 16, 24)
     assert best["fused_max_band"] in (2, 4)
+    assert best["leaf_block"] in (4, 8, 16)
     assert best["ms"] > 0
     got = P.bakron_get_tuning(m, n)
-    assert got == {"tc_min_band": best["tc_min_band"], "fused_max_band": best["fused_max_band"]}
+    assert got == {k: best[k] for k in ("tc_min_band", "fused_max_band", "leaf_block")}
     # a solve of the tuned shape launches what the same thresholds set by hand launch
     P.bakron_solve(W, fac, 4, 0)
     tuned_launches = P.bakron_last_launches()
     monkeypatch.setenv("BAKRON_TC_MIN_BAND", str(best["tc_min_band"]))
     monkeypatch.setenv("BAKRON_FUSED_MAX_BAND", str(best["fused_max_band"]))
+    monkeypatch.setenv("BAKRON_LEAF_BLOCK", str(best["leaf_block"]))
     P.bakron_solve(W, fac, 4, 0)
     assert P.bakron_last_launches() == tuned_launches
     # the environment wins over the table
@@ -60,12 +63,13 @@ def test_autotune_choice_is_used_and_cleared(monkeypatch):
     assert P.bakron_get_tuning(m, n)["tc_min_band"] == 0
     monkeypatch.delenv("BAKRON_TC_MIN_BAND")
     monkeypatch.delenv("BAKRON_FUSED_MAX_BAND")
+    monkeypatch.delenv("BAKRON_LEAF_BLOCK")
     P.bakron_autotune_clear()
-    assert P.bakron_get_tuning(m, n) == {"tc_min_band": 6, "fused_max_band": 2}
+    assert P.bakron_get_tuning(m, n) == default
 
 
 def test_tuned_solve_keeps_parity(monkeypatch):
-    for v in ("BAKRON_TC_MIN_BAND", "BAKRON_FUSED_MAX_BAND"):
+    for v in ("BAKRON_TC_MIN_BAND", "BAKRON_FUSED_MAX_BAND", "BAKRON_LEAF_BLOCK"):
         monkeypatch.delenv(v, raising=False)
     m, n = 300, 417
     W, fac = _problem(m, n, 2000 + m + n)
