@@ -63,18 +63,29 @@ __global__ void k_grid(const void* W, int wdt, int m, int n, int64_t ldw, int gs
 }
 
 // X <- W widened to fp32 over the padded mp x np workspace (zeros outside).
+// Grid-stride over chunks of 8 entries of a row (np is a multiple of 128, so
+// a chunk never straddles a row), stored as two 16-byte vectors.
 __global__ void k_init(const void* W, int wdt, int m, int n, int64_t ldw, float* X,
                        int64_t mp, int64_t np) {
   pdl_wait();
   pdl_trigger();
-  const int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (idx >= mp * np) return;
-  const int64_t r = idx / np, c = idx % np;
-  float v = 0.f;
-  if (r < m && c < n)
-    v = (wdt == BAKRON_BF16) ? __bfloat162float(((const __nv_bfloat16*)W)[r * ldw + c])
-                             : ((const float*)W)[r * ldw + c];
-  X[idx] = v;
+  const int64_t chunks = mp * np / 8;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < chunks;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t idx = 8 * i, r = idx / np, c = idx - r * np;
+    float v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      v[j] = 0.f;
+      if (r < m && c + j < n)
+        v[j] = (wdt == BAKRON_BF16)
+                   ? __bfloat162float(((const __nv_bfloat16*)W)[r * ldw + c + j])
+                   : ((const float*)W)[r * ldw + c + j];
+    }
+    float4* o = reinterpret_cast<float4*>(X + idx);
+    o[0] = make_float4(v[0], v[1], v[2], v[3]);
+    o[1] = make_float4(v[4], v[5], v[6], v[7]);
+  }
 }
 
 __global__ void k_copy_out(const float* X, int64_t np, int m, int n, float* out) {
@@ -1309,10 +1320,11 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
                                                                  a.qmax, scales, zeros);
   }
   {
-    const int64_t tot = a.mp * a.np;
+    const int64_t chunks = a.mp * a.np / 8;
     LaunchScope ls(kFamInit, s);
-    note(a, launch_pdl(k_init, dim3((unsigned)((tot + 255) / 256)), dim3(256), 0, s, W, wdt, m, n,
-                       ldw, a.X, a.mp, a.np));
+    const unsigned blocks = (unsigned)std::min<int64_t>((chunks + 255) / 256, 152 * 8);
+    note(a, launch_pdl(k_init, dim3(blocks), dim3(256), 0, s, W, wdt, m, n, ldw, a.X, a.mp,
+                       a.np));
   }
   rec(a, 0, a.Mt + a.Nt - 1);
   if (prerounding) {
