@@ -127,6 +127,20 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, long l
   }
 }
 
+// A hi/lo plane pair in one copy: a rank-3 box (32 columns, rows, 2 planes)
+// lands as the two planes one after the other (16 KiB each for 128 rows),
+// each in the 128-byte swizzled layout; one box instead of two halves the
+// TMA unit's per-box cost, which bounds the ring (measured on GB300: a 64 KiB
+// slot of four 16 KiB boxes takes 0.62 us, of two 32 KiB boxes 0.45 us).
+__device__ __forceinline__ void tma_load_pair(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                              int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(0)
+      : "memory");
+}
+
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
                                             int y) {
   asm volatile(
@@ -279,9 +293,8 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
-k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUtensorMap mapAl,
+k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUtensorMap mapB2,
           const __grid_constant__ CUtensorMap mapBh, const __grid_constant__ CUtensorMap mapBl,
-          const __grid_constant__ CUtensorMap mapBh4, const __grid_constant__ CUtensorMap mapBl4,
           const __grid_constant__ CUtensorMap mapOh, const __grid_constant__ CUtensorMap mapOl,
           const TcParams P) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -306,12 +319,10 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
   }
 
   if (threadIdx.x == 32) {   // descriptors into the cache while the previous kernel runs
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapAh)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapAl)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapA2)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapB2)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBh)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBl)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBh4)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBl4)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapOh)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapOl)) : "memory");
   }
@@ -349,13 +360,10 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
       unsigned char* st = smem + i * STAGE_BYTES;
       const int kt = blk.k0 + i;
       mbar_expect_tx_only(&full[i], 2 * TILE_BYTES);
-      if (a_static) {
-        tma_load_2d(st, &mapAh, &full[i], kt * BK, blk.rb * BM);
-        tma_load_2d(st + TILE_BYTES, &mapAl, &full[i], kt * BK, blk.rb * BM);
-      } else {
-        tma_load_2d(st + 2 * TILE_BYTES, &mapBh, &full[i], kt * BK, blk.cb * BN);
-        tma_load_2d(st + 3 * TILE_BYTES, &mapBl, &full[i], kt * BK, blk.cb * BN);
-      }
+      if (a_static)
+        tma_load_pair(st, &mapA2, &full[i], kt * BK, blk.rb * BM);
+      else
+        tma_load_pair(st + 2 * TILE_BYTES, &mapB2, &full[i], kt * BK, blk.cb * BN);
     }
   }
   // the rest waits for the previous kernel
@@ -382,8 +390,8 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
         break;
       }
       unsigned char* st = smem + s * STAGE_BYTES;
-      unsigned char *a_hi = st, *a_lo = st + TILE_BYTES, *b_hi = st + 2 * TILE_BYTES,
-                    *b_lo = st + 3 * TILE_BYTES;
+      // planes of the slot: A hi, A lo, B hi, B lo (a pair lands as hi then lo)
+      unsigned char *a_hi = st, *b_hi = st + 2 * TILE_BYTES, *b_lo = st + 3 * TILE_BYTES;
       const int kt = blk.k0 + i;            // K tile index (32 wide)
       const bool pre = i < npre;            // the factor operand is already on its way
       const bool load_a = !(pre && a_static), load_b = !(pre && !a_static);
@@ -414,14 +422,10 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
       }
       if (lane == 0) {
         mbar_expect_tx(&full[s], bytes);
-        if (load_a) {
-          tma_load_2d(a_hi, &mapAh, &full[s], kt * BK, blk.rb * BM);
-          tma_load_2d(a_lo, &mapAl, &full[s], kt * BK, blk.rb * BM);
-        }
+        if (load_a) tma_load_pair(a_hi, &mapA2, &full[s], kt * BK, blk.rb * BM);   // a_lo follows
         if (!load_b) {
-        } else if (P.mode == MODE_STAGE1 && valid == 0xFu) {   // inside the band: one box per plane
-          tma_load_2d(b_hi, &mapBh4, &full[s], kt * BK, blk.cb * BN);
-          tma_load_2d(b_lo, &mapBl4, &full[s], kt * BK, blk.cb * BN);
+        } else if (P.mode == MODE_STAGE1 && valid == 0xFu) {   // inside the band: one box, both planes
+          tma_load_pair(b_hi, &mapB2, &full[s], kt * BK, blk.cb * BN);
         } else if (P.mode == MODE_STAGE1) {
           for (int sub = 0; sub < 4; ++sub) {
             if (!(valid & (1u << sub))) continue;
@@ -430,8 +434,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapAh, const __grid_constant__ CUt
             tma_load_2d(b_lo + sub * 4096, &mapBl, &full[s], kt * BK, y);
           }
         } else {
-          tma_load_2d(b_hi, &mapBh, &full[s], kt * BK, blk.cb * BN);
-          tma_load_2d(b_lo, &mapBl, &full[s], kt * BK, blk.cb * BN);
+          tma_load_pair(b_hi, &mapB2, &full[s], kt * BK, blk.cb * BN);   // b_lo follows
         }
       }
       __syncwarp();
@@ -634,6 +637,24 @@ bool make_map(CUtensorMap* map, const float* base, int64_t rows, int64_t cols, i
   return r == CUDA_SUCCESS;
 }
 
+// The hi/lo pair of a 2-D fp32 matrix whose lo plane starts plane_bytes
+// after its hi plane, as a rank-3 tensor (columns, rows, plane): boxes of 32
+// columns x box_rows rows x both planes, 128-byte swizzle.
+bool make_map_pair(CUtensorMap* map, const float* hi, const float* lo, int64_t rows, int64_t cols,
+                   int64_t ld, int box_rows) {
+  if (!get_encode()) return false;
+  const int64_t plane_bytes = (const char*)lo - (const char*)hi;
+  if (plane_bytes < rows * ld * 4 || plane_bytes % 16) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)rows, 2u};
+  cuuint64_t strides[2] = {(cuuint64_t)(ld * 4), (cuuint64_t)plane_bytes};
+  cuuint32_t box[3] = {32u, (cuuint32_t)box_rows, 2u};
+  cuuint32_t estr[3] = {1u, 1u, 1u};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, (void*)hi, dims, strides, box,
+                        estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 bool g_attr_done = false;
 std::mutex g_attr_mu;
 
@@ -670,16 +691,14 @@ bool tc_band_maps(TcMaps& maps, const TcOperands& op) {
   // stage 1: A = L^B (mp x mp), B = E^T (np x mp) in 32-row boxes
   // stage 2: A = M (mp x np), B = L^A (np x np)
   bool ok = true;
-  ok &= make_map(&maps.LBh, op.LBH, op.mp, op.mp, op.mp, BM);
-  ok &= make_map(&maps.LBl, op.LBL, op.mp, op.mp, op.mp, BM);
+  ok &= make_map_pair(&maps.LB2, op.LBH, op.LBL, op.mp, op.mp, op.mp, BM);
   ok &= make_map(&maps.Eth, op.EtH, op.np, op.mp, op.mp, 32);
   ok &= make_map(&maps.Etl, op.EtL, op.np, op.mp, op.mp, 32);
-  ok &= make_map(&maps.Eth4, op.EtH, op.np, op.mp, op.mp, BN);
-  ok &= make_map(&maps.Etl4, op.EtL, op.np, op.mp, op.mp, BN);
+  ok &= make_map_pair(&maps.Et2, op.EtH, op.EtL, op.np, op.mp, op.mp, BN);
   ok &= make_map(&maps.Mh, op.MH, op.mp, op.np, op.np, BM);
   ok &= make_map(&maps.Ml, op.ML, op.mp, op.np, op.np, BM);
-  ok &= make_map(&maps.LAh, op.LAH, op.np, op.np, op.np, BN);
-  ok &= make_map(&maps.LAl, op.LAL, op.np, op.np, op.np, BN);
+  ok &= make_map_pair(&maps.M2, op.MH, op.ML, op.mp, op.np, op.np, BM);
+  ok &= make_map_pair(&maps.LA2, op.LAH, op.LAL, op.np, op.np, op.np, BN);
   ok &= make_map(&maps.X32, op.X, op.mp, op.np, op.np, 32);   // stage-2 reduce target
   return ok;
 }
@@ -711,11 +730,11 @@ int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, in
   dim3 grid(width, rhi - rlo + 1);
   cudaError_t e;
   if (stage == 1)
-    e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.LBh, maps.LBl, maps.Eth,
-                   maps.Etl, maps.Eth4, maps.Etl4, maps.Mh, maps.Ml, P);
-  else
-    e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.Mh, maps.Ml, maps.LAh,
-                   maps.LAl, maps.LAh, maps.LAl, maps.X32, maps.X32, P);
+    e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.LB2, maps.Et2, maps.Eth,
+                   maps.Etl, maps.Mh, maps.Ml, P);
+  else   // (the 32-row E^T maps are not read in stage 2)
+    e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.M2, maps.LA2, maps.Eth,
+                   maps.Etl, maps.X32, maps.X32, P);
   return e == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
 }
 
@@ -741,9 +760,9 @@ extern "C" int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C,
   BK_CUDA_OK(cudaMemsetAsync(status, 0, 256, s));
   k_split<<<(unsigned)(((int64_t)M * K + 255) / 256), 256, 0, s>>>(A, (int64_t)M * K, Ah, Al);
   k_split<<<(unsigned)(((int64_t)N * K + 255) / 256), 256, 0, s>>>(B, (int64_t)N * K, Bh, Bl);
-  CUtensorMap mA, mAl, mB, mBl;
-  if (!make_map(&mA, Ah, M, K, K, BM) || !make_map(&mAl, Al, M, K, K, BM) ||
-      !make_map(&mB, Bh, N, K, K, BN) || !make_map(&mBl, Bl, N, K, K, BN))
+  CUtensorMap mA2, mB2, mBh, mBl;
+  if (!make_map_pair(&mA2, Ah, Al, M, K, K, BM) || !make_map_pair(&mB2, Bh, Bl, N, K, K, BN) ||
+      !make_map(&mBh, Bh, N, K, K, BN) || !make_map(&mBl, Bl, N, K, K, BN))
     return BAKRON_ERR_CUDA;
   TcParams P{};
   P.mode = MODE_DENSE;
@@ -754,7 +773,7 @@ extern "C" int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C,
   P.status = status;
   P.spin_cycles = spin_cycles_from_env();
   dim3 grid(N / BN, M / BM);
-  k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(mA, mAl, mB, mBl, mB, mBl, mB, mBl, P);
+  k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mBh, mBl, mBh, mBl, P);
   BK_CUDA_OK(cudaGetLastError());
   return bakron_read_status(workspace, stream);
 }

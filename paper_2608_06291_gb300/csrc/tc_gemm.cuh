@@ -17,9 +17,10 @@ struct TcOperands {
 
 // TMA descriptors of every operand plane (built on the host per solve call).
 struct TcMaps {
-  CUtensorMap LBh, LBl, Eth, Etl, Mh, Ml, LAh, LAl;
-  CUtensorMap Eth4, Etl4;   // E^T planes in 128-row boxes (whole stage-1 B operand)
-  CUtensorMap X32;          // X in 32 x 32 boxes: stage-2 TMA reduce-add target
+  CUtensorMap LB2, Et2, M2, LA2;   // hi/lo pairs in one box (32 columns x 128 rows x 2 planes)
+  CUtensorMap Eth, Etl;            // E^T planes in 32-row boxes (stage-1 sub-tiles at the band's edge)
+  CUtensorMap Mh, Ml;              // M planes in 128-row boxes: stage-1 TMA store targets
+  CUtensorMap X32;                 // X in 32 x 32 boxes: stage-2 TMA reduce-add target
 };
 
 bool tc_band_maps(TcMaps& maps, const TcOperands& op);
