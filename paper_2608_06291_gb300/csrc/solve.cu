@@ -162,7 +162,8 @@ int build_leaf_blocks(const FactorLayout& fl, char* f, cudaStream_t s) {
 // x / s is evaluated as the exact product x * fl(1/s), rounded once to an
 // integer; fl(1/s) can differ from 1/s by half an ulp, which only matters
 // within 1e-6 grid units of a rounding boundary.
-// Outputs: codes, X (pre-rounding values) and E^T as a tf32 hi/lo pair.
+// Outputs: codes, X (pre-rounding values), E^T as a tf32 hi/lo pair and in
+// fp32, and the tile's final G (for the window of the tiles below it).
 // Three helper warps, so that each of the SM's four schedulers runs one warp
 // of the leaf (warp w issues from scheduler w mod 4) and the chain shares its
 // scheduler with nobody; 12 rows each (the last one's rows 32..35 are padding
@@ -208,7 +209,7 @@ struct LeafSmem {
   float Xs[TILE][TILE];                   // W after inbound updates
   __align__(16) float LBs[TILE][36];      // stride 36: conflict-free float4 row reads
   __align__(16) float LA0[TILE][KM];      // LA0[j][q] = L^A[J,J][q][j]
-  float T1s[TILE][TILE + 1];              // left neighbour's feedback: initial G (absorbing leaf)
+  float T1s[TILE][TILE + 1];              // T1, the initial G of a window-P leaf (P >= 1)
   __align__(16) float Ebr[4][LEAF_ROWS_PADDED];   // errors of a step, by row (ring of 4 steps)
   float Part[4][LEAF_HELPERS][TILE];              // partial pre of a step (ring of 4 steps)
   float4 Lsub[TILE];                              // (L^B[p][p-1], L^B[p][p-2], L^B[p][p-3], 0)
@@ -286,7 +287,8 @@ __device__ __forceinline__ void copy_block(float* dst, const float* src, int t) 
 
 // Rounds tile (I, J); run by threads 0 .. LEAF_THREADS-1 of the CTA.  With
 // PDL, the factor blocks and the grid (read-only during the solve, the grid
-// written by the solve's first kernel, more than one kernel ago) are loaded
+// written by the solve's first kernel, more than one kernel ago), and the
+// window's terms from tiles two or more anti-diagonals back, are handled
 // before waiting for the previous kernel.
 //
 // A window-P leaf (1 <= P <= LEAF_WINDOW) also applies everything the P
