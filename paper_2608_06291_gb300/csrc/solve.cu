@@ -213,6 +213,7 @@ struct LeafSmem {
   __align__(16) float Ebr[4][LEAF_ROWS_PADDED];   // errors of a step, by row (ring of 4 steps)
   float Part[4][LEAF_HELPERS][TILE];              // partial pre of a step (ring of 4 steps)
   float4 Lsub[TILE];                              // (L^B[p][p-1], L^B[p][p-2], L^B[p][p-3], 0)
+  __align__(16) float4 Srzl[TILE][TILE];          // (s, 1/s, -z, 0) per entry
   union {
     struct {   // prologue of a window-P leaf: its window, staged one d at a time
       // buffer b holds the operands of one d: [0] E[I, J-d] k-major
@@ -222,10 +223,7 @@ struct LeafSmem {
       __align__(16) float B[3][4][TILE][KM];
     } pro;
     struct {   // the wavefront
-      union {
-        __align__(16) float4 Srzl[TILE][TILE];  // (s, 1/s, -z, 0) per entry
-        float EsT[TILE][TILE + 1];              // after the wavefront: E transposed
-      };
+      float EsT[TILE][TILE + 1];              // after the wavefront: E transposed
       __align__(8) float2 XE[TILE][TILE];     // (pre-rounding value, error)
       uint8_t Cs[TILE][TILE];
     } w;
@@ -382,6 +380,13 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     scv[k] = real ? a.scales[og] : 1.f;
     zv[k] = real ? a.zeros[og] : 0.f;
   }
+  // the grid of every entry, and the error ring, before the wait
+#pragma unroll
+  for (int k = 0; k < LEAF_PER_THREAD; ++k) {
+    const int e = t + k * LEAF_THREADS;
+    S.Srzl[e / TILE][e % TILE] = make_float4(scv[k], 1.f / scv[k], -zv[k], 0.f);
+  }
+  for (int e = t; e < 4 * LEAF_ROWS_PADDED; e += LEAF_THREADS) (&S.Ebr[0][0])[e] = 0.f;
   if (P >= 2) {
 #pragma unroll
     for (int d = 2; d <= P && d <= 3; ++d) {
@@ -435,16 +440,10 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     S.Xs[pr + i][pc] = xv[i][0];
     S.Xs[pr + i][pc + 1] = xv[i][1];
   }
-#pragma unroll
-  for (int k = 0; k < LEAF_PER_THREAD; ++k) {
-    const int e = t + k * LEAF_THREADS;
-    const int p = e / TILE, c = e % TILE;
-    S.u.w.Srzl[p][c] = make_float4(scv[k], 1.f / scv[k], -zv[k], 0.f);
-  }
+
   if (t < TILE)
     S.Lsub[t] = make_float4(t >= 1 ? S.LBs[t][t - 1] : 0.f, t >= 2 ? S.LBs[t][t - 2] : 0.f,
                             t >= 3 ? S.LBs[t][t - 3] : 0.f, 0.f);
-  for (int e = t; e < 4 * LEAF_ROWS_PADDED; e += LEAF_THREADS) (&S.Ebr[0][0])[e] = 0.f;
   leaf_sync();
   // ---------------------------------------------------------- the wavefront
   // Steps go in intervals of two (steps 2k and 2k+1) with one barrier at the
@@ -516,7 +515,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     };
     // (s, 1/s, -z) and the sub-diagonal L^B of the next interval's entries are
     // loaded one interval ahead
-    float4 g0 = S.u.w.Srzl[(0 - q) & (TILE - 1)][q], g1 = S.u.w.Srzl[(1 - q) & (TILE - 1)][q];
+    float4 g0 = S.Srzl[(0 - q) & (TILE - 1)][q], g1 = S.Srzl[(1 - q) & (TILE - 1)][q];
     float4 lb0 = S.Lsub[(0 - q) & (TILE - 1)], lb1 = S.Lsub[(1 - q) & (TILE - 1)];
     leaf_sync();   // the helpers' pre of steps 0 and 1
 #pragma unroll 1
@@ -529,8 +528,8 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
       const float pre1 = (pb[0] + pb[TILE]) + pb[2 * TILE];
       const float4 g0c = g0, g1c = g1, lb0c = lb0, lb1c = lb1;
       const int n0 = (d0 + 2 - q) & (TILE - 1), n1 = (d1 + 2 - q) & (TILE - 1);
-      g0 = S.u.w.Srzl[n0][q];
-      g1 = S.u.w.Srzl[n1][q];
+      g0 = S.Srzl[n0][q];
+      g1 = S.Srzl[n1][q];
       lb0 = S.Lsub[n0];
       lb1 = S.Lsub[n1];
       step(d0, false, pre0, g0c, lb0c);

@@ -109,6 +109,39 @@ def test_solve_leaf_blocks(block, monkeypatch):
     _assert_parity_or_certified_tie(_solve_small(512, 544, 4242, bits=4))
 
 
+def test_leaf_blocks_of_16_with_groups(monkeypatch):
+    """Blocks of 16 (windows up to 15) with 32-column groups: the per-entry
+    grid of the window's tiles and of the leaves that absorb them."""
+    monkeypatch.setenv("BAKRON_LEAF_BLOCK", "16")
+    _assert_parity_or_certified_tie(_solve_small(512, 544, 4343, bits=3, group=32))
+
+
+def test_b_identity_is_gptq_on_gpu(monkeypatch):
+    """B = I: the solve is GPTQ per row under the input-side Hessian (Sec. 1).
+    The GPU's codes equal the oracle's textbook GPTQ loop (upper Cholesky of
+    H^-1, error / U_ii) under H = (L L^T)^-1, whose GPTQ updates are exactly
+    the unit-lower factor L the GPU was given; small enough that no decision
+    falls inside the tie band."""
+    monkeypatch.setenv("BAKRON_LEAF_BLOCK", "4")   # band products as well as leaves
+    m, n = 120, 200
+    W, A, B = WL.small_problem(m, n, 515)
+    f, LA32, _ = oracle_factors_fp32(A, B, 0.01)
+    dev = "cuda"
+    fac = P.bakron_set_factors(torch.from_numpy(LA32).to(dev), torch.eye(m, device=dev))
+    codes, scales, zeros, X = P.bakron_solve(W.to(dev), fac, 4, 0, prerounding=True)
+    torch.cuda.synchronize()
+    W64 = to_np(W)
+    g = O.quant_grid(W64, 4, 0)
+    S, Z = g.expand(n)
+    LA = LA32.astype(np.float64)
+    H = np.linalg.inv(LA @ LA.T)
+    gp = O.gptq_rows(W64, H, S, Z, g.qmax)
+    got = codes.cpu().numpy().astype(np.int64)
+    st = compare_codes(W64, got, g, LA, np.eye(m), gp.codes)
+    assert st["cert_mismatch_outside_band"] == 0, st
+    assert st["raw_match"] == 1.0, st
+
+
 @pytest.mark.parametrize("bits", [1, 2, 3, 8])
 def test_solve_matches_oracle_bits(bits):
     _assert_parity(_solve_small(70, 90, 77 + bits, bits=bits))
