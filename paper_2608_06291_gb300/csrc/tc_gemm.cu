@@ -302,7 +302,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint64_t* bars = (uint64_t*)(smem + STAGES * STAGE_BYTES);
   uint64_t* full = bars;                 // [STAGES] smem stage loaded
-  uint64_t* empty = bars + STAGES;       // [STAGES] smem stage consumed by the MMAs
+  // bars + STAGES .. 2 STAGES - 1: unused (a slot is free when its stage's accF arrives)
   uint64_t* accum = bars + 2 * STAGES;   // [1] every MMA of the CTA complete
   uint64_t* accF = accum + 1;            // [NACC] accumulator holds a finished K stage
   uint64_t* accE = accum + 1 + NACC;     // [NACC] accumulator read out by the epilogue
@@ -329,7 +329,6 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
     }
     mbar_init(accum, 1);
     for (int a = 0; a < NACC; ++a) {
@@ -377,9 +376,14 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
     int issued = 0;
     for (int i = 0; i < nk; ++i) {
       const int s = i % STAGES;
-      const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
       bool ok = true;
-      if (lane == 0) ok = mbar_wait(&empty[s], ph ^ 1u, P.spin_cycles);
+      // slot s was last read by the MMAs of stage j = i - STAGES, which are
+      // complete when their accumulator's commit arrives (accF); that barrier
+      // cannot have moved on to stage j + NACC yet, which needs this load
+      if (lane == 0 && i >= STAGES) {
+        const int j = i - STAGES;
+        ok = mbar_wait(&accF[j % NACC], (uint32_t)(j / NACC) & 1u, P.spin_cycles);
+      }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok || *abort_flag) {
         if (lane == 0 && !ok) { raise_status(P.status, BAKRON_ERR_TIMEOUT); *abort_flag = 1; }
@@ -486,8 +490,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
           mma_tf32(d, dah + o, dbl + o, idesc, 1u);
           mma_tf32(d, dal + o, dbh + o, idesc, 1u);
         }
-        mma_commit(&empty[s]);    // frees the smem stage when these MMAs are done
-        mma_commit(&accF[a]);     // hands the stage's sum to the epilogue
+        mma_commit(&accF[a]);     // the stage's sum to the epilogue; its slot to the producer
       }
       if (nk > 0) mma_commit(accum);  // tracks every MMA issued above
       else mbar_arrive(accum);
