@@ -159,6 +159,60 @@ def quant_grid(W: np.ndarray, bits: int, group: int = 0) -> Grid:
     return Grid(s, z, qmax, group)
 
 
+def symmetric_candidates(amax, levels: int, shrink_steps: int) -> np.ndarray:
+    """Candidate scales of the symmetric alphabet (Appendix "Experiments").
+
+    The scale starts at the row's maximal |w| divided by l and may shrink by
+    up to a factor of 2: candidate k = 0..K (K = shrink_steps) is
+        t_k = fl32((2K - k) / (2K l)),   s_k = fl32(amax * t_k)
+    (K = 0: the single candidate t_0 = fl32(1 / l)).  Each is one correctly
+    rounded fp32 operation on exact operands, so these are bit-identical to an
+    fp32 implementation.  An all-zero row/group uses amax = 1."""
+    amax = F32(amax)
+    if amax == 0:
+        amax = F32(1)
+    if shrink_steps == 0:
+        t = np.array([F32(F64(1) / F64(levels))], dtype=F32)
+    else:
+        k = np.arange(shrink_steps + 1, dtype=F64)
+        t = ((2 * shrink_steps - k) / F64(2 * shrink_steps * levels)).astype(F32)
+    return (F64(amax) * t.astype(F64)).astype(F32)
+
+
+def symmetric_errors(w, scales, levels: int) -> np.ndarray:
+    """Squared rounding error of the values w under each candidate scale:
+    sum_q (s * clamp(rint(w_q / s), -l, l) - w_q)^2, in fp64."""
+    w = np.asarray(w, dtype=F32).astype(F64)
+    s = np.asarray(scales, dtype=F32).astype(F64)[:, None]
+    c = np.clip(np.rint(w[None, :] / s), -levels, levels)
+    return ((s * c - w[None, :]) ** 2).sum(axis=1)
+
+
+def symmetric_grid(W: np.ndarray, levels: int, group: int = 0,
+                   shrink_steps: int = 50) -> Grid:
+    """The paper's experimental alphabet (Appendix "Experiments"): codes
+    {-l, ..., +l} per row (or per (row, group)), scale = max |w| / l shrunk by
+    the candidate factor in [1/2, 1] (``symmetric_candidates``) whose
+    round-to-nearest squared error over the row is least (the first such
+    candidate, i.e. the largest scale, on exact ties).  Expressed in the
+    affine form of ``Grid``: z = l, qmax = 2 l, so code c stands for the
+    integer c - l and value s (c - l)."""
+    W = np.asarray(W, dtype=F32)
+    m, n = W.shape
+    g = n if group == 0 else group
+    if n % g:
+        raise ValueError("group must divide n")
+    G = n // g
+    s = np.empty((m, G), dtype=F32)
+    for i in range(m):
+        for j in range(G):
+            w = W[i, j * g:(j + 1) * g]
+            cand = symmetric_candidates(np.abs(w).max(), levels, shrink_steps)
+            err = symmetric_errors(w, cand, levels)
+            s[i, j] = cand[int(np.argmin(err))]
+    return Grid(s, np.full((m, G), F32(levels)), 2 * levels, group)
+
+
 def integer_grid(m: int) -> Grid:
     """The paper's plain round() onto Z: s = 1, z = 0, no clamping."""
     return Grid(np.ones((m, 1), F32), np.zeros((m, 1), F32), None, 0)
