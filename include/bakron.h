@@ -128,6 +128,52 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw,
                  int sync, void* stream);
 
 /*
+ * bakron_grid_symmetric -- the quantisation grid of the paper's experiments
+ * (Appendix "Experiments"): the symmetric alphabet {-l, ..., +l}, one scale
+ * per row (group_size 0) or per (row, group of group_size columns), chosen
+ * from max |w| / l by a squared-error search over shrink factors in [1/2, 1]:
+ *   candidate k = 0..K (K = shrink_steps):
+ *     s_k = fl(amax * fl((2K - k) / (2K l)))   (K = 0: s_0 = fl(amax * fl(1/l)))
+ *   error_k = sum over the row/group of (s_k clamp(rint(w / s_k), -l, l) - w)^2
+ * and the least error_k wins (the first, i.e. the larger scale, on ties).  An
+ * all-zero row/group uses amax = 1.  The paper fixes l = 3 and a shrink of
+ * "up to a factor of 2"; the number of steps is the caller's (K = 50 gives
+ * factors 1.00, 0.99, ..., 0.50).
+ *   W        device, as bakron_solve (read only)
+ *   levels   l, 1..127 (2l + 1 codes)
+ *   shrink_steps K, 0..1024
+ *   scales, zeros  device, m x G fp32, written: the chosen s and z = l, so
+ *            that the affine form of bakron_solve holds: code c in 0..2l has
+ *            value s (c - l)
+ * The errors are summed in fp32 (per-thread partial sums, then a fixed
+ * tree); rows whose two best candidates lie within that rounding may pick
+ * either.  Asynchronous on `stream`; returns BAKRON_ERR_INVALID_ARG before
+ * any launch for bad arguments.  Pass the result to bakron_solve_with_grid
+ * with qmax = 2 l.
+ */
+int bakron_grid_symmetric(const void* W, int wdtype, int m, int n, int64_t ldw,
+                          int levels, int group_size, int shrink_steps,
+                          float* scales, float* zeros, void* stream);
+
+/*
+ * bakron_solve_with_grid -- bakron_solve with the caller's grid instead of
+ * the min-max one: the same rounding (Alg. 5) onto codes 0..qmax, code c of
+ * row p / group g standing for s[p, g] (c - z[p, g]).
+ *   qmax     1..255 (codes are uint8)
+ *   scales, zeros  device, m x G fp32 (G = 1 or n / group_size), read only;
+ *            each scale finite and > 0, each zero an integer in [0, qmax]
+ *            (not checked: other values give meaningless codes, but every
+ *            memory access stays in bounds)
+ * Other arguments, outputs, `sync` and errors as bakron_solve.  The solve's
+ * schedule comes from the same per-shape table as bakron_solve.
+ */
+int bakron_solve_with_grid(const void* W, int wdtype, int m, int n, int64_t ldw,
+                           const void* factors, int qmax, int group_size,
+                           const float* scales, const float* zeros,
+                           uint8_t* codes, float* prerounding, void* workspace,
+                           size_t workspace_bytes, int sync, void* stream);
+
+/*
  * bakron_autotune -- choose, for this problem shape, which kernels run each
  * node of the recursion, by timing candidate schedules on the caller's data.
  * No counterpart in the paper: Alg. 5 fixes the recursion (halving of the

@@ -7,7 +7,7 @@ ctypes binding with the same entry-point names.
 from .bakron import (BakronError, Factors, alloc_workspace, bakron_diag_gemm_tf32x3,  # noqa: F401
                      bakron_diag_mma_rate,
                      bakron_autotune, bakron_autotune_clear, bakron_get_factors,
-                     bakron_get_tuning,
+                     bakron_get_tuning, bakron_grid_symmetric, bakron_solve_with_grid,
                      bakron_last_launches, bakron_prepare, bakron_profile_enable,
                      bakron_profile_read, bakron_read_status, bakron_set_factors, bakron_solve,
                      bakron_solve_noalloc,

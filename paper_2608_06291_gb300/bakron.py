@@ -52,6 +52,11 @@ def lib() -> ctypes.CDLL:
     L.bakron_get_factors.restype = i32
     L.bakron_solve.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, vp, sz, i32, vp]
     L.bakron_solve.restype = i32
+    L.bakron_grid_symmetric.argtypes = [vp, i32, i32, i32, i64, i32, i32, i32, vp, vp, vp]
+    L.bakron_grid_symmetric.restype = i32
+    L.bakron_solve_with_grid.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp,
+                                         vp, sz, i32, vp]
+    L.bakron_solve_with_grid.restype = i32
     L.bakron_solve_noalloc.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, i32, vp]
     L.bakron_solve_noalloc.restype = i32
     L.bakron_read_status.argtypes = [vp, vp]
@@ -164,18 +169,21 @@ def bakron_get_factors(f: Factors, stream=None):
     return LA, LB, rA, rB
 
 
+def _w_dtype(W):
+    if not W.is_cuda or W.dim() != 2 or W.stride(1) != 1:
+        raise ValueError("W must be a 2-D CUDA tensor with unit column stride")
+    if W.dtype == torch.float32:
+        return F32
+    if W.dtype == torch.bfloat16:
+        return BF16
+    raise ValueError("W must be float32 or bfloat16")
+
+
 def bakron_solve(W, f: Factors, bits: int, group_size: int = 0, workspace=None,
                  prerounding: bool = False, sync: bool = True, out=None, stream=None):
     """Round W (CUDA fp32/bf16, unit column stride).  Returns (codes uint8,
     scales, zeros[, prerounding fp32])."""
-    if not W.is_cuda or W.dim() != 2 or W.stride(1) != 1:
-        raise ValueError("W must be a 2-D CUDA tensor with unit column stride")
-    if W.dtype == torch.float32:
-        dt = F32
-    elif W.dtype == torch.bfloat16:
-        dt = BF16
-    else:
-        raise ValueError("W must be float32 or bfloat16")
+    dt = _w_dtype(W)
     m, n = W.shape
     if (f.m, f.n) != (m, n):
         raise ValueError("factor buffer was built for a different shape")
@@ -194,6 +202,49 @@ def bakron_solve(W, f: Factors, bits: int, group_size: int = 0, workspace=None,
                             _ptr(ws), ws.numel(), 1 if sync else 0, _stream(stream))
     _check(rc, "bakron_solve")
     return (codes, scales, zeros, xpre) if prerounding else (codes, scales, zeros)
+
+
+def bakron_grid_symmetric(W, levels: int = 3, group_size: int = 0, shrink_steps: int = 50,
+                          stream=None):
+    """The paper's experimental grid: symmetric codes {-l..l} with the
+    MSE-shrunk max-abs scale per row (or per (row, group)).  Returns (scales,
+    zeros), m x G fp32, zeros = l; asynchronous on `stream`."""
+    dt = _w_dtype(W)
+    m, n = W.shape
+    G = 1 if group_size == 0 else n // group_size
+    scales = torch.empty(m, G, dtype=torch.float32, device=W.device)
+    zeros = torch.empty(m, G, dtype=torch.float32, device=W.device)
+    rc = lib().bakron_grid_symmetric(_ptr(W), dt, m, n, W.stride(0), int(levels),
+                                     int(group_size), int(shrink_steps), _ptr(scales),
+                                     _ptr(zeros), _stream(stream))
+    _check(rc, "bakron_grid_symmetric")
+    return scales, zeros
+
+
+def bakron_solve_with_grid(W, f: Factors, scales, zeros, qmax: int, group_size: int = 0,
+                           workspace=None, prerounding: bool = False, sync: bool = True,
+                           stream=None):
+    """Round W onto the caller's grid (codes 0..qmax, value s (c - z)).
+    Returns codes uint8 [, prerounding fp32]."""
+    dt = _w_dtype(W)
+    m, n = W.shape
+    if (f.m, f.n) != (m, n):
+        raise ValueError("factor buffer was built for a different shape")
+    G = 1 if group_size == 0 else n // group_size
+    for t, name in ((scales, "scales"), (zeros, "zeros")):
+        if (not t.is_cuda or t.dtype != torch.float32 or tuple(t.shape) != (m, G)
+                or not t.is_contiguous()):
+            raise ValueError(f"{name} must be a contiguous CUDA float32 tensor of shape {(m, G)}")
+    dev = W.device
+    codes = torch.empty(m, n, dtype=torch.uint8, device=dev)
+    xpre = torch.empty(m, n, dtype=torch.float32, device=dev) if prerounding else None
+    ws = workspace if workspace is not None else alloc_workspace(m, n, dev)
+    rc = lib().bakron_solve_with_grid(_ptr(W), dt, m, n, W.stride(0), _ptr(f.buf), int(qmax),
+                                      int(group_size), _ptr(scales), _ptr(zeros), _ptr(codes),
+                                      _ptr(xpre), _ptr(ws), ws.numel(), 1 if sync else 0,
+                                      _stream(stream))
+    _check(rc, "bakron_solve_with_grid")
+    return (codes, xpre) if prerounding else codes
 
 
 def bakron_autotune(W, f: Factors, bits: int, group_size: int = 0, workspace=None,

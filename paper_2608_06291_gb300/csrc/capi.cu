@@ -10,9 +10,12 @@
 namespace bakron {
 int prepare_impl(const float* A, const float* B, int m, int n, float damp, void* factors,
                  void* workspace, cudaStream_t s);
-int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int bits,
+int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
                int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s, const Tuning* force);
+               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given);
+int launch_grid_sym(const void* W, int wdt, int m, int n, int64_t ldw, int levels,
+                    int group_size, int shrink_steps, float* scales, float* zeros,
+                    cudaStream_t s);
 
 // Largest side accepted.  Keeps every index product inside int64 and every
 // grid dimension inside CUDA's limits (mp / 32 tiles per side).
@@ -121,8 +124,39 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw, const voi
   if (group_size < 0 || (group_size > 0 && n % group_size != 0)) return BAKRON_ERR_INVALID_ARG;
   if (workspace_bytes < SolveLayout(m, n).bytes) return BAKRON_ERR_WORKSPACE;
   cudaStream_t s = (cudaStream_t)stream;
-  int rc = solve_impl(W, wdtype, m, n, ldw, factors, bits, group_size, codes, scales, zeros,
-                      prerounding, workspace, s, nullptr);
+  int rc = solve_impl(W, wdtype, m, n, ldw, factors, (1 << bits) - 1, group_size, codes, scales,
+                      zeros, prerounding, workspace, s, nullptr, false);
+  if (rc != BAKRON_OK || !sync) return rc;
+  return bakron_read_status(workspace, stream);
+}
+
+int bakron_grid_symmetric(const void* W, int wdtype, int m, int n, int64_t ldw, int levels,
+                          int group_size, int shrink_steps, float* scales, float* zeros,
+                          void* stream) {
+  if (!W || !scales || !zeros || !dims_ok(m, n)) return BAKRON_ERR_INVALID_ARG;
+  if (wdtype != BAKRON_F32 && wdtype != BAKRON_BF16) return BAKRON_ERR_INVALID_ARG;
+  if (ldw < n || levels < 1 || levels > 127) return BAKRON_ERR_INVALID_ARG;
+  if (shrink_steps < 0 || shrink_steps > 1024) return BAKRON_ERR_INVALID_ARG;
+  if (group_size < 0 || (group_size > 0 && n % group_size != 0)) return BAKRON_ERR_INVALID_ARG;
+  return launch_grid_sym(W, wdtype, m, n, ldw, levels, group_size, shrink_steps, scales, zeros,
+                         (cudaStream_t)stream);
+}
+
+int bakron_solve_with_grid(const void* W, int wdtype, int m, int n, int64_t ldw,
+                           const void* factors, int qmax, int group_size, const float* scales,
+                           const float* zeros, uint8_t* codes, float* prerounding,
+                           void* workspace, size_t workspace_bytes, int sync, void* stream) {
+  if (!W || !factors || !codes || !scales || !zeros || !workspace || !dims_ok(m, n))
+    return BAKRON_ERR_INVALID_ARG;
+  if (wdtype != BAKRON_F32 && wdtype != BAKRON_BF16) return BAKRON_ERR_INVALID_ARG;
+  if (ldw < n || qmax < 1 || qmax > 255) return BAKRON_ERR_INVALID_ARG;
+  if (group_size < 0 || (group_size > 0 && n % group_size != 0)) return BAKRON_ERR_INVALID_ARG;
+  if (workspace_bytes < SolveLayout(m, n).bytes) return BAKRON_ERR_WORKSPACE;
+  cudaStream_t s = (cudaStream_t)stream;
+  // the grid is only read when grid_given is set
+  int rc = solve_impl(W, wdtype, m, n, ldw, factors, qmax, group_size, codes,
+                      const_cast<float*>(scales), const_cast<float*>(zeros), prerounding,
+                      workspace, s, nullptr, true);
   if (rc != BAKRON_OK || !sync) return rc;
   return bakron_read_status(workspace, stream);
 }

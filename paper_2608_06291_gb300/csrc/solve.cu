@@ -62,6 +62,84 @@ __global__ void k_grid(const void* W, int wdt, int m, int n, int64_t ldw, int gs
   }
 }
 
+// Symmetric alphabet {-l, ..., +l} of the paper's experiments (Appendix
+// "Experiments"): per (row, group) the scale starts at max |w| / l and may
+// shrink by up to a factor of 2; of the K + 1 candidates
+//     s_k = fl(amax * fl((2K - k) / (2K l))),  k = 0..K   (K = 0: fl(1 / l))
+// the one with the least round-to-nearest squared error
+//     sum_q (s_k clamp(rint(w_q / s_k), -l, l) - w_q)^2
+// wins, the first on ties.  An all-zero row/group uses amax = 1.  Stored in
+// the affine form the solve reads: z = l, codes 0..2l.  One block of
+// GRID_SYM_THREADS per (row, group); the row is re-read from L1 per
+// candidate; sums are fp32 per thread, then a fixed tree.
+constexpr int GRID_SYM_THREADS = 256;
+
+__device__ __forceinline__ float block_sum_or_max(float v, bool is_max, float* red) {
+  for (int o = 16; o; o >>= 1) {
+    const float u = __shfl_xor_sync(0xffffffffu, v, o);
+    v = is_max ? fmaxf(v, u) : v + u;
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __syncthreads();                       // red[] free from the last call
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  v = red[0];
+  for (int w = 1; w < GRID_SYM_THREADS / 32; ++w) v = is_max ? fmaxf(v, red[w]) : v + red[w];
+  return v;
+}
+
+__global__ void __launch_bounds__(GRID_SYM_THREADS)
+    k_grid_sym(const void* W, int wdt, int m, int n, int64_t ldw, int gsz, int G, int levels,
+               int K, float* scales, float* zeros) {
+  __shared__ float red[GRID_SYM_THREADS / 32];
+  const int64_t items = (int64_t)m * G;
+  // block-uniform loop: every thread of a block reaches the same barriers
+  for (int64_t item = blockIdx.x; item < items; item += gridDim.x) {
+    const int row = (int)(item / G), grp = (int)(item % G);
+    const int64_t base = (int64_t)row * ldw + (int64_t)grp * gsz;
+    auto load = [&](int c) -> float {
+      return (wdt == BAKRON_BF16) ? __bfloat162float(((const __nv_bfloat16*)W)[base + c])
+                                  : ((const float*)W)[base + c];
+    };
+    float amax = 0.f;
+    for (int c = threadIdx.x; c < gsz; c += GRID_SYM_THREADS) amax = fmaxf(amax, fabsf(load(c)));
+    amax = block_sum_or_max(amax, true, red);
+    if (amax == 0.f) amax = 1.f;
+    const float L = (float)levels;
+    float best_s = 0.f, best_err = INFINITY;
+    for (int k = 0; k <= K; ++k) {
+      const float t = K == 0 ? __fdiv_rn(1.f, L)
+                             : __fdiv_rn((float)(2 * K - k), (float)(2 * K * levels));
+      const float s = __fmul_rn(amax, t);
+      float err = 0.f;
+      for (int c = threadIdx.x; c < gsz; c += GRID_SYM_THREADS) {
+        const float v = load(c);
+        const float q = fminf(fmaxf(rintf(__fdiv_rn(v, s)), -L), L);
+        const float d = fmaf(s, q, -v);
+        err = fmaf(d, d, err);
+      }
+      err = block_sum_or_max(err, false, red);
+      if (k == 0 || err < best_err) { best_err = err; best_s = s; }
+    }
+    if (threadIdx.x == 0) {
+      scales[item] = best_s;
+      zeros[item] = L;
+    }
+  }
+}
+
+int launch_grid_sym(const void* W, int wdt, int m, int n, int64_t ldw, int levels,
+                    int group_size, int shrink_steps, float* scales, float* zeros,
+                    cudaStream_t s) {
+  const int gsz = group_size == 0 ? n : group_size;
+  const int G = n / gsz;
+  const int64_t blocks = std::min<int64_t>((int64_t)m * G, 152 * 16);
+  k_grid_sym<<<(unsigned)blocks, GRID_SYM_THREADS, 0, s>>>(
+      W, wdt, m, n, ldw, gsz, G, levels, shrink_steps, scales, zeros);
+  BK_CUDA_OK(cudaGetLastError());
+  return BAKRON_OK;
+}
+
 // X <- W widened to fp32 over the padded mp x np workspace (zeros outside).
 // Grid-stride over chunks of 8 entries of a row (np is a multiple of 128, so
 // a chunk never straddles a row), stored as two 16-byte vectors.
@@ -1255,9 +1333,11 @@ static void rec(SolveArgs& a, int k, int l) {
 }
 
 // `force`: thresholds to use instead of tuning_for(m, n) (the autotuner's candidates).
-int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int bits,
+// `grid_given`: scales and zeros hold the caller's grid (read only); otherwise
+// the min-max grid over qmax + 1 codes is computed into them first.
+int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
                int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s, const Tuning* force) {
+               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given) {
   FactorLayout fl(m, n);
   SolveLayout sl(m, n);
   char* ws = (char*)workspace;
@@ -1267,7 +1347,7 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
   a.Mt = ceil_div(m, TILE); a.Nt = ceil_div(n, TILE);
   a.gsz = group_size == 0 ? n : group_size;
   a.G = n / a.gsz;
-  a.qmax = (1 << bits) - 1;
+  a.qmax = qmax;
   a.mp = sl.mp; a.np = sl.np;
   a.X = (float*)(ws + sl.off_X);
   a.EtH = (float*)(ws + sl.off_EtH);
@@ -1314,7 +1394,7 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
   }
   reset_launch_count();
   BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_status, 0, 256, s));
-  {
+  if (!grid_given) {
     const int64_t warps = (int64_t)m * a.G;
     LaunchScope ls(kFamInit, s);
     k_grid<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(W, wdt, m, n, ldw, a.gsz, a.G,

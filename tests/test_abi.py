@@ -61,4 +61,21 @@ def test_invalid_arguments_rejected_on_host(L):
     assert L.bakron_prepare(fake, fake, 4, 4, ctypes.c_float(0.01), fake, fake, 16, None) == 5
     assert L.bakron_set_factors(None, fake, None, None, 4, 4, fake, None) == 1
     assert L.bakron_read_status(None, None) == 1
+    # symmetric grid: levels, shrink steps, group, ldw, dtype
+    g = L.bakron_grid_symmetric
+    assert g(None, 0, 4, 4, 4, 3, 0, 50, fake, fake, None) == 1
+    assert g(fake, 0, 4, 4, 4, 0, 0, 50, fake, fake, None) == 1
+    assert g(fake, 0, 4, 4, 4, 128, 0, 50, fake, fake, None) == 1
+    assert g(fake, 0, 4, 4, 4, 3, 0, -1, fake, fake, None) == 1
+    assert g(fake, 0, 4, 4, 4, 3, 0, 1025, fake, fake, None) == 1
+    assert g(fake, 0, 4, 6, 6, 3, 4, 50, fake, fake, None) == 1
+    assert g(fake, 0, 4, 6, 5, 3, 0, 50, fake, fake, None) == 1
+    assert g(fake, 2, 4, 4, 4, 3, 0, 50, fake, fake, None) == 1
+    # solve with the caller's grid: qmax, null grid, group, workspace
+    sg = L.bakron_solve_with_grid
+    assert sg(fake, 0, 4, 4, 4, fake, 0, 0, fake, fake, fake, None, fake, 1 << 30, 0, None) == 1
+    assert sg(fake, 0, 4, 4, 4, fake, 256, 0, fake, fake, fake, None, fake, 1 << 30, 0, None) == 1
+    assert sg(fake, 0, 4, 4, 4, fake, 6, 0, None, fake, fake, None, fake, 1 << 30, 0, None) == 1
+    assert sg(fake, 0, 4, 6, 6, fake, 6, 4, fake, fake, fake, None, fake, 1 << 30, 0, None) == 1
+    assert sg(fake, 0, 4, 4, 4, fake, 6, 0, fake, fake, fake, None, fake, 16, 0, None) == 5
     assert P.strerror(2) == "damped Gram is not positive definite"
