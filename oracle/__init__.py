@@ -12,3 +12,5 @@ from .bakron_oracle import (Factors, Grid, Result, bakron, bakron_antidiagonal, 
                             quantize, rev_cholesky, rtn, teacher_forced,
                             unit_lower_factor, unit_lower_factor_via_rev,
                             certificate_rows, grid_rows)
+from .hessian import (gram, kfac_factors, kronecker_hessian, rearranged_hessian,  # noqa: F401
+                      sample_quadforms, sample_sqnorms, shampoo_factors)
