@@ -429,6 +429,110 @@ def run_gpu(args):
     return 0
 
 
+def run_extra(args):
+    """One JSON line for a workload next to the solve (no graph, N = 1 only):
+      gram     K-FAC input-side factor A = X^T X / k of the 4096-feature layer
+               from k = 65536 bf16 activation rows (32 sequences of 2048
+               tokens), one bakron_gram call per step;
+      symgrid  the symmetric l = 3 grid with 50 shrink steps of the 4096 x 4096
+               weights (one bakron_grid_symmetric call per step)."""
+    import torch
+
+    import paper_2608_06291_gb300 as P
+    import workloads as WL
+
+    ws_n, rank, local = _dist()
+    if rank != 0:
+        return 0
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    P.build()
+    P.lib()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    peaks = _peaks() or {}
+    if args.workload == "gram":
+        k, d = 65536, 4096
+        g = torch.Generator(device=dev).manual_seed(4096)
+        X = (torch.randn(k, d, generator=g, device=dev)
+             * torch.linspace(0.2, 3.0, d, device=dev)).to(torch.bfloat16)
+        G = torch.empty(d, d, dtype=torch.float32, device=dev)
+        wsb = torch.empty(P.bakron_gram_workspace_bytes(d, k, False), dtype=torch.uint8,
+                          device=dev)
+
+        def step():
+            P.bakron_gram(X, alpha=1.0 / k, G=G, workspace=wsb, sync=False)
+        nb = d // 128
+        units = d * (d + 1) * k                   # 2k flops per unique entry
+        mma = nb * (nb + 1) // 2 * 2 * 128 * 128 * k
+        unit, metric = "flop/s", "K-FAC Gram X^T X / k flop/s (4096 features, 65536 bf16 rows)"
+        per_launch = 2                            # transpose-split + tensor-core Gram
+        bf16 = float(peaks.get("bf16_tflops", 1892.3))
+        roof_peak = bf16 * 1.1 / 2.25            # tf32 rate: bf16 rows are exact in tf32
+        roof_src = "of measured: bf16_tflops x 1.1/2.25 (tf32/bf16 nominal)"
+        cfg = {"workload": "kfac_gram", "k": k, "d": d, "dtype_in": "bf16",
+               "l2": "flushed (256 MiB write) between steps; X 512 MiB > L2"}
+    else:
+        cfg2 = WL.CONFIGS[2]
+        W, _, _ = WL.make(cfg2, device=dev)
+        m, n = cfg2.m, cfg2.n
+
+        def step():
+            P.bakron_grid_symmetric(W, 3, 0, 50)
+        units = m * n
+        mma = None
+        unit, metric = "entries/s", "symmetric l=3 grid, 50 shrink steps, 4096x4096 bf16 W"
+        per_launch = 1
+        # FP32-pipe operations per entry and candidate: mul, rint, max, min, 2 fma
+        roof_peak = 152 * 128 * 2.07e9 / 1e12     # lane-ops/s at the maximum SM clock (T)
+        roof_src = "152 SMs x 128 FP32 lanes x 2.07 GHz (one op per lane per clock)"
+        cfg = {"workload": "grid_symmetric", "m": m, "n": n, "levels": 3, "shrink_steps": 50,
+               "l2": "flushed (256 MiB write) between steps"}
+    for _ in range(max(3, args.warmup)):
+        flush.fill_(1)
+        step()
+    torch.cuda.synchronize()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    bus = None
+    try:
+        bus = torch.cuda.get_device_properties(dev).pci_bus_id
+    except Exception:
+        pass
+    sampler = ClockSampler(bus)
+    time.sleep(0.3)
+    torch.cuda.synchronize()
+    w0 = time.time()
+    for i in range(args.steps):
+        flush.fill_(i & 0xFF)
+        starts[i].record(stream)
+        step()
+        ends[i].record(stream)
+    torch.cuda.synchronize()
+    w1 = time.time()
+    clocks = sampler.stop(w0, w1)
+    ms = sum(a.elapsed_time(b) for a, b in zip(starts, ends)) / args.steps
+    value = units / (ms / 1e3)
+    if args.workload == "gram":
+        roof = {"bound": "tensor", "achieved": value / 1e12, "peak": roof_peak,
+                "unit": "TFLOP/s", "frac": value / 1e12 / roof_peak, "traffic": None,
+                "peak_source": roof_src,
+                "note": "algorithmic flops d(d+1)k over the whole call (split kernel included); "
+                        f"MMA flops issued {mma:.3e} per step (whole diagonal blocks)"}
+    else:
+        ops = 6.0 * units * 51
+        roof = {"bound": "alu", "achieved": ops / (ms / 1e3) / 1e12, "peak": roof_peak,
+                "unit": "Tops/s", "frac": ops / (ms / 1e3) / 1e12 / roof_peak, "traffic": None,
+                "peak_source": roof_src}
+    print(json.dumps({
+        "metric": metric, "value": value, "unit": unit, "n_gpus": 1, "steps": args.steps,
+        "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": cfg, "roofline": roof, "gpu_launches": per_launch * args.steps,
+        "clocks": clocks, "e2e": None, "cpu_baseline": None}))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -445,7 +549,12 @@ def main():
                     help="use the library's default schedule thresholds")
     ap.add_argument("--no-graph", action="store_true",
                     help="launch each solve's kernels eagerly instead of replaying a CUDA graph")
+    ap.add_argument("--workload", default="solve", choices=["solve", "gram", "symgrid"],
+                    help="solve (the headline line), or a line for the Gram accumulation or "
+                         "the symmetric grid")
     args = ap.parse_args()
+    if args.workload != "solve" and args.impl == "ours":
+        return run_extra(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_gpu(args)

@@ -136,18 +136,18 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw,
  *     s_k = fl(amax * fl((2K - k) / (2K l)))   (K = 0: s_0 = fl(amax * fl(1/l)))
  *   error_k = sum over the row/group of (s_k clamp(rint(w / s_k), -l, l) - w)^2
  * and the least error_k wins (the first, i.e. the larger scale, on ties).  An
- * all-zero row/group uses amax = 1.  The paper fixes l = 3 and a shrink of
- * "up to a factor of 2"; the number of steps is the caller's (K = 50 gives
- * factors 1.00, 0.99, ..., 0.50).
+ * all-zero row/group uses amax = 1.  The paper's runs use l = 3 and shrink
+ * the scale by at most 2x; it leaves the search's resolution open, so the
+ * number of steps is the caller's (K = 50 gives factors 1.00, 0.99, ..., 0.50).
  *   W        device, as bakron_solve (read only)
  *   levels   l, 1..127 (2l + 1 codes)
  *   shrink_steps K, 0..1024
  *   scales, zeros  device, m x G fp32, written: the chosen s and z = l, so
  *            that the affine form of bakron_solve holds: code c in 0..2l has
  *            value s (c - l)
- * The errors are summed in fp32 (per-thread partial sums, then a fixed
- * tree); rows whose two best candidates lie within that rounding may pick
- * either.  Asynchronous on `stream`; returns BAKRON_ERR_INVALID_ARG before
+ * The quotient w / s_k is formed as w * fl(1 / s_k) and the errors are summed
+ * in fp32 (per-thread partial sums, then a fixed tree); rows whose two best
+ * candidates lie within that rounding may pick either.  Asynchronous on `stream`; returns BAKRON_ERR_INVALID_ARG before
  * any launch for bad arguments.  Pass the result to bakron_solve_with_grid
  * with qmax = 2 l.
  */
@@ -172,6 +172,50 @@ int bakron_solve_with_grid(const void* W, int wdtype, int m, int n, int64_t ldw,
                            const float* scales, const float* zeros,
                            uint8_t* codes, float* prerounding, void* workspace,
                            size_t workspace_bytes, int sync, void* stream);
+
+/*
+ * Kronecker factors of the Hessian (Sec. 4, "Choosing the Factorization";
+ * appendix on the Hessian factorisation).  For H = E[a a^T (x) b b^T]:
+ *   K-FAC:    A = E[a a^T], B = E[b b^T]
+ *   Shampoo (one power-iteration step from identity):
+ *             A = E[|b|^2 a a^T], B = E[|a|^2 b b^T]
+ * Both are weighted Grams, accumulated by
+ *
+ * bakron_gram -- G <- beta G + alpha X^T diag(w) X.
+ *   X        device, k samples (rows) of d values, row stride ldx elements
+ *            (>= d), dtype BAKRON_F32 or BAKRON_BF16: the activations' tokens
+ *            x features layout; a matrix sample (d x r) enters as r rows
+ *   w        device, k fp32 weights, or NULL for all ones
+ *   alpha, beta  scalars (K-FAC over k samples: alpha = 1/k; beta = 1 adds
+ *            to a running sum; beta = 0 never reads G)
+ *   G        device, d x d fp32, row stride ldg (>= d): every entry written,
+ *            (i, j) and (j, i) to the same value
+ *   workspace device scratch of at least bakron_gram_workspace_bytes(d, 1,
+ *            w != NULL) bytes; the samples are processed in chunks of as many
+ *            as fit (bakron_gram_workspace_bytes(d, c, weighted) holds c), so
+ *            a larger workspace means fewer, larger launches
+ *   sync     nonzero: synchronise `stream` and return the device status
+ * On the tensor cores (tcgen05, kind::tf32), FP32-accurate: operands split
+ * x = hi + lo in tf32 and A B^T ~ hi hi^T + hi lo^T + lo hi^T; bf16 samples
+ * are exact in tf32 (their lo is 0, so those MMAs are skipped).  Each 32
+ * samples are accumulated afresh and added in fp32.  Only the lower-triangle
+ * 128 x 128 blocks are computed.  Returns BAKRON_ERR_INVALID_ARG (bad
+ * pointer, k < 1, d outside 1..65536, strides), BAKRON_ERR_WORKSPACE, or the
+ * device status (BAKRON_ERR_TIMEOUT if a bounded wait ran out).
+ */
+size_t bakron_gram_workspace_bytes(int d, int k_chunk, int weighted);
+int bakron_gram(const void* X, int xdtype, int k, int d, int64_t ldx,
+                const float* w, float alpha, float beta, float* G, int64_t ldg,
+                void* workspace, size_t workspace_bytes, int sync, void* stream);
+
+/*
+ * bakron_sample_sqnorms -- out[t] = |y_t|^2 = sum_j Y[t, j]^2 for the k rows
+ * of Y (device, row stride ldy >= d, fp32 or bf16), in fp32: the one-step
+ * Shampoo weight tr(b_t^T b_t) of sample t.  out: device, k fp32.
+ * Asynchronous; BAKRON_ERR_INVALID_ARG before any launch for bad arguments.
+ */
+int bakron_sample_sqnorms(const void* Y, int ydtype, int k, int d, int64_t ldy,
+                          float* out, void* stream);
 
 /*
  * bakron_autotune -- choose, for this problem shape, which kernels run each

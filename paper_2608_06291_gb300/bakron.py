@@ -57,6 +57,12 @@ def lib() -> ctypes.CDLL:
     L.bakron_solve_with_grid.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp,
                                          vp, sz, i32, vp]
     L.bakron_solve_with_grid.restype = i32
+    L.bakron_gram_workspace_bytes.argtypes = [i32, i32, i32]
+    L.bakron_gram_workspace_bytes.restype = sz
+    L.bakron_gram.argtypes = [vp, i32, i32, i32, i64, vp, f32, f32, vp, i64, vp, sz, i32, vp]
+    L.bakron_gram.restype = i32
+    L.bakron_sample_sqnorms.argtypes = [vp, i32, i32, i32, i64, vp, vp]
+    L.bakron_sample_sqnorms.restype = i32
     L.bakron_solve_noalloc.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, i32, vp]
     L.bakron_solve_noalloc.restype = i32
     L.bakron_read_status.argtypes = [vp, vp]
@@ -245,6 +251,72 @@ def bakron_solve_with_grid(W, f: Factors, scales, zeros, qmax: int, group_size: 
                                       _stream(stream))
     _check(rc, "bakron_solve_with_grid")
     return (codes, xpre) if prerounding else codes
+
+
+def _rows_dtype(X, name):
+    if not X.is_cuda or X.dim() != 2 or X.stride(1) != 1:
+        raise ValueError(f"{name} must be a 2-D CUDA tensor with unit column stride")
+    if X.dtype == torch.float32:
+        return F32
+    if X.dtype == torch.bfloat16:
+        return BF16
+    raise ValueError(f"{name} must be float32 or bfloat16")
+
+
+def bakron_gram_workspace_bytes(d: int, k_chunk: int, weighted: bool = False) -> int:
+    return int(lib().bakron_gram_workspace_bytes(int(d), int(k_chunk), 1 if weighted else 0))
+
+
+def bakron_gram(X, w=None, alpha: float = 1.0, beta: float = 0.0, G=None, workspace=None,
+                chunk: int = 8192, sync: bool = True, stream=None):
+    """G <- beta G + alpha X^T diag(w) X for X (k samples x d, CUDA fp32/bf16).
+    Returns G (d x d fp32); a new G (beta ignored) when G is None."""
+    dt = _rows_dtype(X, "X")
+    k, d = X.shape
+    if w is not None and (not w.is_cuda or w.dtype != torch.float32 or w.numel() != k
+                          or not w.is_contiguous()):
+        raise ValueError("w must be a contiguous CUDA float32 vector of length k")
+    if G is None:
+        G = torch.empty(d, d, dtype=torch.float32, device=X.device)
+        beta = 0.0
+    elif (not G.is_cuda or G.dtype != torch.float32 or tuple(G.shape) != (d, d)
+          or G.stride(1) != 1):
+        raise ValueError("G must be a CUDA float32 d x d tensor with unit column stride")
+    if workspace is None:
+        nb = bakron_gram_workspace_bytes(d, min(k, chunk), w is not None)
+        workspace = torch.empty(nb, dtype=torch.uint8, device=X.device)
+    rc = lib().bakron_gram(_ptr(X), dt, k, d, X.stride(0), _ptr(w), float(alpha), float(beta),
+                           _ptr(G), G.stride(0), _ptr(workspace), workspace.numel(),
+                           1 if sync else 0, _stream(stream))
+    _check(rc, "bakron_gram")
+    return G
+
+
+def bakron_sample_sqnorms(Y, stream=None):
+    """|y_t|^2 per row of Y (k x d, CUDA fp32/bf16) -> k fp32."""
+    dt = _rows_dtype(Y, "Y")
+    k, d = Y.shape
+    out = torch.empty(k, dtype=torch.float32, device=Y.device)
+    rc = lib().bakron_sample_sqnorms(_ptr(Y), dt, k, d, Y.stride(0), _ptr(out), _stream(stream))
+    _check(rc, "bakron_sample_sqnorms")
+    return out
+
+
+def kfac_factors(a, b, stream=None):
+    """K-FAC: (E[a a^T], E[b b^T]) from paired samples a (k x n), b (k x m)."""
+    k = a.shape[0]
+    return (bakron_gram(a, alpha=1.0 / k, stream=stream),
+            bakron_gram(b, alpha=1.0 / k, stream=stream))
+
+
+def shampoo_factors(a, b, stream=None):
+    """One Shampoo power-iteration step from identity:
+    (E[|b|^2 a a^T], E[|a|^2 b b^T])."""
+    k = a.shape[0]
+    wa = bakron_sample_sqnorms(b, stream)
+    wb = bakron_sample_sqnorms(a, stream)
+    return (bakron_gram(a, wa, alpha=1.0 / k, stream=stream),
+            bakron_gram(b, wb, alpha=1.0 / k, stream=stream))
 
 
 def bakron_autotune(W, f: Factors, bits: int, group_size: int = 0, workspace=None,

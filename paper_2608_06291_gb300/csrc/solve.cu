@@ -68,7 +68,9 @@ __global__ void k_grid(const void* W, int wdt, int m, int n, int64_t ldw, int gs
 //     s_k = fl(amax * fl((2K - k) / (2K l))),  k = 0..K   (K = 0: fl(1 / l))
 // the one with the least round-to-nearest squared error
 //     sum_q (s_k clamp(rint(w_q / s_k), -l, l) - w_q)^2
-// wins, the first on ties.  An all-zero row/group uses amax = 1.  Stored in
+// wins, the first on ties.  w_q / s_k is formed as w_q * fl(1 / s_k): it can
+// only move a value lying within rounding of a midpoint between two levels
+// to the other level, where both have the same squared error.  An all-zero row/group uses amax = 1.  Stored in
 // the affine form the solve reads: z = l, codes 0..2l.  One block of
 // GRID_SYM_THREADS per (row, group); the row is re-read from L1 per
 // candidate; sums are fp32 per thread, then a fixed tree.
@@ -110,11 +112,11 @@ __global__ void __launch_bounds__(GRID_SYM_THREADS)
     for (int k = 0; k <= K; ++k) {
       const float t = K == 0 ? __fdiv_rn(1.f, L)
                              : __fdiv_rn((float)(2 * K - k), (float)(2 * K * levels));
-      const float s = __fmul_rn(amax, t);
+      const float s = __fmul_rn(amax, t), rs = __fdiv_rn(1.f, s);
       float err = 0.f;
       for (int c = threadIdx.x; c < gsz; c += GRID_SYM_THREADS) {
         const float v = load(c);
-        const float q = fminf(fmaxf(rintf(__fdiv_rn(v, s)), -L), L);
+        const float q = fminf(fmaxf(rintf(v * rs), -L), L);
         const float d = fmaf(s, q, -v);
         err = fmaf(d, d, err);
       }

@@ -36,6 +36,7 @@
 // CTA winds down, draining its own TMA copies and MMAs (with a separate,
 // generous limit) before it frees TMEM.
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
 #include <stdint.h>
@@ -63,7 +64,7 @@ constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*ba
 constexpr int NACC = 4;                         // TMEM accumulators, rotating per K stage
 constexpr uint32_t TMEM_COLS = NACC * BN;       // all 512 columns: one CTA per SM (shared memory)
 
-enum Mode { MODE_DENSE = 0, MODE_STAGE1 = 1, MODE_STAGE2 = 2 };
+enum Mode { MODE_DENSE = 0, MODE_STAGE1 = 1, MODE_STAGE2 = 2, MODE_GRAM = 3 };
 
 struct TcParams {
   int mode;
@@ -77,6 +78,12 @@ struct TcParams {
   int64_t ldo;          // leading dimension of out_hi/out_lo/X (elements)
   int* status;
   long long spin_cycles;  // bound of the working waits (clock64 cycles)
+  // Gram mode: G <- beta G + alpha A B^T on the lower-triangle blocks, each
+  // entry (i, j <= i) < dreal written and mirrored to (j, i); a_exact /
+  // b_exact: that operand's lo plane is zero (skip its correction MMA)
+  float alpha, beta;
+  int dreal;
+  int a_exact, b_exact;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -265,6 +272,18 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
   b.rb = P.row0 + (P.mode == MODE_DENSE ? blockIdx.y : gridDim.y - 1 - blockIdx.y);
   if (P.mode == MODE_DENSE) {
     b.cb = blockIdx.x;
+    b.k0 = 0;
+    b.nk = P.K / BK;
+    return true;
+  }
+  if (P.mode == MODE_GRAM) {
+    // block t of the lower triangle, row by row: t = rb (rb + 1) / 2 + cb, cb <= rb
+    const int t = blockIdx.x;
+    int rb = (int)((sqrtf(8.f * (float)t + 1.f) - 1.f) * 0.5f);
+    while ((rb + 1) * (rb + 2) / 2 <= t) ++rb;
+    while (rb * (rb + 1) / 2 > t) --rb;
+    b.rb = rb;
+    b.cb = t - rb * (rb + 1) / 2;
     b.k0 = 0;
     b.nk = P.K / BK;
     return true;
@@ -487,8 +506,8 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
         for (int kk = 0; kk < BK / 8; ++kk) {
           const uint64_t o = (uint64_t)(2 * kk);   // 8 tf32 = 32 bytes along K inside the swizzle row
           mma_tf32(d, dah + o, dbh + o, idesc, kk > 0 ? 1u : 0u);
-          mma_tf32(d, dah + o, dbl + o, idesc, 1u);
-          mma_tf32(d, dal + o, dbh + o, idesc, 1u);
+          if (!P.b_exact) mma_tf32(d, dah + o, dbl + o, idesc, 1u);
+          if (!P.a_exact) mma_tf32(d, dal + o, dbh + o, idesc, 1u);
         }
         mma_commit(&accF[a]);     // the stage's sum to the epilogue; its slot to the producer
       }
@@ -533,7 +552,26 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
       __syncwarp();
       if (lane == 0) mbar_arrive(&accE[a]);
     }
-    if (P.mode == MODE_DENSE) {
+    if (P.mode == MODE_GRAM) {
+      // entry (gi, gj <= gi) and its mirror (gj, gi); for a fixed u the warp's
+      // 32 lanes hold 32 consecutive gi, so the mirror stores are coalesced
+      const int64_t gi = (int64_t)blk.rb * BM + row;
+      const int64_t gj0 = (int64_t)blk.cb * BN + c0;
+      if (write && gi < P.dreal) {
+#pragma unroll
+        for (int u = 0; u < EPI_COLS; ++u) {
+          const int64_t gj = gj0 + u;
+          if (gj > gi) continue;          // also keeps gj < dreal
+          const float v = P.alpha * acc[u];
+          float* p = P.out_hi + gi * P.ldo + gj;
+          *p = P.beta == 0.f ? v : fmaf(P.beta, *p, v);
+          if (gj < gi) {
+            float* q2 = P.out_hi + gj * P.ldo + gi;
+            *q2 = P.beta == 0.f ? v : fmaf(P.beta, *q2, v);
+          }
+        }
+      }
+    } else if (P.mode == MODE_DENSE) {
       const int64_t gi = (int64_t)blk.rb * BM + row;
 #pragma unroll
       for (int c = 0; c < EPI_COLS / 32; ++c) {
@@ -679,6 +717,62 @@ __global__ void k_split(const float* src, int64_t count, float* hi, float* lo) {
   lo[i] = v - h;
 }
 
+// Gram operands: samples t0 .. t0 + kc of X (k x d, row stride ldx, fp32 or
+// bf16) transposed into the K-major planes T = X^T (dp x kc, zeros past k and
+// d), split as hi + lo; with weights, also WT = (diag(w) X)^T, the product
+// w_t x_ti rounded once to fp32 before the split.  32 x 32 tiles through
+// shared memory: coalesced reads along features, writes along samples.
+__global__ void k_gram_split(const void* X, int xdt, int k, int d, int64_t ldx, int t0, int kc,
+                             const float* w, float* Th, float* Tl, float* Wh, float* Wl) {
+  __shared__ float tile[32][33];
+  __shared__ float wt[32];
+  const int tx = threadIdx.x, ty = threadIdx.y;     // 32 x 8
+  const int tb = blockIdx.x * 32, ib = blockIdx.y * 32;
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const int t = t0 + tb + ty + 8 * r, i = ib + tx;
+    float v = 0.f;
+    if (t < k && i < d) {
+      const int64_t o = (int64_t)t * ldx + i;
+      v = xdt == BAKRON_BF16 ? __bfloat162float(((const __nv_bfloat16*)X)[o])
+                             : ((const float*)X)[o];
+    }
+    tile[ty + 8 * r][tx] = v;
+  }
+  if (w && ty == 0) wt[tx] = (t0 + tb + tx < k) ? w[t0 + tb + tx] : 0.f;
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const int i = ib + ty + 8 * r, tc = tb + tx;
+    const int64_t o = (int64_t)i * kc + tc;
+    const float v = tile[tx][ty + 8 * r], h = tf32_hi(v);
+    Th[o] = h;
+    Tl[o] = v - h;
+    if (w) {
+      const float u = wt[tx] * v, uh = tf32_hi(u);
+      Wh[o] = uh;
+      Wl[o] = u - uh;
+    }
+  }
+}
+
+// |y_t|^2 per row (warp per row, fp32, lane-strided partial sums then a
+// butterfly): the one-step Shampoo weight tr(b_t^T b_t) of a vector sample.
+__global__ void k_sqnorms(const void* Y, int ydt, int k, int d, int64_t ldy, float* out) {
+  const int64_t row = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= k) return;
+  float acc = 0.f;
+  for (int j = lane; j < d; j += 32) {
+    const int64_t o = row * ldy + j;
+    const float v = ydt == BAKRON_BF16 ? __bfloat162float(((const __nv_bfloat16*)Y)[o])
+                                       : ((const float*)Y)[o];
+    acc = fmaf(v, v, acc);
+  }
+  for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (lane == 0) out[row] = acc;
+}
+
 }  // namespace
 
 long long spin_cycles_from_env() {
@@ -779,4 +873,80 @@ extern "C" int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C,
   k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mBh, mBl, mBh, mBl, P);
   BK_CUDA_OK(cudaGetLastError());
   return bakron_read_status(workspace, stream);
+}
+
+// ------------------------------------------------------------ Gram matrices
+namespace {
+constexpr int GRAM_MAX_D = 1 << 16;
+}  // namespace
+
+extern "C" size_t bakron_gram_workspace_bytes(int d, int k_chunk, int weighted) {
+  if (d < 1 || d > GRAM_MAX_D || k_chunk < 1) return 0;
+  const int64_t dp = round_up(d, BM), kc = round_up(k_chunk, BK);
+  return 256 + (size_t)(weighted ? 4 : 2) * (size_t)dp * (size_t)kc * 4;
+}
+
+extern "C" int bakron_gram(const void* X, int xdtype, int k, int d, int64_t ldx, const float* w,
+                           float alpha, float beta, float* G, int64_t ldg, void* workspace,
+                           size_t workspace_bytes, int sync, void* stream) {
+  if (!X || !G || !workspace || k < 1 || d < 1 || d > GRAM_MAX_D || ldx < d || ldg < d)
+    return BAKRON_ERR_INVALID_ARG;
+  if (xdtype != BAKRON_F32 && xdtype != BAKRON_BF16) return BAKRON_ERR_INVALID_ARG;
+  const int64_t dp = round_up(d, BM);
+  const int planes = w ? 4 : 2;
+  if (workspace_bytes < 256) return BAKRON_ERR_WORKSPACE;
+  int64_t kc = (int64_t)((workspace_bytes - 256) / ((size_t)planes * dp * 4)) / BK * BK;
+  kc = std::min<int64_t>(kc, round_up(k, BK));
+  kc = std::min<int64_t>(kc, (int64_t)1 << 30);
+  if (kc < BK) return BAKRON_ERR_WORKSPACE;
+  if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
+  cudaStream_t s = (cudaStream_t)stream;
+  char* ws = (char*)workspace;
+  int* status = (int*)ws;
+  float* Th = (float*)(ws + 256);
+  float* Tl = Th + dp * kc;
+  float* Wh = w ? Tl + dp * kc : nullptr;
+  float* Wl = w ? Wh + dp * kc : nullptr;
+  BK_CUDA_OK(cudaMemsetAsync(status, 0, 256, s));
+  const int nb = (int)(dp / BM);
+  const unsigned ntri = (unsigned)((int64_t)nb * (nb + 1) / 2);
+  const long long spin = spin_cycles_from_env();
+  for (int64_t t0 = 0; t0 < k; t0 += kc) {
+    const int64_t kcl = std::min<int64_t>(kc, round_up(k - t0, BK));   // this chunk's K
+    dim3 sg((unsigned)(kcl / 32), (unsigned)(dp / 32));
+    k_gram_split<<<sg, dim3(32, 8), 0, s>>>(X, xdtype, k, d, ldx, (int)t0, (int)kc, w, Th, Tl, Wh,
+                                            Wl);
+    BK_CUDA_OK(cudaGetLastError());
+    CUtensorMap mA2, mB2;
+    const float* ah = w ? Wh : Th;
+    const float* al = w ? Wl : Tl;
+    if (!make_map_pair(&mA2, ah, al, dp, kcl, kc, BM) || !make_map_pair(&mB2, Th, Tl, dp, kcl, kc, BN))
+      return BAKRON_ERR_CUDA;
+    TcParams P{};
+    P.mode = MODE_GRAM;
+    P.K = (int)kcl;
+    P.out_hi = G;
+    P.ldo = ldg;
+    P.status = status;
+    P.spin_cycles = spin;
+    P.alpha = alpha;
+    P.beta = t0 == 0 ? beta : 1.f;
+    P.dreal = d;
+    P.b_exact = xdtype == BAKRON_BF16;              // bf16 is exact in tf32: lo plane zero
+    P.a_exact = xdtype == BAKRON_BF16 && !w;
+    k_tc_band<<<ntri, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mB2, mB2, mB2, mB2, P);
+    BK_CUDA_OK(cudaGetLastError());
+  }
+  if (!sync) return BAKRON_OK;
+  return bakron_read_status(workspace, stream);
+}
+
+extern "C" int bakron_sample_sqnorms(const void* Y, int ydtype, int k, int d, int64_t ldy,
+                                     float* out, void* stream) {
+  if (!Y || !out || k < 1 || d < 1 || ldy < d) return BAKRON_ERR_INVALID_ARG;
+  if (ydtype != BAKRON_F32 && ydtype != BAKRON_BF16) return BAKRON_ERR_INVALID_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  k_sqnorms<<<(unsigned)(((int64_t)k * 32 + 255) / 256), 256, 0, s>>>(Y, ydtype, k, d, ldy, out);
+  BK_CUDA_OK(cudaGetLastError());
+  return BAKRON_OK;
 }

@@ -78,4 +78,24 @@ def test_invalid_arguments_rejected_on_host(L):
     assert sg(fake, 0, 4, 4, 4, fake, 6, 0, None, fake, fake, None, fake, 1 << 30, 0, None) == 1
     assert sg(fake, 0, 4, 6, 6, fake, 6, 4, fake, fake, fake, None, fake, 1 << 30, 0, None) == 1
     assert sg(fake, 0, 4, 4, 4, fake, 6, 0, fake, fake, fake, None, fake, 16, 0, None) == 5
+    # Gram accumulation: k, d, strides, dtype, workspace
+    gr = L.bakron_gram
+    f1, f0 = ctypes.c_float(1.0), ctypes.c_float(0.0)
+    assert gr(None, 0, 8, 4, 4, None, f1, f0, fake, 4, fake, 1 << 30, 0, None) == 1
+    assert gr(fake, 0, 0, 4, 4, None, f1, f0, fake, 4, fake, 1 << 30, 0, None) == 1
+    assert gr(fake, 0, 8, 4, 3, None, f1, f0, fake, 4, fake, 1 << 30, 0, None) == 1
+    assert gr(fake, 0, 8, 4, 4, None, f1, f0, fake, 3, fake, 1 << 30, 0, None) == 1
+    assert gr(fake, 0, 8, (1 << 16) + 1, 1 << 17, None, f1, f0, fake, 1 << 17, fake, 1 << 40,
+              0, None) == 1
+    assert gr(fake, 3, 8, 4, 4, None, f1, f0, fake, 4, fake, 1 << 30, 0, None) == 1
+    need = L.bakron_gram_workspace_bytes(4, 1, 0)
+    assert need == 256 + 2 * 128 * 32 * 4
+    assert L.bakron_gram_workspace_bytes(4, 33, 1) == 256 + 4 * 128 * 64 * 4
+    assert L.bakron_gram_workspace_bytes(0, 1, 0) == 0
+    assert gr(fake, 0, 8, 4, 4, None, f1, f0, fake, 4, fake, need - 1, 0, None) == 5
+    assert gr(fake, 0, 8, 4, 4, fake, f1, f0, fake, 4, fake, need, 0, None) == 5   # weighted: 4 planes
+    sq = L.bakron_sample_sqnorms
+    assert sq(None, 0, 4, 4, 4, fake, None) == 1
+    assert sq(fake, 0, 4, 4, 3, fake, None) == 1
+    assert sq(fake, 0, 0, 4, 4, fake, None) == 1
     assert P.strerror(2) == "damped Gram is not positive definite"
