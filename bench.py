@@ -430,12 +430,16 @@ def run_gpu(args):
 
 
 def run_extra(args):
-    """One JSON line for a workload next to the solve (no graph, N = 1 only):
+    """One JSON line for a workload next to the solve (N = 1 only):
       gram     K-FAC input-side factor A = X^T X / k of the 4096-feature layer
                from k = 65536 bf16 activation rows (32 sequences of 2048
                tokens), one bakron_gram call per step;
       symgrid  the symmetric l = 3 grid with 50 shrink steps of the 4096 x 4096
-               weights (one bakron_grid_symmetric call per step)."""
+               weights (one bakron_grid_symmetric call per step);
+      batched  the 4096 x 4096 weights as 32 heads of 128 rows, each with its
+               own 128 x 128 output-side Gram and the layer's input-side one,
+               one bakron_solve_batched call over 16 lanes per step (CUDA graph
+               replay; the same call on one lane is timed for context)."""
     import torch
 
     import paper_2608_06291_gb300 as P
@@ -472,6 +476,70 @@ def run_extra(args):
         roof_src = "of measured: bf16_tflops x 1.1/2.25 (tf32/bf16 nominal)"
         cfg = {"workload": "kfac_gram", "k": k, "d": d, "dtype_in": "bf16",
                "l2": "flushed (256 MiB write) between steps; X 512 MiB > L2"}
+    elif args.workload == "batched":
+        cfg2 = WL.CONFIGS[2]
+        W, A, _ = WL.make(cfg2, device=dev)
+        Hh, mh, n = 32, 128, cfg2.n
+        lanes = 16
+        Ws = [W[h * mh:(h + 1) * mh] for h in range(Hh)]
+        # the shared input-side factor once; each head's output-side factor
+        # from a small prepare of its own Gram; assembled per head
+        Bs = [WL.power_law_gram(mh, cfg2.n_samples, cfg2.alpha_b, 9000 + h, 9100 + h, dev)
+              for h in range(Hh)]
+        LA, _, rA, _ = P.bakron_get_factors(P.bakron_prepare(A, Bs[0], cfg2.damp))
+        fs = []
+        for h in range(Hh):
+            LBh, _, rBh, _ = P.bakron_get_factors(P.bakron_prepare(Bs[h], Bs[h], cfg2.damp))
+            fs.append(P.bakron_set_factors(LA, LBh, rA, rBh))
+        outs = [(torch.empty(mh, n, dtype=torch.uint8, device=dev),
+                 torch.empty(mh, 1, dtype=torch.float32, device=dev),
+                 torch.empty(mh, 1, dtype=torch.float32, device=dev)) for _ in range(Hh)]
+
+        def graph_of(S):
+            wsb = torch.empty(P.bakron_batched_workspace_bytes(mh, n, S), dtype=torch.uint8,
+                              device=dev)
+            P.bakron_solve_batched(Ws, fs, cfg2.bits, 0, streams=S, workspace=wsb, out=outs)
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr):
+                P.bakron_solve_batched(Ws, fs, cfg2.bits, 0, streams=S, workspace=wsb,
+                                       sync=False, out=outs)
+            return gr, wsb
+        g1, _ = graph_of(1)
+        launches_per = P.bakron_last_launches()
+        gS, wsS = graph_of(lanes)
+
+        def one_lane():
+            g1.replay()
+
+        def step():
+            gS.replay()
+        for _ in range(3):
+            one_lane()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(3):
+            one_lane()
+        e1.record(stream)
+        e1.synchronize()
+        one_lane_ms = e0.elapsed_time(e1) / 3
+        units = Hh * mh * n
+        mma = None
+        unit = "entries/s"
+        metric = ("per-head BaKron solves: 32 heads of 128x4096 (bf16, 4-bit), "
+                  "16 lanes, entries/s")
+        per_launch = launches_per
+        f_alg = Hh * float(mh) * n * (mh + n)
+        bf16_sus = float(peaks.get("bf16_tflops_sustained", 1700.0))
+        p_eff = bf16_sus * (1.1 / 2.25) / 3.0
+        hbm = float(peaks.get("hbm_gbs", 6800.0))
+        roof_peak = p_eff
+        roof_src = "of measured: bf16_tflops_sustained x 1.1/2.25 (tf32/bf16) / 3"
+        cfg = {"workload": "batched_heads", "heads": Hh, "m_head": mh, "n": n, "bits": 4,
+               "lanes": lanes, "launch": "cuda graph replay",
+               "one_lane_ms": one_lane_ms, "A": "shared (4096x4096 layer's)",
+               "B": "one 128x128 power-law Gram per head",
+               "l2": "flushed (256 MiB write) between steps"}
     else:
         cfg2 = WL.CONFIGS[2]
         W, _, _ = WL.make(cfg2, device=dev)
@@ -513,7 +581,16 @@ def run_extra(args):
     clocks = sampler.stop(w0, w1)
     ms = sum(a.elapsed_time(b) for a, b in zip(starts, ends)) / args.steps
     value = units / (ms / 1e3)
-    if args.workload == "gram":
+    if args.workload == "batched":
+        if P.lib().bakron_read_status_batched(wsS.data_ptr(), mh, n, lanes, None) != 0:
+            raise RuntimeError("device status set during the timed steps")
+        t_roof = f_alg / (p_eff * 1e12) + 17.0 * units / (hbm * 1e9)
+        roof = {"bound": "tensor", "achieved": f_alg / (ms / 1e3) / 1e12, "peak": p_eff,
+                "unit": "TFLOP/s", "frac": 1e3 * t_roof / ms, "traffic": None,
+                "peak_source": roof_src, "roofline_ms": 1e3 * t_roof,
+                "note": "whole-call roofline: sum over heads of F_alg at the FP32-effective "
+                        "tensor rate plus 17 B/entry at HBM rate"}
+    elif args.workload == "gram":
         roof = {"bound": "tensor", "achieved": value / 1e12, "peak": roof_peak,
                 "unit": "TFLOP/s", "frac": value / 1e12 / roof_peak, "traffic": None,
                 "peak_source": roof_src,
@@ -549,9 +626,10 @@ def main():
                     help="use the library's default schedule thresholds")
     ap.add_argument("--no-graph", action="store_true",
                     help="launch each solve's kernels eagerly instead of replaying a CUDA graph")
-    ap.add_argument("--workload", default="solve", choices=["solve", "gram", "symgrid"],
-                    help="solve (the headline line), or a line for the Gram accumulation or "
-                         "the symmetric grid")
+    ap.add_argument("--workload", default="solve",
+                    choices=["solve", "gram", "symgrid", "batched"],
+                    help="solve (the headline line), or a line for the Gram accumulation, "
+                         "the symmetric grid or the batched per-head solve")
     args = ap.parse_args()
     if args.workload != "solve" and args.impl == "ours":
         return run_extra(args)

@@ -218,6 +218,44 @@ int bakron_sample_sqnorms(const void* Y, int ydtype, int k, int d, int64_t ldy,
                           float* out, void* stream);
 
 /*
+ * bakron_solve_batched -- H independent solves of one shape m x n in one
+ * call: the per-head problems of attention layers whose output-side factor
+ * is block diagonal (one B per head, a shared input-side A; the local
+ * attention Hessians of Sec. 4 and the BoA setting).  Problem h rounds W[h]
+ * under factors[h] exactly as bakron_solve would (same kernels, same
+ * schedule table, same codes bit for bit).
+ *   W, factors, codes, scales, zeros  HOST arrays of H device pointers (the
+ *            buffers of problem h; factors[h] may repeat); the device
+ *            buffers are those of bakron_solve for one m x n problem
+ *   streams  S, 1..32: problems run side by side on S library-owned CUDA
+ *            streams, problem h on lane h mod S, each lane in order; the
+ *            lanes fork from `stream` and join back into it through events,
+ *            so later work on `stream` sees every result
+ *   workspace device, >= bakron_batched_workspace_bytes(m, n, min(S, H))
+ *            bytes: lane l uses slice l (bakron_workspace_bytes(m, n) rounded
+ *            up to 256 bytes, at offset l times that)
+ *   sync     nonzero: synchronise and return the first nonzero device status
+ *            of any lane; zero: asynchronous (bakron_read_status_batched)
+ * The first call on a device creates its lane streams and events (kept until
+ * the process exits): make it outside any stream capture; later calls with
+ * sync = 0 can be captured into a CUDA graph.  Calls from several host
+ * threads are serialised while they enqueue.  Arguments are validated on
+ * the host as in bakron_solve (BAKRON_ERR_INVALID_ARG, BAKRON_ERR_WORKSPACE)
+ * before anything is enqueued.
+ */
+size_t bakron_batched_workspace_bytes(int m, int n, int streams);
+int bakron_solve_batched(int H, const void* const* W, int wdtype, int m, int n,
+                         int64_t ldw, const void* const* factors, int bits,
+                         int group_size, uint8_t* const* codes,
+                         float* const* scales, float* const* zeros,
+                         void* workspace, size_t workspace_bytes, int streams,
+                         int sync, void* stream);
+/* Synchronise `stream`; return and clear the status words of the first
+ * `streams` lane slices of a batched workspace (the first nonzero one). */
+int bakron_read_status_batched(void* workspace, int m, int n, int streams,
+                               void* stream);
+
+/*
  * bakron_autotune -- choose, for this problem shape, which kernels run each
  * node of the recursion, by timing candidate schedules on the caller's data.
  * No counterpart in the paper: Alg. 5 fixes the recursion (halving of the

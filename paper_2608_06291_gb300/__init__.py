@@ -9,7 +9,8 @@ from .bakron import (BakronError, Factors, alloc_workspace, bakron_diag_gemm_tf3
                      bakron_autotune, bakron_autotune_clear, bakron_get_factors,
                      bakron_get_tuning, bakron_grid_symmetric, bakron_solve_with_grid,
                      bakron_gram, bakron_gram_workspace_bytes, bakron_sample_sqnorms,
-                     kfac_factors, shampoo_factors,
+                     kfac_factors, shampoo_factors, bakron_solve_batched,
+                     bakron_batched_workspace_bytes,
                      bakron_last_launches, bakron_prepare, bakron_profile_enable,
                      bakron_profile_read, bakron_read_status, bakron_set_factors, bakron_solve,
                      bakron_solve_noalloc,

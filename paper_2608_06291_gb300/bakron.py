@@ -63,6 +63,14 @@ def lib() -> ctypes.CDLL:
     L.bakron_gram.restype = i32
     L.bakron_sample_sqnorms.argtypes = [vp, i32, i32, i32, i64, vp, vp]
     L.bakron_sample_sqnorms.restype = i32
+    L.bakron_batched_workspace_bytes.argtypes = [i32, i32, i32]
+    L.bakron_batched_workspace_bytes.restype = sz
+    pp = ctypes.POINTER(vp)
+    L.bakron_solve_batched.argtypes = [i32, pp, i32, i32, i32, i64, pp, i32, i32, pp, pp, pp,
+                                       vp, sz, i32, i32, vp]
+    L.bakron_solve_batched.restype = i32
+    L.bakron_read_status_batched.argtypes = [vp, i32, i32, i32, vp]
+    L.bakron_read_status_batched.restype = i32
     L.bakron_solve_noalloc.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, i32, vp]
     L.bakron_solve_noalloc.restype = i32
     L.bakron_read_status.argtypes = [vp, vp]
@@ -317,6 +325,51 @@ def shampoo_factors(a, b, stream=None):
     wb = bakron_sample_sqnorms(a, stream)
     return (bakron_gram(a, wa, alpha=1.0 / k, stream=stream),
             bakron_gram(b, wb, alpha=1.0 / k, stream=stream))
+
+
+def bakron_batched_workspace_bytes(m: int, n: int, streams: int) -> int:
+    return int(lib().bakron_batched_workspace_bytes(int(m), int(n), int(streams)))
+
+
+def _ptr_array(ts):
+    arr = (ctypes.c_void_p * len(ts))()
+    for i, t in enumerate(ts):
+        arr[i] = t.data_ptr()
+    return arr
+
+
+def bakron_solve_batched(Ws, fs, bits: int, group_size: int = 0, streams: int = 8,
+                         workspace=None, sync: bool = True, out=None, stream=None):
+    """Solve the H problems (Ws[h], fs[h]) of one shape side by side on
+    `streams` lanes.  Returns [(codes, scales, zeros)] per problem."""
+    H = len(Ws)
+    if H < 1 or len(fs) != H:
+        raise ValueError("need as many factor buffers as weight matrices (>= 1)")
+    m, n = Ws[0].shape
+    dt = _w_dtype(Ws[0])
+    ldw = Ws[0].stride(0)
+    for W, f in zip(Ws, fs):
+        if _w_dtype(W) != dt or tuple(W.shape) != (m, n) or W.stride(0) != ldw:
+            raise ValueError("every W must have the same shape, dtype and row stride")
+        if (f.m, f.n) != (m, n):
+            raise ValueError("factor buffer was built for a different shape")
+    G = 1 if group_size == 0 else n // group_size
+    dev = Ws[0].device
+    if out is None:
+        out = [(torch.empty(m, n, dtype=torch.uint8, device=dev),
+                torch.empty(m, G, dtype=torch.float32, device=dev),
+                torch.empty(m, G, dtype=torch.float32, device=dev)) for _ in range(H)]
+    S = min(int(streams), H)
+    if workspace is None:
+        workspace = torch.empty(bakron_batched_workspace_bytes(m, n, S), dtype=torch.uint8,
+                                device=dev)
+    rc = lib().bakron_solve_batched(
+        H, _ptr_array(Ws), dt, m, n, ldw, _ptr_array([f.buf for f in fs]), int(bits),
+        int(group_size), _ptr_array([o[0] for o in out]), _ptr_array([o[1] for o in out]),
+        _ptr_array([o[2] for o in out]), _ptr(workspace), workspace.numel(), S,
+        1 if sync else 0, _stream(stream))
+    _check(rc, "bakron_solve_batched")
+    return out
 
 
 def bakron_autotune(W, f: Factors, bits: int, group_size: int = 0, workspace=None,

@@ -69,6 +69,8 @@ LaunchScope::~LaunchScope() {
 }
 
 void reset_launch_count() { t_launch_count = 0; }
+int launch_count() { return t_launch_count; }
+void set_launch_count(int n) { t_launch_count = n; }
 
 bool profiling_on() { return g_on; }
 

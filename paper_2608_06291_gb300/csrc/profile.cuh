@@ -35,6 +35,8 @@ class LaunchScope {
 };
 
 void reset_launch_count();
+int launch_count();            // kernels enqueued on this host thread since the reset
+void set_launch_count(int n);
 bool profiling_on();
 
 }  // namespace bakron

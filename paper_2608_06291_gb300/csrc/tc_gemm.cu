@@ -84,6 +84,10 @@ struct TcParams {
   float alpha, beta;
   int dreal;
   int a_exact, b_exact;
+  // Gram mode with bf16 operands: mapA2 / mapB2 are plain bf16 maps (64 x
+  // 128 boxes); a ring slot holds one box of each, K = 64 per slot, and the
+  // MMAs are kind::f16 (bf16 x bf16 products exact in fp32)
+  int bf16_ops;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -207,6 +211,24 @@ __device__ __forceinline__ void mma_tf32(uint32_t tmem_d, uint64_t adesc, uint64
       : "memory");
 }
 
+// Instruction descriptor: kind::f16 with bf16 A and B (K-major), D fp32, M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return (1u << 4)            // D format fp32
+         | (1u << 7)          // A format bf16
+         | (1u << 10)         // B format bf16
+         | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
@@ -285,7 +307,7 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
     b.rb = rb;
     b.cb = t - rb * (rb + 1) / 2;
     b.k0 = 0;
-    b.nk = P.K / BK;
+    b.nk = P.K / (P.bf16_ops ? 2 * BK : BK);   // 128-byte rows: 32 fp32 or 64 bf16
     return true;
   }
   int cb_lo, cb_hi;
@@ -373,10 +395,16 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   // wait for the previous kernel, whose output (E^T or M) is the other one.
   const int npre = blk.nk < STAGES ? blk.nk : STAGES;
   const bool a_static = P.mode != MODE_STAGE2;
+  const bool bf16_ops = P.mode == MODE_GRAM && P.bf16_ops;
   if (warp == 0 && lane == 0) {
     for (int i = 0; i < npre; ++i) {
       unsigned char* st = smem + i * STAGE_BYTES;
       const int kt = blk.k0 + i;
+      if (bf16_ops) {
+        mbar_expect_tx_only(&full[i], TILE_BYTES);
+        tma_load_2d(st, &mapA2, &full[i], kt * 2 * BK, blk.rb * BM);
+        continue;
+      }
       mbar_expect_tx_only(&full[i], 2 * TILE_BYTES);
       if (a_static)
         tma_load_pair(st, &mapA2, &full[i], kt * BK, blk.rb * BM);
@@ -417,6 +445,16 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
       unsigned char *a_hi = st, *b_hi = st + 2 * TILE_BYTES, *b_lo = st + 3 * TILE_BYTES;
       const int kt = blk.k0 + i;            // K tile index (32 wide)
       const bool pre = i < npre;            // the factor operand is already on its way
+      if (bf16_ops) {                       // one bf16 box per operand, 64 of K
+        if (lane == 0) {
+          mbar_expect_tx(&full[s], pre ? TILE_BYTES : 2 * TILE_BYTES);
+          if (!pre) tma_load_2d(a_hi, &mapA2, &full[s], kt * 2 * BK, blk.rb * BM);
+          tma_load_2d(b_hi, &mapB2, &full[s], kt * 2 * BK, blk.cb * BN);
+        }
+        __syncwarp();
+        issued = i + 1;
+        continue;
+      }
       const bool load_a = !(pre && a_static), load_b = !(pre && !a_static);
       uint32_t bytes = load_a ? 2 * TILE_BYTES : 0u;   // A hi + A lo
       unsigned valid = 0xF;                 // stage 1: B sub-tiles in the band
@@ -479,7 +517,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
     // accumulation is not round-to-nearest, and its error grows with the
     // number of MMAs summed in place; restarting every 32 of K bounds it.
     if (lane == 0) {
-      const uint32_t idesc = idesc_tf32(BM, BN);
+      const uint32_t idesc = idesc_tf32(BM, BN), idesc_b = idesc_bf16(BM, BN);
       const uint64_t desc0 = smem_desc(smem_u32(smem));   // stage 0, A hi, K step 0
       for (int i = 0; i < nk; ++i) {
         const int s = i % STAGES;
@@ -502,12 +540,18 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
         const uint64_t dal = dah + (TILE_BYTES >> 4), dbh = dah + (2 * TILE_BYTES >> 4),
                        dbl = dah + (3 * TILE_BYTES >> 4);
         const uint32_t d = tmem + (uint32_t)(a * BN);
+        if (bf16_ops) {
 #pragma unroll
-        for (int kk = 0; kk < BK / 8; ++kk) {
-          const uint64_t o = (uint64_t)(2 * kk);   // 8 tf32 = 32 bytes along K inside the swizzle row
-          mma_tf32(d, dah + o, dbh + o, idesc, kk > 0 ? 1u : 0u);
-          if (!P.b_exact) mma_tf32(d, dah + o, dbl + o, idesc, 1u);
-          if (!P.a_exact) mma_tf32(d, dal + o, dbh + o, idesc, 1u);
+          for (int kk = 0; kk < 4; ++kk)            // 16 bf16 = 32 bytes along K per MMA
+            mma_bf16(d, dah + 2 * kk, dbh + 2 * kk, idesc_b, kk > 0 ? 1u : 0u);
+        } else {
+#pragma unroll
+          for (int kk = 0; kk < BK / 8; ++kk) {
+            const uint64_t o = (uint64_t)(2 * kk);   // 8 tf32 = 32 bytes along K inside the swizzle row
+            mma_tf32(d, dah + o, dbh + o, idesc, kk > 0 ? 1u : 0u);
+            if (!P.b_exact) mma_tf32(d, dah + o, dbl + o, idesc, 1u);
+            if (!P.a_exact) mma_tf32(d, dal + o, dbh + o, idesc, 1u);
+          }
         }
         mma_commit(&accF[a]);     // the stage's sum to the epilogue; its slot to the producer
       }
@@ -696,6 +740,21 @@ bool make_map_pair(CUtensorMap* map, const float* hi, const float* lo, int64_t r
   return r == CUDA_SUCCESS;
 }
 
+// 2-D bf16 row-major matrix (rows x cols, row stride ld elements), box of 64
+// columns (128 bytes, one swizzle row) by box_rows rows, 128-byte swizzle.
+bool make_map_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
+                   int box_rows) {
+  if (!get_encode() || (ld * 2) % 16) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
+  cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1u, 1u};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)base, dims, strides,
+                        box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 bool g_attr_done = false;
 std::mutex g_attr_mu;
 
@@ -753,6 +812,27 @@ __global__ void k_gram_split(const void* X, int xdt, int k, int d, int64_t ldx, 
       Wh[o] = uh;
       Wl[o] = u - uh;
     }
+  }
+}
+
+// bf16 samples t0 .. t0 + kc of X (k x d, row stride ldx) transposed into
+// the K-major bf16 plane T = X^T (dp x kc, zeros past k and d): the operand of
+// the kind::f16 Gram, exact (no split).
+__global__ void k_gram_transpose_bf16(const __nv_bfloat16* X, int k, int d, int64_t ldx, int t0,
+                                      int kc, __nv_bfloat16* T) {
+  __shared__ __nv_bfloat16 tile[32][34];
+  const int tx = threadIdx.x, ty = threadIdx.y;     // 32 x 8
+  const int tb = blockIdx.x * 32, ib = blockIdx.y * 32;
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const int t = t0 + tb + ty + 8 * r, i = ib + tx;
+    tile[ty + 8 * r][tx] = (t < k && i < d) ? X[(int64_t)t * ldx + i] : __float2bfloat16(0.f);
+  }
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const int i = ib + ty + 8 * r, tc = tb + tx;
+    T[(int64_t)i * kc + tc] = tile[tx][ty + 8 * r];
   }
 }
 
@@ -893,12 +973,16 @@ extern "C" int bakron_gram(const void* X, int xdtype, int k, int d, int64_t ldx,
     return BAKRON_ERR_INVALID_ARG;
   if (xdtype != BAKRON_F32 && xdtype != BAKRON_BF16) return BAKRON_ERR_INVALID_ARG;
   const int64_t dp = round_up(d, BM);
-  const int planes = w ? 4 : 2;
+  // bf16 samples without weights: one exact bf16 plane, kind::f16 MMAs, K = 64
+  // per ring slot; otherwise tf32 hi/lo planes (two, or four with weights)
+  const bool bf16_ops = xdtype == BAKRON_BF16 && !w;
+  const int64_t kq = bf16_ops ? 2 * BK : BK;              // chunk granularity
+  const size_t per_sample = bf16_ops ? (size_t)dp * 2 : (size_t)(w ? 4 : 2) * dp * 4;
   if (workspace_bytes < 256) return BAKRON_ERR_WORKSPACE;
-  int64_t kc = (int64_t)((workspace_bytes - 256) / ((size_t)planes * dp * 4)) / BK * BK;
-  kc = std::min<int64_t>(kc, round_up(k, BK));
+  int64_t kc = (int64_t)((workspace_bytes - 256) / per_sample) / kq * kq;
+  kc = std::min<int64_t>(kc, round_up(k, kq));
   kc = std::min<int64_t>(kc, (int64_t)1 << 30);
-  if (kc < BK) return BAKRON_ERR_WORKSPACE;
+  if (kc < kq) return BAKRON_ERR_WORKSPACE;
   if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
   cudaStream_t s = (cudaStream_t)stream;
   char* ws = (char*)workspace;
@@ -912,16 +996,26 @@ extern "C" int bakron_gram(const void* X, int xdtype, int k, int d, int64_t ldx,
   const unsigned ntri = (unsigned)((int64_t)nb * (nb + 1) / 2);
   const long long spin = spin_cycles_from_env();
   for (int64_t t0 = 0; t0 < k; t0 += kc) {
-    const int64_t kcl = std::min<int64_t>(kc, round_up(k - t0, BK));   // this chunk's K
+    const int64_t kcl = std::min<int64_t>(kc, round_up(k - t0, kq));   // this chunk's K
     dim3 sg((unsigned)(kcl / 32), (unsigned)(dp / 32));
-    k_gram_split<<<sg, dim3(32, 8), 0, s>>>(X, xdtype, k, d, ldx, (int)t0, (int)kc, w, Th, Tl, Wh,
-                                            Wl);
-    BK_CUDA_OK(cudaGetLastError());
     CUtensorMap mA2, mB2;
-    const float* ah = w ? Wh : Th;
-    const float* al = w ? Wl : Tl;
-    if (!make_map_pair(&mA2, ah, al, dp, kcl, kc, BM) || !make_map_pair(&mB2, Th, Tl, dp, kcl, kc, BN))
-      return BAKRON_ERR_CUDA;
+    if (bf16_ops) {
+      __nv_bfloat16* Tb = (__nv_bfloat16*)(ws + 256);
+      k_gram_transpose_bf16<<<sg, dim3(32, 8), 0, s>>>((const __nv_bfloat16*)X, k, d, ldx,
+                                                       (int)t0, (int)kc, Tb);
+      BK_CUDA_OK(cudaGetLastError());
+      if (!make_map_bf16(&mA2, Tb, dp, kcl, kc, BM) || !make_map_bf16(&mB2, Tb, dp, kcl, kc, BN))
+        return BAKRON_ERR_CUDA;
+    } else {
+      k_gram_split<<<sg, dim3(32, 8), 0, s>>>(X, xdtype, k, d, ldx, (int)t0, (int)kc, w, Th, Tl,
+                                              Wh, Wl);
+      BK_CUDA_OK(cudaGetLastError());
+      const float* ah = w ? Wh : Th;
+      const float* al = w ? Wl : Tl;
+      if (!make_map_pair(&mA2, ah, al, dp, kcl, kc, BM) ||
+          !make_map_pair(&mB2, Th, Tl, dp, kcl, kc, BN))
+        return BAKRON_ERR_CUDA;
+    }
     TcParams P{};
     P.mode = MODE_GRAM;
     P.K = (int)kcl;
@@ -934,6 +1028,7 @@ extern "C" int bakron_gram(const void* X, int xdtype, int k, int d, int64_t ldx,
     P.dreal = d;
     P.b_exact = xdtype == BAKRON_BF16;              // bf16 is exact in tf32: lo plane zero
     P.a_exact = xdtype == BAKRON_BF16 && !w;
+    P.bf16_ops = bf16_ops ? 1 : 0;
     k_tc_band<<<ntri, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mB2, mB2, mB2, mB2, P);
     BK_CUDA_OK(cudaGetLastError());
   }

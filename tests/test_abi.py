@@ -94,6 +94,23 @@ def test_invalid_arguments_rejected_on_host(L):
     assert L.bakron_gram_workspace_bytes(0, 1, 0) == 0
     assert gr(fake, 0, 8, 4, 4, None, f1, f0, fake, 4, fake, need - 1, 0, None) == 5
     assert gr(fake, 0, 8, 4, 4, fake, f1, f0, fake, 4, fake, need, 0, None) == 5   # weighted: 4 planes
+    # batched solve: H, lanes, null pointer arrays / entries, workspace
+    pp = ctypes.c_void_p * 2
+    arr, bad = pp(0x1000, 0x2000), pp(0x1000, None)
+    b = L.bakron_solve_batched
+    assert b(0, arr, 0, 4, 4, 4, arr, 4, 0, arr, arr, arr, fake, 1 << 30, 2, 0, None) == 1
+    assert b(2, arr, 0, 4, 4, 4, arr, 4, 0, arr, arr, arr, fake, 1 << 30, 0, 0, None) == 1
+    assert b(2, arr, 0, 4, 4, 4, arr, 4, 0, arr, arr, arr, fake, 1 << 30, 33, 0, None) == 1
+    assert b(2, None, 0, 4, 4, 4, arr, 4, 0, arr, arr, arr, fake, 1 << 30, 2, 0, None) == 1
+    assert b(2, arr, 0, 4, 4, 4, bad, 4, 0, arr, arr, arr, fake, 1 << 30, 2, 0, None) == 1
+    assert b(2, arr, 0, 4, 4, 4, arr, 9, 0, arr, arr, arr, fake, 1 << 30, 2, 0, None) == 1
+    one = L.bakron_batched_workspace_bytes(4, 4, 1)
+    assert one > 0 and one % 256 == 0          # the solve's scratch alone
+    assert L.bakron_batched_workspace_bytes(4, 4, 3) == 3 * one
+    assert L.bakron_batched_workspace_bytes(4, 4, 0) == 0
+    assert b(2, arr, 0, 4, 4, 4, arr, 4, 0, arr, arr, arr, fake, 2 * one - 1, 2, 0, None) == 5
+    # with H = 1 only one lane is needed
+    assert b(1, arr, 0, 4, 4, 4, arr, 4, 0, arr, arr, arr, fake, one - 1, 8, 0, None) == 5
     sq = L.bakron_sample_sqnorms
     assert sq(None, 0, 4, 4, 4, fake, None) == 1
     assert sq(fake, 0, 4, 4, 3, fake, None) == 1
