@@ -439,7 +439,9 @@ def run_extra(args):
       batched  the 4096 x 4096 weights as 32 heads of 128 rows, each with its
                own 128 x 128 output-side Gram and the layer's input-side one,
                one bakron_solve_batched call over 16 lanes per step (CUDA graph
-               replay; the same call on one lane is timed for context)."""
+               replay; the same call on one lane is timed for context);
+      gptq     the 4096 x 4096 solve with B = I (GPTQ, the method's special
+               case) under the layer's input-side factor, graph replay."""
     import torch
 
     import paper_2608_06291_gb300 as P
@@ -470,12 +472,44 @@ def run_extra(args):
         units = d * (d + 1) * k                   # 2k flops per unique entry
         mma = nb * (nb + 1) // 2 * 2 * 128 * 128 * k
         unit, metric = "flop/s", "K-FAC Gram X^T X / k flop/s (4096 features, 65536 bf16 rows)"
-        per_launch = 2                            # transpose-split + tensor-core Gram
-        bf16 = float(peaks.get("bf16_tflops", 1892.3))
-        roof_peak = bf16 * 1.1 / 2.25            # tf32 rate: bf16 rows are exact in tf32
-        roof_src = "of measured: bf16_tflops x 1.1/2.25 (tf32/bf16 nominal)"
+        per_launch = 2                            # bf16 transpose + tensor-core Gram
+        roof_peak = float(peaks.get("bf16_tflops", 1892.3))   # kind::f16 bf16 MMAs
+        roof_src = "of measured: bf16_tflops (burst; the Gram runs bf16 x bf16 MMAs)"
         cfg = {"workload": "kfac_gram", "k": k, "d": d, "dtype_in": "bf16",
                "l2": "flushed (256 MiB write) between steps; X 512 MiB > L2"}
+    elif args.workload == "gptq":
+        # GPTQ as the method's B = I case (Sec. 1): the 4096 x 4096 weights
+        # under the layer's input-side factor only
+        cfg2 = WL.CONFIGS[2]
+        W, A, B = WL.make(cfg2, device=dev)
+        m, n = cfg2.m, cfg2.n
+        LA, _, rA, _ = P.bakron_get_factors(P.bakron_prepare(A, B, cfg2.damp))
+        fac = P.bakron_set_factors(LA, torch.eye(m, device=dev), rA, torch.ones(m, device=dev))
+        wsb = P.alloc_workspace(m, n, dev)
+        outg = (torch.empty(m, n, dtype=torch.uint8, device=dev),
+                torch.empty(m, 1, dtype=torch.float32, device=dev),
+                torch.empty(m, 1, dtype=torch.float32, device=dev), None)
+        P.bakron_solve(W, fac, cfg2.bits, 0, workspace=wsb, out=outg)
+        launches_per = P.bakron_last_launches()
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr):
+            P.bakron_solve(W, fac, cfg2.bits, 0, workspace=wsb, sync=False, out=outg)
+
+        def step():
+            gr.replay()
+        units = m * n
+        mma = None
+        unit, metric = "entries/s", "GPTQ (BaKron with B = I), 4096x4096 bf16 W, 4-bit per row"
+        per_launch = launches_per
+        bf16_sus = float(peaks.get("bf16_tflops_sustained", 1700.0))
+        p_eff = bf16_sus * (1.1 / 2.25) / 3.0
+        hbm = float(peaks.get("hbm_gbs", 6800.0))
+        f_alg = float(m) * n * (m + n)
+        roof_peak = p_eff
+        roof_src = "of measured: bf16_tflops_sustained x 1.1/2.25 (tf32/bf16) / 3"
+        cfg = {"workload": "gptq_b_identity", "m": m, "n": n, "bits": 4,
+               "launch": "cuda graph replay", "paper_gptq_s_rtx_pro_6000": 0.025,
+               "l2": "flushed (256 MiB write) between steps"}
     elif args.workload == "batched":
         cfg2 = WL.CONFIGS[2]
         W, A, _ = WL.make(cfg2, device=dev)
@@ -581,7 +615,16 @@ def run_extra(args):
     clocks = sampler.stop(w0, w1)
     ms = sum(a.elapsed_time(b) for a, b in zip(starts, ends)) / args.steps
     value = units / (ms / 1e3)
-    if args.workload == "batched":
+    if args.workload == "gptq":
+        if P.bakron_read_status(wsb) != 0:
+            raise RuntimeError("device status set during the timed steps")
+        t_roof = f_alg / (p_eff * 1e12) + 17.0 * units / (hbm * 1e9)
+        roof = {"bound": "tensor", "achieved": f_alg / (ms / 1e3) / 1e12, "peak": p_eff,
+                "unit": "TFLOP/s", "frac": 1e3 * t_roof / ms, "traffic": None,
+                "peak_source": roof_src, "roofline_ms": 1e3 * t_roof,
+                "note": "whole-solve roofline as for the general solve (the kernels do not "
+                        "specialise L^B = I)"}
+    elif args.workload == "batched":
         if P.lib().bakron_read_status_batched(wsS.data_ptr(), mh, n, lanes, None) != 0:
             raise RuntimeError("device status set during the timed steps")
         t_roof = f_alg / (p_eff * 1e12) + 17.0 * units / (hbm * 1e9)
@@ -627,9 +670,9 @@ def main():
     ap.add_argument("--no-graph", action="store_true",
                     help="launch each solve's kernels eagerly instead of replaying a CUDA graph")
     ap.add_argument("--workload", default="solve",
-                    choices=["solve", "gram", "symgrid", "batched"],
+                    choices=["solve", "gram", "symgrid", "batched", "gptq"],
                     help="solve (the headline line), or a line for the Gram accumulation, "
-                         "the symmetric grid or the batched per-head solve")
+                         "the symmetric grid, the batched per-head solve or GPTQ (B = I)")
     args = ap.parse_args()
     if args.workload != "solve" and args.impl == "ours":
         return run_extra(args)

@@ -195,10 +195,12 @@ int bakron_solve_with_grid(const void* W, int wdtype, int m, int n, int64_t ldw,
  *            as fit (bakron_gram_workspace_bytes(d, c, weighted) holds c), so
  *            a larger workspace means fewer, larger launches
  *   sync     nonzero: synchronise `stream` and return the device status
- * On the tensor cores (tcgen05, kind::tf32), FP32-accurate: operands split
- * x = hi + lo in tf32 and A B^T ~ hi hi^T + hi lo^T + lo hi^T; bf16 samples
- * are exact in tf32 (their lo is 0, so those MMAs are skipped).  Each 32
- * samples are accumulated afresh and added in fp32.  Only the lower-triangle
+ * On the tensor cores (tcgen05), FP32-accurate.  bf16 samples without
+ * weights: kind::f16 MMAs on the bf16 values (products exact in fp32), each
+ * 256 samples accumulated afresh in the tensor core and added in fp32.
+ * Otherwise kind::tf32 with operands split x = hi + lo and A B^T ~ hi hi^T +
+ * hi lo^T + lo hi^T (bf16 rows are exact in tf32, so their lo MMAs are
+ * skipped), each 32 samples accumulated afresh.  Only the lower-triangle
  * 128 x 128 blocks are computed.  Returns BAKRON_ERR_INVALID_ARG (bad
  * pointer, k < 1, d outside 1..65536, strides), BAKRON_ERR_WORKSPACE, or the
  * device status (BAKRON_ERR_TIMEOUT if a bounded wait ran out).

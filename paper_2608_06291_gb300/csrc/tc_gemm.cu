@@ -88,6 +88,10 @@ struct TcParams {
   // 128 boxes); a ring slot holds one box of each, K = 64 per slot, and the
   // MMAs are kind::f16 (bf16 x bf16 products exact in fp32)
   int bf16_ops;
+  // ring slots summed in place per TMEM accumulator before the epilogue reads
+  // it (0 or 1: one slot, the slot freed by its accumulator's commit; more:
+  // each slot freed by its own commit to `empty`)
+  int kgroup;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -343,7 +347,8 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint64_t* bars = (uint64_t*)(smem + STAGES * STAGE_BYTES);
   uint64_t* full = bars;                 // [STAGES] smem stage loaded
-  // bars + STAGES .. 2 STAGES - 1: unused (a slot is free when its stage's accF arrives)
+  uint64_t* empty = bars + STAGES;       // [STAGES] slot read by its MMAs (kgroup > 1 only;
+                                         // otherwise the slot's accF commit frees it)
   uint64_t* accum = bars + 2 * STAGES;   // [1] every MMA of the CTA complete
   uint64_t* accF = accum + 1;            // [NACC] accumulator holds a finished K stage
   uint64_t* accE = accum + 1 + NACC;     // [NACC] accumulator read out by the epilogue
@@ -370,6 +375,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
     }
     mbar_init(accum, 1);
     for (int a = 0; a < NACC; ++a) {
@@ -417,6 +423,8 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   pdl_trigger();
   const long long drain = 4000000000LL;   // ~2 s at 2 GHz: wind-down bound
   const int nk = blk.nk;
+  const int kgroup = P.kgroup > 1 ? P.kgroup : 1;
+  const int ngroups = (nk + kgroup - 1) / kgroup;   // accumulator hand-overs
 
   if (warp == 0) {
     // ---------------------------------------------------------- producer
@@ -429,7 +437,9 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
       // cannot have moved on to stage j + NACC yet, which needs this load
       if (lane == 0 && i >= STAGES) {
         const int j = i - STAGES;
-        ok = mbar_wait(&accF[j % NACC], (uint32_t)(j / NACC) & 1u, P.spin_cycles);
+        ok = kgroup > 1
+                 ? mbar_wait(&empty[s], (uint32_t)(j / STAGES) & 1u, P.spin_cycles)
+                 : mbar_wait(&accF[j % NACC], (uint32_t)(j / NACC) & 1u, P.spin_cycles);
       }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok || *abort_flag) {
@@ -512,22 +522,25 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
     }
   } else if (warp == 1) {
     // --------------------------------------------------------- MMA issuer
-    // Each K stage accumulates afresh into accumulator (stage mod NACC); the
-    // epilogue adds the stages in fp32 registers.  The tensor core's TF32
-    // accumulation is not round-to-nearest, and its error grows with the
-    // number of MMAs summed in place; restarting every 32 of K bounds it.
+    // Each group of kgroup K stages (one stage in the band products, four of
+    // exact bf16 products in the Gram) accumulates afresh into accumulator
+    // (group mod NACC); the epilogue adds the groups in fp32 registers.  The
+    // tensor core's accumulation is not round-to-nearest, and its error grows
+    // with the number of MMAs summed in place; restarting every group bounds it.
     if (lane == 0) {
       const uint32_t idesc = idesc_tf32(BM, BN), idesc_b = idesc_bf16(BM, BN);
       const uint64_t desc0 = smem_desc(smem_u32(smem));   // stage 0, A hi, K step 0
       for (int i = 0; i < nk; ++i) {
         const int s = i % STAGES;
         const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
-        const int a = i % NACC;
-        // accumulator a was last used by stage i - NACC: wait until it was read out
-        // (the producer's and the epilogue's aborts surface here as time-outs)
+        const int g = i / kgroup, a = g % NACC;     // accumulator group of this slot
+        const bool first = i % kgroup == 0;
+        const bool last = i % kgroup == kgroup - 1 || i == nk - 1;
+        // accumulator a was last used by group g - NACC: wait until it was read
+        // out (the producer's and the epilogue's aborts surface here as time-outs)
         const bool ok = mbar_wait(&full[s], ph, P.spin_cycles) &&
-                        (i < NACC ||
-                         mbar_wait(&accE[a], (uint32_t)(i / NACC - 1) & 1u, P.spin_cycles));
+                        (!first || g < NACC ||
+                         mbar_wait(&accE[a], (uint32_t)(g / NACC - 1) & 1u, P.spin_cycles));
         if (!ok) {
           raise_status(P.status, BAKRON_ERR_TIMEOUT);
           *abort_flag = 1;
@@ -543,17 +556,18 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
         if (bf16_ops) {
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)            // 16 bf16 = 32 bytes along K per MMA
-            mma_bf16(d, dah + 2 * kk, dbh + 2 * kk, idesc_b, kk > 0 ? 1u : 0u);
+            mma_bf16(d, dah + 2 * kk, dbh + 2 * kk, idesc_b, (kk > 0 || !first) ? 1u : 0u);
         } else {
 #pragma unroll
           for (int kk = 0; kk < BK / 8; ++kk) {
             const uint64_t o = (uint64_t)(2 * kk);   // 8 tf32 = 32 bytes along K inside the swizzle row
-            mma_tf32(d, dah + o, dbh + o, idesc, kk > 0 ? 1u : 0u);
+            mma_tf32(d, dah + o, dbh + o, idesc, (kk > 0 || !first) ? 1u : 0u);
             if (!P.b_exact) mma_tf32(d, dah + o, dbl + o, idesc, 1u);
             if (!P.a_exact) mma_tf32(d, dal + o, dbh + o, idesc, 1u);
           }
         }
-        mma_commit(&accF[a]);     // the stage's sum to the epilogue; its slot to the producer
+        if (kgroup > 1) mma_commit(&empty[s]);   // the slot back to the producer
+        if (last) mma_commit(&accF[a]);  // the group's sum to the epilogue (kgroup 1: and the slot)
       }
       if (nk > 0) mma_commit(accum);  // tracks every MMA issued above
       else mbar_arrive(accum);
@@ -570,7 +584,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
 #pragma unroll
     for (int u = 0; u < EPI_COLS; ++u) acc[u] = 0.f;
     bool write = true;
-    for (int i = 0; i < nk; ++i) {
+    for (int i = 0; i < ngroups; ++i) {
       const int a = i % NACC;
       // one lane waits; the decision is warp-uniform (tcgen05.ld is warp-collective)
       int ok = 1;
@@ -1029,6 +1043,8 @@ extern "C" int bakron_gram(const void* X, int xdtype, int k, int d, int64_t ldx,
     P.b_exact = xdtype == BAKRON_BF16;              // bf16 is exact in tf32: lo plane zero
     P.a_exact = xdtype == BAKRON_BF16 && !w;
     P.bf16_ops = bf16_ops ? 1 : 0;
+    // exact bf16 products: 4 slots (256 samples) per accumulator hand-over
+    P.kgroup = bf16_ops ? 4 : 1;
     k_tc_band<<<ntri, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mB2, mB2, mB2, mB2, P);
     BK_CUDA_OK(cudaGetLastError());
   }

@@ -3,11 +3,12 @@ Factorization"): bakron_gram (G <- beta G + alpha X^T diag(w) X on the
 tensor cores), bakron_sample_sqnorms and the K-FAC / one-step Shampoo factors,
 against the float64 oracle.
 
-Tolerance, from the arithmetic: each product is formed from tf32 hi/lo parts
-with a relative error below 2^-21 (exact for bf16 samples), each 32 samples
-are summed in the tensor core's accumulator and the stages in fp32, so
-|G - G_ref| <= 2^-14 * sum_t |alpha w_t x_ti x_tj| + 2^-20 |beta G0| holds
-with a wide margin for the sample counts used here (k <= 8192).
+Tolerance, from the arithmetic: each product is exact (bf16 samples, kind::f16)
+or formed from tf32 hi/lo parts with a relative error below 2^-21; at most 256
+products are summed in place in the tensor core's fp32 accumulator (<= 256 *
+2^-23 of their absolute sum, about 3e-5) and the groups in fp32 registers
+(<= k/256 * 2^-24), so |G - G_ref| <= 2^-14 * sum_t |alpha w_t x_ti x_tj| +
+2^-20 |beta G0| holds for the sample counts used here (k <= 8192).
 """
 import numpy as np
 import pytest
@@ -59,23 +60,28 @@ def test_gram_matches_oracle(k, d, dtype, weighted):
     _check(G, X.double().numpy(), None if w is None else w.double().numpy(), 1.0 / k, 0.0, None)
 
 
-def test_gram_beta_and_chunks():
+@pytest.mark.parametrize("dtype,weighted", [(torch.float32, True), (torch.bfloat16, False)])
+def test_gram_beta_and_chunks(dtype, weighted):
     """beta applies once, before the first chunk; many small chunks (a
-    workspace holding 64 samples) give the one-chunk result to rounding."""
+    workspace sized for 64 samples: 64 of them on the tf32 path, 256 on the
+    bf16 one, whose last chunk ends in a partial group of slots) give the
+    one-chunk result to rounding."""
     k, d = 1000, 200
-    X = _samples(k, d, 3, torch.float32).cuda()
-    w = (torch.rand(k, generator=torch.Generator().manual_seed(1)) + 0.5).cuda()
+    X = _samples(k, d, 3, dtype).cuda()
+    w = (torch.rand(k, generator=torch.Generator().manual_seed(1)) + 0.5).cuda() if weighted \
+        else None
     G0 = torch.randn(d, d, generator=torch.Generator().manual_seed(2))
     G0 = (G0 + G0.T).cuda()
     G1 = G0.clone()
     P.bakron_gram(X, w, alpha=0.25, beta=-0.5, G=G1)
     G2 = G0.clone()
-    ws = torch.empty(P.bakron_gram_workspace_bytes(d, 64, True), dtype=torch.uint8, device="cuda")
+    ws = torch.empty(P.bakron_gram_workspace_bytes(d, 64, weighted), dtype=torch.uint8,
+                     device="cuda")
     P.bakron_gram(X, w, alpha=0.25, beta=-0.5, G=G2, workspace=ws)
     torch.cuda.synchronize()
     for G in (G1, G2):
-        _check(G, X.double().cpu().numpy(), w.double().cpu().numpy(), 0.25, -0.5,
-               G0.double().cpu().numpy())
+        _check(G, X.double().cpu().numpy(), None if w is None else w.double().cpu().numpy(),
+               0.25, -0.5, G0.double().cpu().numpy())
 
 
 def test_gram_strided_operands():
