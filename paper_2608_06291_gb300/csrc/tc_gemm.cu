@@ -84,15 +84,21 @@ struct TcParams {
   float alpha, beta;
   int dreal;
   int a_exact, b_exact;
-  // Gram mode with bf16 operands: mapA2 / mapB2 are plain bf16 maps (64 x
-  // 128 boxes); a ring slot holds one box of each, K = 64 per slot, and the
-  // MMAs are kind::f16 (bf16 x bf16 products exact in fp32)
-  int bf16_ops;
-  // ring slots summed in place per TMEM accumulator before the epilogue reads
-  // it (0 or 1: one slot, the slot freed by its accumulator's commit; more:
-  // each slot freed by its own commit to `empty`)
-  int kgroup;
 };
+
+// Kernel variants (compile time, so that the band products' issue loop
+// carries no Gram logic):
+//   V_BAND      band products and the dense diagnostic: 3xTF32, one K stage
+//               per TMEM accumulator, a slot freed by its accumulator's commit
+//   V_GRAM_TF32 Gram on tf32 hi/lo planes; a_exact / b_exact skip the MMAs
+//               of an operand whose lo plane is zero
+//   V_GRAM_BF16 Gram on bf16 planes: mapA2 / mapB2 are plain bf16 maps (64 x
+//               128 boxes), a ring slot holds one box of each (K = 64), the
+//               MMAs are kind::f16 (bf16 x bf16 products exact in fp32), and
+//               GRAM_KGROUP slots are summed in place per accumulator, each
+//               slot freed by its own commit to `empty`
+enum Variant { V_BAND = 0, V_GRAM_TF32 = 1, V_GRAM_BF16 = 2 };
+constexpr int GRAM_KGROUP = 4;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);
@@ -311,7 +317,7 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
     b.rb = rb;
     b.cb = t - rb * (rb + 1) / 2;
     b.k0 = 0;
-    b.nk = P.K / (P.bf16_ops ? 2 * BK : BK);   // 128-byte rows: 32 fp32 or 64 bf16
+    b.nk = P.K / BK;   // K stages; the bf16 variant's K counts 128-byte rows of 64
     return true;
   }
   int cb_lo, cb_hi;
@@ -337,6 +343,7 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
   return true;
 }
 
+template <int V>
 __global__ void __launch_bounds__(THREADS, 1)
 k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUtensorMap mapB2,
           const __grid_constant__ CUtensorMap mapBh, const __grid_constant__ CUtensorMap mapBl,
@@ -401,12 +408,12 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   // wait for the previous kernel, whose output (E^T or M) is the other one.
   const int npre = blk.nk < STAGES ? blk.nk : STAGES;
   const bool a_static = P.mode != MODE_STAGE2;
-  const bool bf16_ops = P.mode == MODE_GRAM && P.bf16_ops;
+  constexpr bool bf16_ops = V == V_GRAM_BF16;
   if (warp == 0 && lane == 0) {
     for (int i = 0; i < npre; ++i) {
       unsigned char* st = smem + i * STAGE_BYTES;
       const int kt = blk.k0 + i;
-      if (bf16_ops) {
+      if constexpr (bf16_ops) {
         mbar_expect_tx_only(&full[i], TILE_BYTES);
         tma_load_2d(st, &mapA2, &full[i], kt * 2 * BK, blk.rb * BM);
         continue;
@@ -423,7 +430,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   pdl_trigger();
   const long long drain = 4000000000LL;   // ~2 s at 2 GHz: wind-down bound
   const int nk = blk.nk;
-  const int kgroup = P.kgroup > 1 ? P.kgroup : 1;
+  constexpr int kgroup = V == V_GRAM_BF16 ? GRAM_KGROUP : 1;
   const int ngroups = (nk + kgroup - 1) / kgroup;   // accumulator hand-overs
 
   if (warp == 0) {
@@ -437,9 +444,10 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
       // cannot have moved on to stage j + NACC yet, which needs this load
       if (lane == 0 && i >= STAGES) {
         const int j = i - STAGES;
-        ok = kgroup > 1
-                 ? mbar_wait(&empty[s], (uint32_t)(j / STAGES) & 1u, P.spin_cycles)
-                 : mbar_wait(&accF[j % NACC], (uint32_t)(j / NACC) & 1u, P.spin_cycles);
+        if constexpr (kgroup > 1)
+          ok = mbar_wait(&empty[s], (uint32_t)(j / STAGES) & 1u, P.spin_cycles);
+        else
+          ok = mbar_wait(&accF[j % NACC], (uint32_t)(j / NACC) & 1u, P.spin_cycles);
       }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok || *abort_flag) {
@@ -455,7 +463,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
       unsigned char *a_hi = st, *b_hi = st + 2 * TILE_BYTES, *b_lo = st + 3 * TILE_BYTES;
       const int kt = blk.k0 + i;            // K tile index (32 wide)
       const bool pre = i < npre;            // the factor operand is already on its way
-      if (bf16_ops) {                       // one bf16 box per operand, 64 of K
+      if constexpr (bf16_ops) {             // one bf16 box per operand, 64 of K
         if (lane == 0) {
           mbar_expect_tx(&full[s], pre ? TILE_BYTES : 2 * TILE_BYTES);
           if (!pre) tma_load_2d(a_hi, &mapA2, &full[s], kt * 2 * BK, blk.rb * BM);
@@ -553,7 +561,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
         const uint64_t dal = dah + (TILE_BYTES >> 4), dbh = dah + (2 * TILE_BYTES >> 4),
                        dbl = dah + (3 * TILE_BYTES >> 4);
         const uint32_t d = tmem + (uint32_t)(a * BN);
-        if (bf16_ops) {
+        if constexpr (bf16_ops) {
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)            // 16 bf16 = 32 bytes along K per MMA
             mma_bf16(d, dah + 2 * kk, dbh + 2 * kk, idesc_b, (kk > 0 || !first) ? 1u : 0u);
@@ -562,11 +570,11 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
           for (int kk = 0; kk < BK / 8; ++kk) {
             const uint64_t o = (uint64_t)(2 * kk);   // 8 tf32 = 32 bytes along K inside the swizzle row
             mma_tf32(d, dah + o, dbh + o, idesc, (kk > 0 || !first) ? 1u : 0u);
-            if (!P.b_exact) mma_tf32(d, dah + o, dbl + o, idesc, 1u);
-            if (!P.a_exact) mma_tf32(d, dal + o, dbh + o, idesc, 1u);
+            if (V == V_BAND || !P.b_exact) mma_tf32(d, dah + o, dbl + o, idesc, 1u);
+            if (V == V_BAND || !P.a_exact) mma_tf32(d, dal + o, dbh + o, idesc, 1u);
           }
         }
-        if (kgroup > 1) mma_commit(&empty[s]);   // the slot back to the producer
+        if constexpr (kgroup > 1) mma_commit(&empty[s]);   // the slot back to the producer
         if (last) mma_commit(&accF[a]);  // the group's sum to the epilogue (kgroup 1: and the slot)
       }
       if (nk > 0) mma_commit(accum);  // tracks every MMA issued above
@@ -776,7 +784,14 @@ cudaError_t ensure_attr() {
   std::lock_guard<std::mutex> lk(g_attr_mu);
   if (g_attr_done) return cudaSuccess;
   cudaError_t e =
-      cudaFuncSetAttribute(k_tc_band, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+      cudaFuncSetAttribute(k_tc_band<V_BAND>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           SMEM_BYTES);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_tc_band<V_GRAM_TF32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             SMEM_BYTES);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_tc_band<V_GRAM_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             SMEM_BYTES);
   if (e == cudaSuccess) g_attr_done = true;
   return e;
 }
@@ -921,10 +936,12 @@ int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, in
   dim3 grid(width, rhi - rlo + 1);
   cudaError_t e;
   if (stage == 1)
-    e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.LB2, maps.Et2, maps.Eth,
+    e = launch_pdl(k_tc_band<V_BAND>, grid, dim3(THREADS), SMEM_BYTES, s, maps.LB2, maps.Et2,
+                   maps.Eth,
                    maps.Etl, maps.Mh, maps.Ml, P);
   else   // (the 32-row E^T maps are not read in stage 2)
-    e = launch_pdl(k_tc_band, grid, dim3(THREADS), SMEM_BYTES, s, maps.M2, maps.LA2, maps.Eth,
+    e = launch_pdl(k_tc_band<V_BAND>, grid, dim3(THREADS), SMEM_BYTES, s, maps.M2, maps.LA2,
+                   maps.Eth,
                    maps.Etl, maps.X32, maps.X32, P);
   return e == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
 }
@@ -964,7 +981,7 @@ extern "C" int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C,
   P.status = status;
   P.spin_cycles = spin_cycles_from_env();
   dim3 grid(N / BN, M / BM);
-  k_tc_band<<<grid, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mBh, mBl, mBh, mBl, P);
+  k_tc_band<V_BAND><<<grid, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mBh, mBl, mBh, mBl, P);
   BK_CUDA_OK(cudaGetLastError());
   return bakron_read_status(workspace, stream);
 }
@@ -1042,10 +1059,14 @@ extern "C" int bakron_gram(const void* X, int xdtype, int k, int d, int64_t ldx,
     P.dreal = d;
     P.b_exact = xdtype == BAKRON_BF16;              // bf16 is exact in tf32: lo plane zero
     P.a_exact = xdtype == BAKRON_BF16 && !w;
-    P.bf16_ops = bf16_ops ? 1 : 0;
-    // exact bf16 products: 4 slots (256 samples) per accumulator hand-over
-    P.kgroup = bf16_ops ? 4 : 1;
-    k_tc_band<<<ntri, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mB2, mB2, mB2, mB2, P);
+    // bf16: K counted in 128-byte rows of 64; exact products, GRAM_KGROUP
+    // slots (256 samples) per accumulator hand-over
+    if (bf16_ops) {
+      P.K = (int)(kcl / 2);
+      k_tc_band<V_GRAM_BF16><<<ntri, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mB2, mB2, mB2, mB2, P);
+    } else {
+      k_tc_band<V_GRAM_TF32><<<ntri, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mB2, mB2, mB2, mB2, P);
+    }
     BK_CUDA_OK(cudaGetLastError());
   }
   if (!sync) return BAKRON_OK;
