@@ -53,6 +53,25 @@ def _dist():
     return ws, rank, local
 
 
+def max_over_ranks(x: float, ws_n: int, device="cpu") -> float:
+    """The slowest rank's time: all-reduce MAX of x over the process group
+    (identity for one process).  `device` is where the collective's tensor
+    lives (the GPU for NCCL, "cpu" for gloo)."""
+    if ws_n <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, ws_n: int, ms: float) -> float:
+    """Units all ranks processed (each rank the same, weak scaling) per second
+    of the slowest rank's time."""
+    return ws_n * units_per_rank / (ms / 1e3)
+
+
 def _peaks():
     try:
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
@@ -286,13 +305,10 @@ def run_gpu(args):
     w1 = time.time()
     clocks = sampler.stop(w0, w1) if sampler else None
     ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / args.steps
-    if ws_n > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, ws_n, dev)
     if P.bakron_read_status(work) != 0:
         raise RuntimeError("device status set during the timed steps")
-    value = ws_n * m * n / (ms / 1e3)
+    value = whole_job_rate(m * n, ws_n, ms)
 
     # per-family device time, live, with events on the launch stream
     P.bakron_profile_enable(True)
@@ -390,12 +406,8 @@ def run_gpu(args):
         e1.record(stream)
         e1.synchronize()
         tot += e0.elapsed_time(e1)
-    e2e_ms = tot / e2e_steps
-    if ws_n > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e = {"value": ws_n * m * n / (e2e_ms / 1e3), "unit": UNIT,
+    e2e_ms = max_over_ranks(tot / e2e_steps, ws_n, dev)
+    e2e = {"value": whole_job_rate(m * n, ws_n, e2e_ms), "unit": UNIT,
            "h2d_bytes_per_step": Wh.numel() * Wh.element_size(),
            "d2h_bytes_per_step": ch.numel() + 4 * (sh.numel() + zh.numel()),
            "ms_per_step": e2e_ms}
