@@ -846,22 +846,48 @@ __global__ void k_gram_split(const void* X, int xdt, int k, int d, int64_t ldx, 
 
 // bf16 samples t0 .. t0 + kc of X (k x d, row stride ldx) transposed into
 // the K-major bf16 plane T = X^T (dp x kc, zeros past k and d): the operand of
-// the kind::f16 Gram, exact (no split).
-__global__ void k_gram_transpose_bf16(const __nv_bfloat16* X, int k, int d, int64_t ldx, int t0,
-                                      int kc, __nv_bfloat16* T) {
-  __shared__ __nv_bfloat16 tile[32][34];
-  const int tx = threadIdx.x, ty = threadIdx.y;     // 32 x 8
-  const int tb = blockIdx.x * 32, ib = blockIdx.y * 32;
+// the kind::f16 Gram, exact (no split).  64 x 64 tiles through shared memory,
+// 16-byte vectors both ways: a load is 8 features of one sample (when X and
+// ldx allow 16-byte alignment and the 8 lie inside d; else element by
+// element), a store 8 samples of one feature (always whole: dp and kc are
+// multiples of 64).  A warp reads 4 rows of 128 bytes and stores 32 rows'
+// 16-byte pieces; its shared-memory gathers read one 64-byte row segment.
+constexpr int TR_TILE = 64, TR_LD = 72;   // row stride 144 B: 16-byte aligned rows
+
+__global__ void __launch_bounds__(256)
+    k_gram_transpose_bf16(const __nv_bfloat16* X, int k, int d, int64_t ldx, int t0, int kc,
+                          int vec_ok, __nv_bfloat16* T) {
+  __shared__ __align__(16) __nv_bfloat16 tile[TR_TILE][TR_LD];
+  const int tb = blockIdx.x * TR_TILE, ib = blockIdx.y * TR_TILE;
 #pragma unroll
-  for (int r = 0; r < 4; ++r) {
-    const int t = t0 + tb + ty + 8 * r, i = ib + tx;
-    tile[ty + 8 * r][tx] = (t < k && i < d) ? X[(int64_t)t * ldx + i] : __float2bfloat16(0.f);
+  for (int r = 0; r < 2; ++r) {
+    const int c = threadIdx.x + 256 * r;          // 512 chunks of 8 features
+    const int tr = c >> 3, i0 = ib + 8 * (c & 7);
+    const int t = t0 + tb + tr;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (t < k) {
+      const __nv_bfloat16* src = X + (int64_t)t * ldx + i0;
+      if (vec_ok && i0 + 8 <= d) {
+        v = *reinterpret_cast<const uint4*>(src);
+      } else {
+        __align__(16) __nv_bfloat16 e[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) e[j] = (i0 + j < d) ? src[j] : __float2bfloat16(0.f);
+        v = *reinterpret_cast<const uint4*>(e);
+      }
+    }
+    *reinterpret_cast<uint4*>(&tile[tr][8 * (c & 7)]) = v;
   }
   __syncthreads();
 #pragma unroll
-  for (int r = 0; r < 4; ++r) {
-    const int i = ib + ty + 8 * r, tc = tb + tx;
-    T[(int64_t)i * kc + tc] = tile[tx][ty + 8 * r];
+  for (int r = 0; r < 2; ++r) {
+    const int c = threadIdx.x + 256 * r;          // 512 chunks of 8 samples
+    const int ir = c & 63, tc = c >> 6;
+    __align__(16) __nv_bfloat16 e[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) e[j] = tile[8 * tc + j][ir];
+    *reinterpret_cast<uint4*>(T + (int64_t)(ib + ir) * kc + tb + 8 * tc) =
+        *reinterpret_cast<const uint4*>(e);
   }
 }
 
@@ -1032,8 +1058,10 @@ extern "C" int bakron_gram(const void* X, int xdtype, int k, int d, int64_t ldx,
     CUtensorMap mA2, mB2;
     if (bf16_ops) {
       __nv_bfloat16* Tb = (__nv_bfloat16*)(ws + 256);
-      k_gram_transpose_bf16<<<sg, dim3(32, 8), 0, s>>>((const __nv_bfloat16*)X, k, d, ldx,
-                                                       (int)t0, (int)kc, Tb);
+      const int vec_ok = ((uintptr_t)X % 16 == 0 && ldx % 8 == 0) ? 1 : 0;
+      dim3 tg((unsigned)(kcl / TR_TILE), (unsigned)(dp / TR_TILE));
+      k_gram_transpose_bf16<<<tg, 256, 0, s>>>((const __nv_bfloat16*)X, k, d, ldx, (int)t0,
+                                               (int)kc, vec_ok, Tb);
       BK_CUDA_OK(cudaGetLastError());
       if (!make_map_bf16(&mA2, Tb, dp, kcl, kc, BM) || !make_map_bf16(&mB2, Tb, dp, kcl, kc, BN))
         return BAKRON_ERR_CUDA;

@@ -102,3 +102,35 @@ def test_batched_graph_capture():
     for h in range(H):
         c, sc, z = P.bakron_solve(Ws[h], fs[h], 4, 0)
         assert torch.equal(outs[h][0], c) and torch.equal(outs[h][1], sc)
+
+
+def test_batched_bench_workload_certificate():
+    """The bench's workload: the 4096 x 4096 layer as 32 heads of 128 x 4096
+    over 16 lanes, each head certified (teacher-forced, every entry) against
+    fp64 factors of its own damped Grams."""
+    cfg = WL.CONFIGS[2]
+    W, A, _ = WL.make(cfg, device="cuda")
+    Hh, mh, n = 32, 128, cfg.n
+    Bs = [WL.power_law_gram(mh, cfg.n_samples, cfg.alpha_b, 9000 + h, 9100 + h, "cuda")
+          for h in range(Hh)]
+    LA, _, rA, _ = P.bakron_get_factors(P.bakron_prepare(A, Bs[0], cfg.damp))
+    fs = []
+    for h in range(Hh):
+        LBh, _, rBh, _ = P.bakron_get_factors(P.bakron_prepare(Bs[h], Bs[h], cfg.damp))
+        fs.append(P.bakron_set_factors(LA, LBh, rA, rBh))
+    Ws = [W[h * mh:(h + 1) * mh] for h in range(Hh)]
+    outs = P.bakron_solve_batched(Ws, fs, cfg.bits, 0, streams=16)
+    torch.cuda.synchronize()
+    RA = O.rev_cholesky(O.damped(to_np(A), cfg.damp))
+    W64 = to_np(W.float())
+    for h in range(Hh):
+        RB = O.rev_cholesky(O.damped(to_np(Bs[h]), cfg.damp))
+        Wh = W64[h * mh:(h + 1) * mh]
+        g = O.quant_grid(Wh, cfg.bits, 0)
+        np.testing.assert_array_equal(outs[h][1].cpu().numpy(), g.s)
+        c = outs[h][0].cpu().numpy().astype(np.int64)
+        rows = np.arange(mh)
+        D = O.dequantize(c, g, n) - Wh
+        _, bad, dist = O.certificate_rows(Wh, c, D, g, RA, RB, rows)
+        assert int((bad & (dist >= 1e-4)).sum()) == 0, h
+        assert int(bad.sum()) <= 1e-3 * bad.size

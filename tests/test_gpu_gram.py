@@ -139,3 +139,26 @@ def test_gram_attention_width_sampled():
     assert np.all(np.abs(got - ref) <= bnd)
     Gc = G.cpu()
     assert torch.equal(Gc, Gc.T)
+
+
+def test_gram_bench_workload_sampled():
+    """The bench's workload: 65536 bf16 rows of 4096 features in one chunk;
+    500 sampled entries against fp64 dot products, and exact symmetry."""
+    k, d = 65536, 4096
+    g = torch.Generator(device="cuda").manual_seed(4096)
+    X = (torch.randn(k, d, generator=g, device="cuda")
+         * torch.linspace(0.2, 3.0, d, device="cuda")).to(torch.bfloat16)
+    ws = torch.empty(P.bakron_gram_workspace_bytes(d, k, False), dtype=torch.uint8,
+                     device="cuda")
+    G = P.bakron_gram(X, alpha=1.0 / k, workspace=ws)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(1)
+    I = rng.integers(0, d, 500)
+    J = rng.integers(0, d, 500)
+    XI = X[:, torch.from_numpy(I).cuda()].double().cpu().numpy()
+    XJ = X[:, torch.from_numpy(J).cuda()].double().cpu().numpy()
+    ref = np.einsum("ti,ti->i", XI, XJ) / k
+    bnd = 2.0 ** -14 * np.einsum("ti,ti->i", np.abs(XI), np.abs(XJ)) / k
+    got = G.cpu().numpy()[I, J].astype(np.float64)
+    assert np.all(np.abs(got - ref) <= bnd)
+    assert torch.equal(G, G.T)
