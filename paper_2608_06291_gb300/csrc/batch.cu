@@ -26,7 +26,8 @@
 namespace bakron {
 int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
                int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given);
+               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
+               bool keep_status);
 
 namespace {
 
@@ -102,13 +103,17 @@ int bakron_solve_batched(int H, const void* const* W, int wdtype, int m, int n, 
   int rc = lanes_for(S, &L);
   if (rc != BAKRON_OK) return rc;
   BK_CUDA_OK(cudaEventRecord(L->fork, s));
-  for (int l = 0; l < S; ++l) BK_CUDA_OK(cudaStreamWaitEvent(L->stream[l], L->fork, 0));
+  // each lane clears its status word once; its solves keep the first error
+  for (int l = 0; l < S; ++l) {
+    BK_CUDA_OK(cudaStreamWaitEvent(L->stream[l], L->fork, 0));
+    BK_CUDA_OK(cudaMemsetAsync(ws + (size_t)l * slice, 0, 256, L->stream[l]));
+  }
   int launches = 0;
   for (int h = 0; h < H && rc == BAKRON_OK; ++h) {
     const int l = h % S;
     rc = solve_impl(W[h], wdtype, m, n, ldw, factors[h], (1 << bits) - 1, group_size, codes[h],
                     scales[h], zeros[h], nullptr, ws + (size_t)l * slice, L->stream[l], nullptr,
-                    false);
+                    false, true);
     launches += launch_count();
   }
   // join every lane, also after a failed enqueue (what was enqueued stays ordered)

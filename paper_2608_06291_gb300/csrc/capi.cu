@@ -12,7 +12,8 @@ int prepare_impl(const float* A, const float* B, int m, int n, float damp, void*
                  void* workspace, cudaStream_t s);
 int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
                int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given);
+               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
+               bool keep_status);
 int launch_grid_sym(const void* W, int wdt, int m, int n, int64_t ldw, int levels,
                     int group_size, int shrink_steps, float* scales, float* zeros,
                     cudaStream_t s);
@@ -125,7 +126,7 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw, const voi
   if (workspace_bytes < SolveLayout(m, n).bytes) return BAKRON_ERR_WORKSPACE;
   cudaStream_t s = (cudaStream_t)stream;
   int rc = solve_impl(W, wdtype, m, n, ldw, factors, (1 << bits) - 1, group_size, codes, scales,
-                      zeros, prerounding, workspace, s, nullptr, false);
+                      zeros, prerounding, workspace, s, nullptr, false, false);
   if (rc != BAKRON_OK || !sync) return rc;
   return bakron_read_status(workspace, stream);
 }
@@ -156,7 +157,7 @@ int bakron_solve_with_grid(const void* W, int wdtype, int m, int n, int64_t ldw,
   // the grid is only read when grid_given is set
   int rc = solve_impl(W, wdtype, m, n, ldw, factors, qmax, group_size, codes,
                       const_cast<float*>(scales), const_cast<float*>(zeros), prerounding,
-                      workspace, s, nullptr, true);
+                      workspace, s, nullptr, true, false);
   if (rc != BAKRON_OK || !sync) return rc;
   return bakron_read_status(workspace, stream);
 }

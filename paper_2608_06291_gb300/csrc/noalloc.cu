@@ -12,7 +12,8 @@
 namespace bakron {
 int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
                int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given);
+               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
+               bool keep_status);
 
 // The scratch.  Every GPU that loads the library holds it until the process
 // exits.  In host code this name is only a stand-in for the device symbol:
@@ -60,7 +61,7 @@ extern "C" int bakron_solve_noalloc(const void* W, int wdtype, int m, int n, int
   if (noalloc_scratch(&scratch) != cudaSuccess) return BAKRON_ERR_CUDA;
   cudaStream_t s = (cudaStream_t)stream;
   int rc = solve_impl(W, wdtype, m, n, ldw, factors, (1 << bits) - 1, group_size, codes, scales,
-                      zeros, prerounding, scratch, s, nullptr, false);
+                      zeros, prerounding, scratch, s, nullptr, false, false);
   if (rc != BAKRON_OK || !sync) return rc;
   return bakron_read_status(scratch, stream);
 }

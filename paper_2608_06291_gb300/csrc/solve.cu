@@ -1337,9 +1337,13 @@ static void rec(SolveArgs& a, int k, int l) {
 // `force`: thresholds to use instead of tuning_for(m, n) (the autotuner's candidates).
 // `grid_given`: scales and zeros hold the caller's grid (read only); otherwise
 // the min-max grid over qmax + 1 codes is computed into them first.
+// `keep_status`: leave the status word as it is (a batch of solves sharing the
+// workspace keeps the first error of any of them); the grid-barrier words
+// after it are cleared either way.
 int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
                int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given) {
+               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
+               bool keep_status) {
   FactorLayout fl(m, n);
   SolveLayout sl(m, n);
   char* ws = (char*)workspace;
@@ -1395,7 +1399,10 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
     }
   }
   reset_launch_count();
-  BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_status, 0, 256, s));
+  if (keep_status)
+    BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_status + 64, 0, 256 - 64, s));
+  else
+    BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_status, 0, 256, s));
   if (!grid_given) {
     const int64_t warps = (int64_t)m * a.G;
     LaunchScope ls(kFamInit, s);

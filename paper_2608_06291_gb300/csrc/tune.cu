@@ -17,7 +17,8 @@ namespace bakron {
 
 int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
                int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given);
+               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
+               bool keep_status);
 
 namespace {
 std::mutex g_mu;
@@ -85,7 +86,7 @@ int bakron_autotune(const void* W, int wdtype, int m, int n, int64_t ldw, const 
       for (int rep = 0; rep < 3 && rc == BAKRON_OK; ++rep) {   // rep 0 warms up
         if (cudaEventRecord(e0, s) != cudaSuccess) { rc = BAKRON_ERR_CUDA; break; }
         rc = solve_impl(W, wdtype, m, n, ldw, factors, (1 << bits) - 1, group_size, codes,
-                        scales, zeros, nullptr, workspace, s, &cand, false);
+                        scales, zeros, nullptr, workspace, s, &cand, false, false);
         if (rc != BAKRON_OK) break;
         if (cudaEventRecord(e1, s) != cudaSuccess) { rc = BAKRON_ERR_CUDA; break; }
         rc = bakron_read_status(workspace, stream);   // synchronises the stream
