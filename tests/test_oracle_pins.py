@@ -261,6 +261,63 @@ def test_config1_recursive_equals_band():
     assert O.objective(W, a.V, f.A_d, f.B_d) < O.objective(W, O.rtn(W, g).V, f.A_d, f.B_d)
 
 
+# ------------------------------------------------------ quadrant recursion
+def _quadrant_order(W, LA, LB, grid):
+    """The rounding in another order than every tier of the oracle: recursion
+    over quadrants, top-left first, then top-right and bottom-left (no entry
+    of either precedes one of the other), then bottom-right; after each
+    quadrant its errors are added to the quadrants after it in the block.
+    Written here, apart from the oracle, from the dependency structure of
+    Sec. 3.3 (an entry's error reaches only entries below and right of it)."""
+    X = np.asarray(W, np.float64).copy()
+    m, n = X.shape
+    S, Z = grid.expand(n)
+    codes = np.zeros((m, n), np.int64)
+    E = np.zeros((m, n))
+
+    def spread(r0, r1, c0, c1, targets):
+        Eb = np.zeros((m, n))
+        Eb[r0:r1, c0:c1] = E[r0:r1, c0:c1]
+        upd = LB @ Eb @ LA.T
+        for (a0, a1, b0, b1) in targets:
+            X[a0:a1, b0:b1] += upd[a0:a1, b0:b1]
+
+    def rec(r0, r1, c0, c1):
+        if r1 - r0 == 1 and c1 - c0 == 1:
+            c, v = O.quantize(X[r0, c0], S[r0, c0], Z[r0, c0], grid.qmax)
+            codes[r0, c0] = int(c)
+            E[r0, c0] = v - X[r0, c0]
+            return
+        rm = (r0 + r1) // 2 if r1 - r0 > 1 else r1
+        cm = (c0 + c1) // 2 if c1 - c0 > 1 else c1
+        tl, tr, bl, br = (r0, rm, c0, cm), (r0, rm, cm, c1), (rm, r1, c0, cm), (rm, r1, cm, c1)
+        live = lambda b: b[0] < b[1] and b[2] < b[3]
+        rec(*tl)
+        spread(*tl, [b for b in (tr, bl, br) if live(b)])
+        for b in (tr, bl):
+            if live(b):
+                rec(*b)
+                if live(br):
+                    spread(*b, [br])
+        if live(br):
+            rec(*br)
+
+    rec(0, m, 0, n)
+    return codes, X
+
+
+@pytest.mark.parametrize("m,n,bits", [(5, 7, 3), (8, 8, 2), (9, 4, 4), (1, 6, 3), (6, 1, 3)])
+def test_quadrant_order_agrees(m, n, bits):
+    """Thm. 3.1: any order that respects the dependencies gives the same
+    codes and pre-rounding values as every tier."""
+    W, f, g = _problem(m, n, 900 + 7 * m + n, bits=bits)
+    codes, X = _quadrant_order(W, f.LA, f.LB, g)
+    ref = O.bakron_vectorized(W, f.A_d, f.B_d, g)
+    np.testing.assert_array_equal(codes, ref.codes)
+    np.testing.assert_allclose(X, ref.X, atol=1e-10)
+    np.testing.assert_array_equal(O.bakron(W, f.LA, f.LB, g).codes, codes)
+
+
 # --------------------------------------------------------- planted mistakes
 def _alg5_original_w(W, LA, LB, grid):
     """Alg. 5 with "V - W" read as values minus the ORIGINAL input (wrong)."""
