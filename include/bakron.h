@@ -19,8 +19,11 @@
  *
  * Conventions for every entry point:
  *  - Matrices are row-major.  Pointers marked "device" are CUDA device memory
- *    owned by the caller; the library never allocates, frees or retains them,
- *    and keeps no state between calls other than read-only constant tables.
+ *    owned by the caller; the library never allocates, frees or retains them.
+ *    State kept between calls: the per-shape schedule table of
+ *    bakron_autotune, the lane streams and events of bakron_solve_batched
+ *    (created on first use), the fixed scratch of bakron_solve_noalloc and
+ *    the profiling counters; all live until the process exits.
  *  - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is
  *    enqueued asynchronously on it unless stated otherwise.
  *  - Arguments are validated on the host before anything is enqueued; an
