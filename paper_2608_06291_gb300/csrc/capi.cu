@@ -6,14 +6,11 @@
 
 #include "common.cuh"
 #include "tune.cuh"
+#include "solve.cuh"
 
 namespace bakron {
 int prepare_impl(const float* A, const float* B, int m, int n, float damp, void* factors,
                  void* workspace, cudaStream_t s);
-int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
-               int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
-               bool keep_status);
 int launch_grid_sym(const void* W, int wdt, int m, int n, int64_t ldw, int levels,
                     int group_size, int shrink_steps, float* scales, float* zeros,
                     cudaStream_t s);

@@ -21,6 +21,7 @@
 #include "profile.cuh"
 #include "tc_gemm.cuh"
 #include "tune.cuh"
+#include "solve.cuh"
 #include <stdlib.h>
 
 #include <type_traits>

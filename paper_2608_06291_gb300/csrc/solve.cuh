@@ -1,0 +1,23 @@
+// The solve's internal entry point, shared by the C ABI (capi.cu), the
+// no-allocation variant (noalloc.cu), the autotuner (tune.cu) and the batched
+// solve (batch.cu).  Defined in solve.cu.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "tune.cuh"
+
+namespace bakron {
+
+// One BaKron solve of W (m x n) enqueued on `s` (arguments as bakron_solve,
+// validated by the caller).  qmax: codes 0..qmax.  force: schedule to use
+// instead of the per-shape table.  grid_given: scales/zeros hold the caller's
+// grid (read only) instead of being computed.  keep_status: leave the
+// workspace's status word as it is (a batch of solves keeps its first error).
+int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
+               int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
+               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
+               bool keep_status);
+
+}  // namespace bakron

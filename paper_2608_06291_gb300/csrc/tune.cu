@@ -12,13 +12,9 @@
 
 #include "common.cuh"
 #include "tune.cuh"
+#include "solve.cuh"
 
 namespace bakron {
-
-int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
-               int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
-               bool keep_status);
 
 namespace {
 std::mutex g_mu;
