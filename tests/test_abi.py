@@ -5,6 +5,7 @@ import os
 import re
 
 import pytest
+import torch
 
 import paper_2608_06291_gb300 as P
 
@@ -116,3 +117,19 @@ def test_invalid_arguments_rejected_on_host(L):
     assert sq(fake, 0, 4, 4, 3, fake, None) == 1
     assert sq(fake, 0, 0, 4, 4, fake, None) == 1
     assert P.strerror(2) == "damped Gram is not positive definite"
+
+
+def test_binding_rejects_bad_tensors_before_the_library():
+    """The ctypes binding checks device, dtype and shapes itself and raises
+    ValueError before calling into the library (no GPU needed)."""
+    cpu = torch.zeros(8, 4)
+    with pytest.raises(ValueError):
+        P.bakron_gram(cpu)                               # not a CUDA tensor
+    with pytest.raises(ValueError):
+        P.bakron_sample_sqnorms(cpu)
+    with pytest.raises(ValueError):
+        P.bakron_grid_symmetric(cpu)
+    with pytest.raises(ValueError):
+        P.bakron_solve_batched([], [], 4)                # no problems
+    with pytest.raises(ValueError):
+        P.bakron_solve_batched([cpu], [], 4)             # factors missing
