@@ -133,3 +133,20 @@ def test_binding_rejects_bad_tensors_before_the_library():
         P.bakron_solve_batched([], [], 4)                # no problems
     with pytest.raises(ValueError):
         P.bakron_solve_batched([cpu], [], 4)             # factors missing
+
+
+def test_header_is_plain_c(tmp_path):
+    """include/bakron.h compiles as C99 (-pedantic, warnings as errors): the
+    boundary carries no C++ or CUDA types."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    src = tmp_path / "use.c"
+    src.write_text('#include "bakron.h"\nint main(void) { return bakron_strerror(0) == 0; }\n')
+    r = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I", inc,
+                        "-c", str(src), "-o", str(tmp_path / "use.o")],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
