@@ -36,6 +36,8 @@ import sys
 import tempfile
 import time
 
+import numpy as np
+
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
@@ -161,6 +163,47 @@ def _oracle_block(W64, f, bits, group, k):
     c1 = os.times()
     cpu = (c1.user - c0.user) + (c1.system - c0.system)
     return wall, max(1, round(cpu / wall)) if wall > 0 else 1
+
+
+def _timed(fn):
+    """Wall time of fn() and the host threads it kept busy on average."""
+    c0 = os.times()
+    t0 = time.perf_counter()
+    fn()
+    wall = time.perf_counter() - t0
+    c1 = os.times()
+    cpu = (c1.user - c0.user) + (c1.system - c0.system)
+    return wall, max(1, round(cpu / wall)) if wall > 0 else 1
+
+
+def extra_cpu_baseline(workload, data):
+    """The oracle, as it stands, on a bounded sample of an extra workload's
+    input, in the unit of that workload's line.  `data` holds host float64
+    arrays (see run_extra):
+      gram     X (k_s x d sample rows): oracle Gram, flop/s d (d + 1) k_s / s
+      symgrid  W (rows x n sample): oracle symmetric grid, entries/s
+      batched / gptq  W, LA, LB (an exact top-left block: entry (i, j) depends
+               only on entries up-left of it), bits: oracle Alg. 4, entries/s"""
+    import oracle as O
+    if workload == "gram":
+        X = data["X"]
+        k_s, d = X.shape
+        wall, cores = _timed(lambda: O.gram(X, alpha=1.0 / k_s))
+        return {"value": d * (d + 1) * k_s / wall, "unit": "flop/s", "cores": cores,
+                "kind": "oracle",
+                "sample": f"first {k_s} of the rows ({k_s} x {d}), float64 Gram, {wall:.2f} s wall"}
+    if workload == "symgrid":
+        W = data["W"]
+        wall, cores = _timed(lambda: O.symmetric_grid(W.astype(np.float32), 3, 0, 50))
+        return {"value": W.size / wall, "unit": "entries/s", "cores": cores, "kind": "oracle",
+                "sample": f"first {W.shape[0]} rows ({W.shape[0]} x {W.shape[1]}), l = 3, "
+                          f"50 shrink steps, {wall:.2f} s wall"}
+    W, LA, LB, bits = data["W"], data["LA"], data["LB"], data["bits"]
+    g = O.quant_grid(W, bits, 0)
+    wall, cores = _timed(lambda: O.bakron_recursive(W, LA, LB, g))
+    return {"value": W.size / wall, "unit": "entries/s", "cores": cores, "kind": "oracle",
+            "sample": f"exact top-left {W.shape[0]} x {W.shape[1]} block, float64 Alg. 4, "
+                      f"{wall:.2f} s wall"}
 
 
 def _oracle_factors(A, B, damp):
@@ -489,6 +532,9 @@ def run_extra(args):
         roof_src = "of measured: bf16_tflops (burst; the Gram runs bf16 x bf16 MMAs)"
         cfg = {"workload": "kfac_gram", "k": k, "d": d, "dtype_in": "bf16",
                "l2": "flushed (256 MiB write) between steps; X 512 MiB > L2"}
+
+        def cpu_data():
+            return {"X": X[:4096].double().cpu().numpy()}
     elif args.workload == "gptq":
         # GPTQ as the method's B = I case (Sec. 1): the 4096 x 4096 weights
         # under the layer's input-side factor only
@@ -522,6 +568,12 @@ def run_extra(args):
         cfg = {"workload": "gptq_b_identity", "m": m, "n": n, "bits": 4,
                "launch": "cuda graph replay", "paper_gptq_s_rtx_pro_6000": 0.025,
                "l2": "flushed (256 MiB write) between steps"}
+
+        def cpu_data():
+            f = _oracle_factors(A, torch.ones(1, 1), cfg2.damp)      # A's factor only
+            b = 512
+            return {"W": W[:b, :b].double().cpu().numpy(), "LA": f.LA[:b, :b],
+                    "LB": np.eye(b), "bits": cfg2.bits}
     elif args.workload == "batched":
         cfg2 = WL.CONFIGS[2]
         W, A, _ = WL.make(cfg2, device=dev)
@@ -581,6 +633,11 @@ def run_extra(args):
         hbm = float(peaks.get("hbm_gbs", 6800.0))
         roof_peak = p_eff
         roof_src = "of measured: bf16_tflops_sustained x 1.1/2.25 (tf32/bf16) / 3"
+        def cpu_data():
+            f = _oracle_factors(A, Bs[0], cfg2.damp)                 # head 0's factors
+            b = 512
+            return {"W": W[:mh, :b].double().cpu().numpy(), "LA": f.LA[:b, :b], "LB": f.LB,
+                    "bits": cfg2.bits}
         cfg = {"workload": "batched_heads", "heads": Hh, "m_head": mh, "n": n, "bits": 4,
                "lanes": lanes, "launch": "cuda graph replay",
                "one_lane_ms": one_lane_ms, "A": "shared (4096x4096 layer's)",
@@ -602,6 +659,9 @@ def run_extra(args):
         roof_src = "152 SMs x 128 FP32 lanes x 2.07 GHz (one op per lane per clock)"
         cfg = {"workload": "grid_symmetric", "m": m, "n": n, "levels": 3, "shrink_steps": 50,
                "l2": "flushed (256 MiB write) between steps"}
+
+        def cpu_data():
+            return {"W": W[:512].double().cpu().numpy()}
     for _ in range(max(3, args.warmup)):
         flush.fill_(1)
         step()
@@ -656,12 +716,13 @@ def run_extra(args):
         roof = {"bound": "alu", "achieved": ops / (ms / 1e3) / 1e12, "peak": roof_peak,
                 "unit": "Tops/s", "frac": ops / (ms / 1e3) / 1e12 / roof_peak, "traffic": None,
                 "peak_source": roof_src}
+    cpu_base = None if args.no_cpu_baseline else extra_cpu_baseline(args.workload, cpu_data())
     print(json.dumps({
         "metric": metric, "value": value, "unit": unit, "n_gpus": 1, "steps": args.steps,
         "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": cfg, "roofline": roof, "gpu_launches": per_launch * args.steps,
-        "clocks": clocks, "e2e": None, "cpu_baseline": None}))
+        "clocks": clocks, "e2e": None, "cpu_baseline": cpu_base}))
     return 0
 
 

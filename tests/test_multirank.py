@@ -63,3 +63,23 @@ def test_reference_arm_only_on_rank_zero(monkeypatch, capsys):
         config, ref_block, steps, warmup = 2, 8, 1, 0
     assert bench.run_reference(Args()) == 0
     assert capsys.readouterr().out == ""
+
+
+def test_extra_lines_cpu_baseline_on_small_samples():
+    """The oracle leg of the extra bench lines runs on host arrays and reports
+    its value in the line's unit (small samples here)."""
+    import numpy as np
+    import workloads as WL
+    rng = np.random.default_rng(0)
+    r = bench.extra_cpu_baseline("gram", {"X": rng.normal(size=(64, 32))})
+    assert r["unit"] == "flop/s" and r["value"] > 0 and r["kind"] == "oracle"
+    r = bench.extra_cpu_baseline("symgrid", {"W": rng.standard_t(4, size=(8, 64))})
+    assert r["unit"] == "entries/s" and r["value"] > 0
+    W, A, B = WL.small_problem(24, 40, 3)
+    f = bench._oracle_factors(A, B, 0.01)
+    for wl in ("batched", "gptq"):
+        r = bench.extra_cpu_baseline(wl, {"W": W.double().numpy(), "LA": f.LA, "LB": f.LB,
+                                          "bits": 4})
+        assert r["unit"] == "entries/s" and r["value"] > 0 and r["cores"] >= 1
+    fa = bench._oracle_factors(A, torch.ones(1, 1), 0.01)           # A's factor alone
+    np.testing.assert_allclose(fa.LA, f.LA, rtol=1e-12, atol=1e-14)
