@@ -23,7 +23,10 @@ Tiers (all fp64, all give the same codes by Thm. 3.1):
                                Cholesky of its inverse, Alg. 1 in vec order.
   * ``bakron_naive``        -- Alg. 2 (row-major, rank-1 updates).
   * ``bakron_antidiagonal`` -- Alg. 3 (one batched update per anti-diagonal).
-  * ``bakron_recursive``    -- Alg. 4 (split the longer side, bulk update).
+  * ``bakron_recursive``    -- Alg. 4 (split the longer side, bulk update);
+                               with ``base`` > 1 it stops at blocks of at most
+                               base x base and rounds each by Alg. 3 restricted
+                               to the block (the full-size comparisons).
   * ``bakron``              -- Alg. 5 (halve the anti-diagonal range).
 Plus the textbook GPTQ loop (``gptq_rows``), round-to-nearest, the
 fixed-point certificate derived from the canonical definition, the objective
@@ -322,16 +325,55 @@ def bakron_antidiagonal(W, LA, LB, grid: Grid) -> Result:
 # ----------------------------------------------------------------------------
 # Alg. 4: BaKron-recursive (divide and conquer on the longer side).
 # ----------------------------------------------------------------------------
-def bakron_recursive(W, LA, LB, grid: Grid) -> Result:
+def bakron_recursive(W, LA, LB, grid: Grid, base: int = 1) -> Result:
     """Split columns if m < n else rows (first part floor(size/2)); solve the
     first part; W_2 += L^B (V_1 - W_1) L^A_21^T (column split) or
     L^B_21 (V_1 - W_1) L^A^T (row split); solve the second part.  The
-    workspace W is shared in place and keeps pre-rounding values."""
+    workspace W is shared in place and keeps pre-rounding values.
+
+    ``base`` (default 1: Alg. 4 down to single entries) stops the splitting at
+    blocks with at most ``base`` rows and ``base`` columns and rounds such a
+    block by Alg. 3 restricted to it: for each of its anti-diagonals, round the
+    entries, then add L^B_blk Delta L^A_blk^T to the block's later entries
+    (Delta: the errors of that anti-diagonal).  Inside a block only entries
+    up-left of an entry feed it, so this is the same problem Alg. 4 would solve
+    there, and by Thm. 3.1 every order gives the same codes; it only trades
+    the recursion's many tiny calls for a few anti-diagonal steps, which keeps
+    full-size problems within minutes."""
     Wk, S, Z = _setup(W, grid)
     m, n = Wk.shape
     V = np.zeros_like(Wk)
     codes = np.zeros_like(Wk)
     qmax = grid.qmax
+
+    diagonals = {}
+
+    def antidiagonals(mm, nn):
+        """Row and column indices of each anti-diagonal of an mm x nn block."""
+        if (mm, nn) not in diagonals:
+            i, j = np.divmod(np.arange(mm * nn), nn)
+            order = np.argsort(i + j, kind="stable")
+            k = (i + j)[order]
+            cuts = np.searchsorted(k, np.arange(mm + nn))
+            diagonals[(mm, nn)] = [(i[order][a:b], j[order][a:b])
+                                   for a, b in zip(cuts[:-1], cuts[1:])]
+        return diagonals[(mm, nn)]
+
+    def block(r0, r1, c0, c1):
+        LBb, LAb = LB[r0:r1, r0:r1], LA[c0:c1, c0:c1]
+        Wb, Sb, Zb = Wk[r0:r1, c0:c1], S[r0:r1, c0:c1], Z[r0:r1, c0:c1]
+        Cb, Vb = codes[r0:r1, c0:c1], V[r0:r1, c0:c1]
+        for ii, jj in antidiagonals(r1 - r0, c1 - c0):
+            x = Wb[ii, jj]
+            c, v = quantize(x, Sb[ii, jj], Zb[ii, jj], qmax)
+            Cb[ii, jj] = c
+            Vb[ii, jj] = v
+            # W_blk += L^B_blk Delta L^A_blk^T with Delta = v - x on this
+            # anti-diagonal: the sum of its columns' outer products.  Earlier
+            # entries receive exact zeros (the factors are lower triangular);
+            # the rounded entries themselves keep their pre-rounding values.
+            Wb += (LBb[:, ii] * (v - x)) @ LAb[:, jj].T
+            Wb[ii, jj] = x
 
     def rec(r0, r1, c0, c1):
         mm, nn = r1 - r0, c1 - c0
@@ -339,6 +381,9 @@ def bakron_recursive(W, LA, LB, grid: Grid) -> Result:
             c, v = quantize(Wk[r0, c0], S[r0, c0], Z[r0, c0], qmax)
             codes[r0, c0] = c
             V[r0, c0] = v
+            return
+        if base > 1 and mm <= base and nn <= base:
+            block(r0, r1, c0, c1)
             return
         if mm < nn:
             h = c0 + nn // 2

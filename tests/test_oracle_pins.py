@@ -89,6 +89,32 @@ def test_grid_degenerate_row_and_group_errors():
         O.quant_grid(np.zeros((2, 6)), 2, group=4)
 
 
+def test_midpoint_distance_hand_values():
+    """Distance in grid units from x/s to the nearest rounding boundary (a
+    half-integer), which decides what the certificate excuses as a tie.
+    Hand values: on a boundary 0, on an integer 1/2, just below a boundary the
+    gap, and negative values measured to the boundary on their own side."""
+    d = O.midpoint_distance
+    assert d(2.5, 1.0) == 0.0
+    assert d(-2.5, 1.0) == 0.0
+    assert d(3.0, 1.0) == 0.5
+    assert d(-3.0, 1.0) == 0.5
+    assert d(0.0, 1.0) == 0.5
+    assert d(4.49999, 1.0) == pytest.approx(1e-5, abs=1e-12)
+    assert d(4.50001, 1.0) == pytest.approx(1e-5, abs=1e-12)
+    assert d(-0.3, 1.0) == pytest.approx(0.2, abs=1e-12)       # nearest boundary -0.5
+    assert d(-0.7, 1.0) == pytest.approx(0.2, abs=1e-12)       # nearest boundary -0.5
+    assert d(1.2, 1.0) == pytest.approx(0.3, abs=1e-12)        # nearest boundary 1.5
+    # grid units: x = 0.75 on a grid of step 0.5 is 1.5 units, on a boundary
+    assert d(0.75, 0.5) == 0.0
+    assert d(0.5, 0.5) == 0.5
+    assert d(-0.2, 0.5) == pytest.approx(0.1, abs=1e-12)       # -0.4 units
+    # a tie exactly at the boundary is where rint's half-to-even rule acts
+    x = np.array([0.5, 1.5, 2.5, -0.5])
+    assert (O.midpoint_distance(x, 1.0) == 0).all()
+    np.testing.assert_array_equal(np.rint(x), [0.0, 2.0, 2.0, -0.0])
+
+
 def test_babai_step_is_argmin_over_alphabet():
     """Babai's greedy step picks the nearest alphabet element (P1)."""
     rng = np.random.default_rng(5)
@@ -142,6 +168,31 @@ def test_all_tiers_agree(m, n, bits):
     ref = O.bakron_vectorized(W, f.A_d, f.B_d, g)
     for solver in (O.bakron_naive, O.bakron_antidiagonal, O.bakron_recursive, O.bakron):
         r = solver(W, f.LA, f.LB, g)
+        np.testing.assert_array_equal(r.codes, ref.codes)
+        np.testing.assert_allclose(r.X, ref.X, atol=1e-10)
+
+
+@pytest.mark.parametrize("m,n", [(1, 7), (7, 1), (5, 9), (9, 5), (13, 11), (16, 16)])
+@pytest.mark.parametrize("base", [2, 3, 4, 8])
+def test_blocked_recursive_agrees(m, n, base):
+    """Alg. 4 stopped at blocks of at most base x base, each rounded by Alg. 3
+    restricted to the block, gives the definition's codes and pre-rounding
+    workspace (Thm. 3.1), also where blocks are ragged."""
+    W, f, g = _problem(m, n, 500 + 3 * m + n + base, bits=3)
+    ref = O.bakron_vectorized(W, f.A_d, f.B_d, g)
+    r = O.bakron_recursive(W, f.LA, f.LB, g, base=base)
+    np.testing.assert_array_equal(r.codes, ref.codes)
+    np.testing.assert_allclose(r.X, ref.X, atol=1e-10)
+    np.testing.assert_allclose(r.V, ref.V, atol=1e-12)
+
+
+def test_blocked_recursive_agrees_medium_with_groups():
+    """The blocked tier at the block sizes the full-size comparisons use, on a
+    problem several blocks wide with a ragged tail and column groups."""
+    W, f, g = _problem(150, 136, 41, bits=4, group=8)
+    ref = O.bakron_recursive(W, f.LA, f.LB, g)
+    for base in (32, 64):
+        r = O.bakron_recursive(W, f.LA, f.LB, g, base=base)
         np.testing.assert_array_equal(r.codes, ref.codes)
         np.testing.assert_allclose(r.X, ref.X, atol=1e-10)
 
@@ -354,6 +405,8 @@ def test_planted_mistakes_are_caught():
     # 2) a transposed factor changes the codes
     assert (O.bakron_naive(W, f.LA.T.copy(), f.LB, g).codes != ref).any()
     assert (O.bakron_recursive(W, f.LA, f.LB.T.copy(), g).codes != ref).any()
+    # 2b) inside a block of the blocked tier, a transposed factor is caught too
+    assert (O.bakron_recursive(W, f.LA, f.LB.T.copy(), g, base=4).codes != ref).any()
     # 3) a wrong sign on the error feedback fails the certificate
     r = O.bakron_recursive(W, -f.LA + 2 * np.eye(7), f.LB, g)
     _, bad, _ = O.certificate(W, r.codes, g, f.LA, f.LB)
