@@ -317,23 +317,36 @@ void bakron_autotune_clear(void);
  * problem fits when the solve's scratch, 256 + 20 * mp * np bytes (mp, np: m
  * and n rounded up to multiples of 128), is at most 64 MiB -- e.g. 1792 x
  * 1792 or 2048 x 1536; larger problems are rejected with BAKRON_ERR_WORKSPACE
- * before anything is enqueued.  The call allocates nothing: no cudaMalloc/cudaFree, no
- * allocating library routine.
+ * before anything is enqueued (sides above 131072 with BAKRON_ERR_INVALID_ARG,
+ * as bakron_solve does).  The call allocates nothing: no cudaMalloc/cudaFree,
+ * no allocating library routine.
  *
- * The first call on a device (the device current at the call) looks up the
- * array's device address once (cudaGetSymbolAddress) and caches it; make
- * that first call before any stream capture on that device.
+ * The first call in a CUDA context (the current device's context at the
+ * call) looks up the array's device address once (cudaGetSymbolAddress) and
+ * caches it under that context's id; make that first call before any stream
+ * capture on that device.  After a device reset the new context gets a new
+ * id, so the address is looked up again.
  * Every call on a device shares the one array and leaves its contents behind;
  * each call clears what must start at zero (the status word) and overwrites
  * the rest before reading it.  Calls whose work overlaps on the GPU (another
  * stream, another host thread, same device) race on the array: serialise
- * them.  Arguments, outputs and `sync` are those of bakron_solve.
+ * them.  Arguments and outputs are those of bakron_solve.  With sync = 1 the
+ * call synchronises `stream` and returns the device status; with sync = 0 it
+ * returns after enqueueing, and the device status of that solve (NOT_SPD,
+ * NONFINITE, TIMEOUT) is read, and cleared, by bakron_read_status_noalloc on
+ * the same device before the next noalloc call clears it.
  */
 #define BAKRON_NOALLOC_SCRATCH_BYTES ((size_t)64 << 20)
 int bakron_solve_noalloc(const void* W, int wdtype, int m, int n, int64_t ldw,
                          const void* factors, int bits, int group_size,
                          uint8_t* codes, float* scales, float* zeros,
                          float* prerounding, int sync, void* stream);
+
+/* bakron_read_status_noalloc -- synchronise `stream`, return and clear the
+ * status word of the last bakron_solve_noalloc on the current device (it
+ * lives in the fixed scratch array, whose address callers never see).
+ * Allocates nothing.  No counterpart in the paper. */
+int bakron_read_status_noalloc(void* stream);
 
 /* Synchronise `stream`, return and clear the device status word kept in
  * `workspace` by the last prepare/solve that used it. */

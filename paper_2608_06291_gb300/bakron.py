@@ -73,6 +73,8 @@ def lib() -> ctypes.CDLL:
     L.bakron_read_status_batched.restype = i32
     L.bakron_solve_noalloc.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, i32, vp]
     L.bakron_solve_noalloc.restype = i32
+    L.bakron_read_status_noalloc.argtypes = [vp]
+    L.bakron_read_status_noalloc.restype = i32
     L.bakron_read_status.argtypes = [vp, vp]
     L.bakron_read_status.restype = i32
     L.bakron_profile_enable.argtypes = [i32]
@@ -446,6 +448,12 @@ def bakron_solve_noalloc(W, f: Factors, bits: int, group_size: int = 0,
 
 def bakron_read_status(workspace, stream=None) -> int:
     return int(lib().bakron_read_status(_ptr(workspace), _stream(stream)))
+
+
+def bakron_read_status_noalloc(stream=None) -> int:
+    """Status of the last bakron_solve_noalloc on the current device (read
+    and cleared); the one way to see a device error of a sync=False call."""
+    return int(lib().bakron_read_status_noalloc(_stream(stream)))
 
 
 PROFILE_FAMILIES = ("init", "leaf", "band1", "band2", "copy", "tc1", "tc2", "fused", "subtree")

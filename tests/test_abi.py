@@ -62,6 +62,16 @@ def test_invalid_arguments_rejected_on_host(L):
     assert L.bakron_prepare(fake, fake, 4, 4, ctypes.c_float(0.01), fake, fake, 16, None) == 5
     assert L.bakron_set_factors(None, fake, None, None, 4, 4, fake, None) == 1
     assert L.bakron_read_status(None, None) == 1
+    # no-alloc solve: sides beyond 131072 are invalid (as for bakron_solve);
+    # valid problems whose scratch exceeds the fixed 64 MiB are refused as
+    # a workspace shortfall -- both on the host, before any device call
+    na = L.bakron_solve_noalloc
+    assert na(fake, 0, (1 << 17) + 1, 4, 4, fake, 4, 0, fake, fake, fake, None, 1, None) == 1
+    assert na(fake, 0, 4, (1 << 17) + 1, (1 << 17) + 1, fake, 4, 0, fake, fake, fake, None, 1,
+              None) == 1
+    assert na(fake, 0, 4096, 4096, 4096, fake, 4, 0, fake, fake, fake, None, 1, None) == 5
+    assert na(fake, 0, 1792, 1793, 1793, fake, 4, 0, fake, fake, fake, None, 1, None) == 5
+    assert na(None, 0, 4, 4, 4, fake, 4, 0, fake, fake, fake, None, 1, None) == 1
     # symmetric grid: levels, shrink steps, group, ldw, dtype
     g = L.bakron_grid_symmetric
     assert g(None, 0, 4, 4, 4, 3, 0, 50, fake, fake, None) == 1
