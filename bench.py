@@ -81,6 +81,76 @@ def _peaks():
         return None
 
 
+def f_alg(m: int, n: int, identity_b: bool = False) -> float:
+    """Algorithmic flops of one m x n solve: twice the multiply-adds with a
+    structurally nonzero factor operand in Alg. 4's recursion down to single
+    entries -- split the longer side (columns when m < n), first part
+    floor(size / 2), each bulk update L^B E L^A^T multiplied in its cheaper
+    order, triangular diagonal blocks counted at their strictly-lower part
+    (their unit diagonal adds, it does not multiply).  With B = I (GPTQ) the
+    output-side factor contributes no products at all.  4096 x 4096: 2.403e11
+    (1.75 m n (m + n))."""
+    memo = {}
+
+    def tri(d):
+        return d * (d - 1) // 2
+
+    def macs(mm, nn):
+        if mm == 1 and nn == 1:
+            return 0
+        key = (mm, nn)
+        if key in memo:
+            return memo[key]
+        if mm < nn:
+            h = nn // 2
+            upd = mm * h * (nn - h) + (0 if identity_b else tri(mm) * min(h, nn - h))
+            r = macs(mm, h) + macs(mm, nn - h) + upd
+        else:
+            h = mm // 2
+            upd = 0 if identity_b else (mm - h) * h * nn + tri(nn) * min(h, mm - h)
+            r = macs(h, nn) + macs(mm - h, nn) + upd
+        memo[key] = r
+        return r
+
+    return 2.0 * macs(int(m), int(n))
+
+
+def fp32_effective_peak(peaks) -> tuple:
+    """FP32-effective tensor rate of the 3xTF32 band products, TFLOP/s: the
+    measured bf16 burst rate halved (tf32 runs at half the bf16 rate) and
+    divided by the three MMAs of the split.  Burst, because a step is a few
+    milliseconds and the timed region well under a second."""
+    bf16 = float((peaks or {}).get("bf16_tflops", 1892.3))
+    return bf16 / 2.0 / 3.0, "of measured: bf16_tflops (burst) / 2 (tf32 rate) / 3 (3xTF32)"
+
+
+def host_info() -> dict:
+    """What the host oracle runs on: logical CPUs, CPU model, BLAS threads."""
+    import platform
+    info = {"os_cpu_count": os.cpu_count(), "machine": platform.machine()}
+    try:
+        for line in open("/proc/cpuinfo"):
+            low = line.lower()
+            if low.startswith("model name") or low.startswith("cpu part"):
+                info["cpu_model"] = line.split(":", 1)[1].strip()
+                break
+    except Exception:
+        pass
+    try:
+        import threadpoolctl
+        blas = [p for p in threadpoolctl.threadpool_info() if p.get("user_api") == "blas"]
+        if blas:
+            info["blas"] = blas[0].get("internal_api")
+            info["blas_threads"] = blas[0].get("num_threads")
+    except Exception:
+        for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+            if os.environ.get(var):
+                info["blas_threads"] = int(os.environ[var])
+                break
+        info.setdefault("blas_threads", "library default (all logical CPUs)")
+    return info
+
+
 def _csrc_hash():
     h = hashlib.sha256()
     for p in sorted(glob.glob(os.path.join(ROOT, "paper_2608_06291_gb300", "csrc", "*"))):
@@ -148,21 +218,38 @@ class ClockSampler:
 
 
 # ----------------------------------------------------------------- oracle legs
+def _grid_block(W64, bits, group, k):
+    """The full problem's grid restricted to the top-left k x k block: per-row
+    (or per-group) min-max over the whole rows, then the block's columns."""
+    import oracle as O
+    g = O.quant_grid(W64[:k], bits, group)
+    if group:
+        return O.Grid(g.s[:, :k // group], g.z[:, :k // group], g.qmax, group)
+    return g
+
+
 def _oracle_block(W64, f, bits, group, k):
-    """Time the float64 oracle (Alg. 4) on the top-left k x k block of the
-    workload: entry (i, j) depends only on entries up-left of it, so with the
-    full problem's factors restricted to the block this is an exact part of
-    the full solve."""
+    """Time the float64 oracle (Alg. 4, Alg. 3 on 64 x 64 blocks) on the
+    top-left k x k block of the workload: entry (i, j) depends only on entries
+    up-left of it, so with the full problem's factors and grid restricted to
+    the block this is an exact part of the full solve."""
     import oracle as O
     Wb = W64[:k, :k]
-    g = O.quant_grid(Wb, bits, group if group and k % group == 0 else 0)
+    g = _grid_block(W64, bits, group, k)
     c0 = os.times()
     t0 = time.perf_counter()
-    O.bakron_recursive(Wb, f.LA[:k, :k], f.LB[:k, :k], g)
+    O.bakron_recursive(Wb, f.LA[:k, :k], f.LB[:k, :k], g, base=64)
     wall = time.perf_counter() - t0
     c1 = os.times()
     cpu = (c1.user - c0.user) + (c1.system - c0.system)
     return wall, max(1, round(cpu / wall)) if wall > 0 else 1
+
+
+def _block_note(m, n, k):
+    """How the per-entry work of the k x k sample compares with the full m x n
+    problem (the oracle's time per entry grows with F_alg / (m n))."""
+    ratio = (f_alg(k, k) / (k * k)) / (f_alg(m, n) / (m * n))
+    return {"sample_entries": k * k, "per_entry_flops_ratio": ratio}
 
 
 def _timed(fn):
@@ -199,11 +286,14 @@ def extra_cpu_baseline(workload, data):
                 "sample": f"first {W.shape[0]} rows ({W.shape[0]} x {W.shape[1]}), l = 3, "
                           f"50 shrink steps, {wall:.2f} s wall"}
     W, LA, LB, bits = data["W"], data["LA"], data["LB"], data["bits"]
-    g = O.quant_grid(W, bits, 0)
-    wall, cores = _timed(lambda: O.bakron_recursive(W, LA, LB, g))
+    # the per-row grid of the full rows (data["rows"]), which the block's
+    # columns share: the block is then an exact part of the full solve
+    g = O.quant_grid(data["rows"], bits, 0)
+    wall, cores = _timed(lambda: O.bakron_recursive(W, LA, LB, g, base=64))
     return {"value": W.size / wall, "unit": "entries/s", "cores": cores, "kind": "oracle",
-            "sample": f"exact top-left {W.shape[0]} x {W.shape[1]} block, float64 Alg. 4, "
-                      f"{wall:.2f} s wall"}
+            "sample": f"exact top-left {W.shape[0]} x {W.shape[1]} block (grid from the full "
+                      f"rows), float64 Alg. 4 with Alg. 3 on 64 x 64 blocks, {wall:.2f} s wall",
+            "host": host_info()}
 
 
 def _oracle_factors(A, B, damp):
@@ -234,14 +324,16 @@ def run_reference(args):
     ms = 1e3 * sum(times) / len(times)
     value = k * k / (ms / 1e3)
     sample = (f"top-left {k}x{k} block of the {cfg.m}x{cfg.n} workload per step (exact "
-              f"sub-problem, full-problem factors), float64 Alg. 4 oracle")
+              f"sub-problem: full-problem factors and grid), float64 Alg. 4 oracle with Alg. 3 "
+              f"on 64 x 64 blocks")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": _config_dict(cfg),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                         "sample": sample},
+        "cpu_baseline": dict({"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                              "sample": sample, "host": host_info()},
+                             **_block_note(cfg.m, cfg.n, k)),
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
     return 0
@@ -366,10 +458,9 @@ def run_gpu(args):
     fam_fl = {k: v[2] / prof_steps for k, v in fam.items()}
 
     peaks = _peaks() or {}
-    f_alg = float(m) * n * (m + n)                    # flops of L^B E L^A^T (structural nonzeros)
+    F_alg = f_alg(m, n)
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
-    bf16_sus = float(peaks.get("bf16_tflops_sustained", 1700.0))
-    p_eff = bf16_sus * (1.1 / 2.25) / 3.0             # 3xTF32: tf32 rate (nominal ratio) / 3
+    p_eff, p_src = fp32_effective_peak(peaks)
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     fp32_simt_peak = 152 * 128 * 2 * sm_max * 1e6 / 1e12     # TFLOP/s, FFMA on CUDA cores
     groups = {
@@ -388,7 +479,7 @@ def run_gpu(args):
         roof = {"kernel": "k_tc_band: band products on tcgen05, 3xTF32 (stages 1 and 2)",
                 "bound": "tensor", "achieved": achieved, "peak": p_eff, "unit": "TFLOP/s",
                 "frac": achieved / p_eff,
-                "peak_source": "of measured: bf16_tflops_sustained x 1.1/2.25 (tf32/bf16) / 3",
+                "peak_source": p_src,
                 "algorithmic_per_step": g_work, "launches_per_step": g_n,
                 "traffic": _traffic("tc")}
     elif dom == "simt":
@@ -413,15 +504,17 @@ def run_gpu(args):
     roof["family_flops_per_step"] = fam_fl
     # whole-solve roofline: F_alg at the FP32-effective tensor rate plus the
     # leaves' bytes at HBM rate
-    t_roof = f_alg / (p_eff * 1e12) + 17.0 * m * n / (hbm * 1e9)
-    solve_roof = {"fp32_effective_tflops": p_eff, "f_alg_flops": f_alg,
+    t_roof = F_alg / (p_eff * 1e12) + 17.0 * m * n / (hbm * 1e9)
+    solve_roof = {"fp32_effective_tflops": p_eff, "f_alg_flops": F_alg,
+                  "leaf_bytes": 17.0 * m * n, "hbm_gbs": hbm,
                   "roofline_ms": 1e3 * t_roof, "frac": 1e3 * t_roof / ms,
-                  "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained x 1.1/2.25 / 3"}
+                  "peak_source": p_src,
+                  "formula": "(F_alg / P_fp32eff + 17 B/entry / BW_hbm) / t_solve"}
     # context: the library's own measurement of the instruction it issues
     # (tcgen05 kind::tf32, 128 x 128 x 8, operands resident, every SM)
     try:
         mr = P.bakron_diag_mma_rate(2000)
-        t_roof_mma = f_alg / (mr["fp32_effective_tflops"] * 1e12) + 17.0 * m * n / (hbm * 1e9)
+        t_roof_mma = F_alg / (mr["fp32_effective_tflops"] * 1e12) + 17.0 * m * n / (hbm * 1e9)
         solve_roof["measured_tf32_mma"] = {
             "tf32_tflops": mr["tf32_tflops"], "cycles_per_mma": mr["cycles_per_mma"],
             "fp32_effective_tflops": mr["fp32_effective_tflops"],
@@ -459,12 +552,15 @@ def run_gpu(args):
     if rank == 0 and not args.no_cpu_baseline:
         f = _oracle_factors(A, B, cfg.damp)
         W64 = W.double().cpu().numpy()
-        k = args.cpu_block
+        k = min(args.cpu_block, m, n)
         wall, cores = _oracle_block(W64, f, cfg.bits, cfg.group, k)
-        cpu_base = {"value": k * k / wall, "unit": UNIT, "cores": cores, "kind": "oracle",
-                    "sample": f"top-left {k}x{k} block of the {m}x{n} workload (exact "
-                              f"sub-problem with the full problem's factors), float64 Alg. 4 "
-                              f"oracle, {wall:.1f} s wall"}
+        cpu_base = dict({"value": k * k / wall, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"top-left {k}x{k} block of the {m}x{n} workload (exact "
+                                   f"sub-problem: the full problem's factors and grid), float64 "
+                                   f"Alg. 4 oracle with Alg. 3 on 64 x 64 blocks, {wall:.1f} s "
+                                   f"wall; the full problem does 1/per_entry_flops_ratio times "
+                                   f"the work per entry",
+                         "host": host_info()}, **_block_note(m, n, k))
 
     if rank == 0:
         vs = value / (4096 * 4096 / PAPER_4096_S) if (m, n) == (4096, 4096) else None
@@ -559,12 +655,10 @@ def run_extra(args):
         mma = None
         unit, metric = "entries/s", "GPTQ (BaKron with B = I), 4096x4096 bf16 W, 4-bit per row"
         per_launch = launches_per
-        bf16_sus = float(peaks.get("bf16_tflops_sustained", 1700.0))
-        p_eff = bf16_sus * (1.1 / 2.25) / 3.0
+        p_eff, roof_src = fp32_effective_peak(peaks)
         hbm = float(peaks.get("hbm_gbs", 6800.0))
-        f_alg = float(m) * n * (m + n)
+        F_alg = f_alg(m, n, identity_b=True)
         roof_peak = p_eff
-        roof_src = "of measured: bf16_tflops_sustained x 1.1/2.25 (tf32/bf16) / 3"
         cfg = {"workload": "gptq_b_identity", "m": m, "n": n, "bits": 4,
                "launch": "cuda graph replay", "paper_gptq_s_rtx_pro_6000": 0.025,
                "l2": "flushed (256 MiB write) between steps"}
@@ -573,7 +667,7 @@ def run_extra(args):
             f = _oracle_factors(A, torch.ones(1, 1), cfg2.damp)      # A's factor only
             b = 512
             return {"W": W[:b, :b].double().cpu().numpy(), "LA": f.LA[:b, :b],
-                    "LB": np.eye(b), "bits": cfg2.bits}
+                    "LB": np.eye(b), "bits": cfg2.bits, "rows": W[:b].double().cpu().numpy()}
     elif args.workload == "batched":
         cfg2 = WL.CONFIGS[2]
         W, A, _ = WL.make(cfg2, device=dev)
@@ -627,17 +721,15 @@ def run_extra(args):
         metric = ("per-head BaKron solves: 32 heads of 128x4096 (bf16, 4-bit), "
                   "16 lanes, entries/s")
         per_launch = launches_per
-        f_alg = Hh * float(mh) * n * (mh + n)
-        bf16_sus = float(peaks.get("bf16_tflops_sustained", 1700.0))
-        p_eff = bf16_sus * (1.1 / 2.25) / 3.0
+        F_alg = Hh * f_alg(mh, n)
+        p_eff, roof_src = fp32_effective_peak(peaks)
         hbm = float(peaks.get("hbm_gbs", 6800.0))
         roof_peak = p_eff
-        roof_src = "of measured: bf16_tflops_sustained x 1.1/2.25 (tf32/bf16) / 3"
         def cpu_data():
             f = _oracle_factors(A, Bs[0], cfg2.damp)                 # head 0's factors
             b = 512
             return {"W": W[:mh, :b].double().cpu().numpy(), "LA": f.LA[:b, :b], "LB": f.LB,
-                    "bits": cfg2.bits}
+                    "bits": cfg2.bits, "rows": W[:mh].double().cpu().numpy()}
         cfg = {"workload": "batched_heads", "heads": Hh, "m_head": mh, "n": n, "bits": 4,
                "lanes": lanes, "launch": "cuda graph replay",
                "one_lane_ms": one_lane_ms, "A": "shared (4096x4096 layer's)",
@@ -690,8 +782,8 @@ def run_extra(args):
     if args.workload == "gptq":
         if P.bakron_read_status(wsb) != 0:
             raise RuntimeError("device status set during the timed steps")
-        t_roof = f_alg / (p_eff * 1e12) + 17.0 * units / (hbm * 1e9)
-        roof = {"bound": "tensor", "achieved": f_alg / (ms / 1e3) / 1e12, "peak": p_eff,
+        t_roof = F_alg / (p_eff * 1e12) + 17.0 * units / (hbm * 1e9)
+        roof = {"bound": "tensor", "achieved": F_alg / (ms / 1e3) / 1e12, "peak": p_eff,
                 "unit": "TFLOP/s", "frac": 1e3 * t_roof / ms, "traffic": None,
                 "peak_source": roof_src, "roofline_ms": 1e3 * t_roof,
                 "note": "whole-solve roofline as for the general solve (the kernels do not "
@@ -699,8 +791,8 @@ def run_extra(args):
     elif args.workload == "batched":
         if P.lib().bakron_read_status_batched(wsS.data_ptr(), mh, n, lanes, None) != 0:
             raise RuntimeError("device status set during the timed steps")
-        t_roof = f_alg / (p_eff * 1e12) + 17.0 * units / (hbm * 1e9)
-        roof = {"bound": "tensor", "achieved": f_alg / (ms / 1e3) / 1e12, "peak": p_eff,
+        t_roof = F_alg / (p_eff * 1e12) + 17.0 * units / (hbm * 1e9)
+        roof = {"bound": "tensor", "achieved": F_alg / (ms / 1e3) / 1e12, "peak": p_eff,
                 "unit": "TFLOP/s", "frac": 1e3 * t_roof / ms, "traffic": None,
                 "peak_source": roof_src, "roofline_ms": 1e3 * t_roof,
                 "note": "whole-call roofline: sum over heads of F_alg at the FP32-effective "
@@ -733,9 +825,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=2)
-    ap.add_argument("--cpu-block", type=int, default=1024,
+    ap.add_argument("--cpu-block", type=int, default=2048,
                     help="side of the top-left block the cpu_baseline oracle solves")
-    ap.add_argument("--ref-block", type=int, default=256,
+    ap.add_argument("--ref-block", type=int, default=1024,
                     help="side of the top-left block each reference-arm step solves")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-autotune", action="store_true",

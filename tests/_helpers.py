@@ -29,3 +29,13 @@ def compare_codes(W64, codes_gpu, g, LA64, LB64, ref_codes=None):
     if ref_codes is not None:
         out["raw_match"] = float((ref_codes == codes_gpu).mean())
     return out
+
+
+def root_mismatches(bad: np.ndarray) -> np.ndarray:
+    """Mismatches with no mismatch up-left of them (i <= p, j <= q, (i, j) !=
+    (p, q)): the entries where two solves first part."""
+    seen = np.maximum.accumulate(np.maximum.accumulate(bad, axis=0), axis=1)
+    before = np.zeros_like(bad)
+    before[1:, :] |= seen[:-1, :]
+    before[:, 1:] |= seen[:, :-1]
+    return bad & ~before

@@ -10,7 +10,8 @@ in fp64 from W, A and B alone, the value every entry must be rounded at given
 the codes before it (canonical definition of the equivalence proof), and
 every GPU code must equal that value's rounding unless the value lies within
 1e-4 grid units of a rounding boundary.  Configs 2-4 are checked on every
-row; config 5 on its first 256 and last 64 rows.
+row; config 5 on its first 256 rows, 256 rows from the middle of B's factor
+(14336..14591) and its last 64 rows.
 """
 import numpy as np
 import pytest
@@ -92,4 +93,4 @@ def test_config_certificate_full(c):
 def test_config5_certificate_sampled_rows():
     r = _run(5)
     m = r["cfg"].m
-    _check(r, rows=[np.arange(256), np.arange(m - 64, m)])
+    _check(r, rows=[np.arange(256), np.arange(m // 2, m // 2 + 256), np.arange(m - 64, m)])

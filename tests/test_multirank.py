@@ -79,7 +79,7 @@ def test_extra_lines_cpu_baseline_on_small_samples():
     f = bench._oracle_factors(A, B, 0.01)
     for wl in ("batched", "gptq"):
         r = bench.extra_cpu_baseline(wl, {"W": W.double().numpy(), "LA": f.LA, "LB": f.LB,
-                                          "bits": 4})
+                                          "bits": 4, "rows": W.double().numpy()})
         assert r["unit"] == "entries/s" and r["value"] > 0 and r["cores"] >= 1
     fa = bench._oracle_factors(A, torch.ones(1, 1), 0.01)           # A's factor alone
     np.testing.assert_allclose(fa.LA, f.LA, rtol=1e-12, atol=1e-14)
