@@ -445,17 +445,32 @@ def run_gpu(args):
         raise RuntimeError("device status set during the timed steps")
     value = whole_job_rate(m * n, ws_n, ms)
 
-    # per-family device time, live, with events on the launch stream
-    P.bakron_profile_enable(True)
+    # per-family device time of the step as it is timed: the solve captured
+    # once more with the library's timeline stamps (no events between the
+    # launches, so the programmatic overlap stays) and replayed; each replay's
+    # launches partition its device time
+    P.bakron_profile_enable(2)
+    if graph is not None:
+        pgraph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(pgraph):
+            eager_step()
+        prof_step = pgraph.replay
+    else:
+        prof_step = eager_step
     prof_steps = max(3, min(args.steps, 10))
     for i in range(prof_steps):
         flush.fill_(i & 0xFF)
-        eager_step()
+        prof_step()
+        P.bakron_profile_collect()
     fam = P.bakron_profile_read()
+    nrep, span_ms = P.bakron_profile_timeline()
     P.bakron_profile_enable(False)
+    if P.bakron_read_status(work) != 0:
+        raise RuntimeError("device status set during the profiling replays")
     fam_ms = {k: v[1] / prof_steps for k, v in fam.items()}
     fam_n = {k: v[0] // prof_steps for k, v in fam.items()}
     fam_fl = {k: v[2] / prof_steps for k, v in fam.items()}
+    timeline_ms = span_ms / max(1, nrep)
 
     peaks = _peaks() or {}
     F_alg = f_alg(m, n)
@@ -472,17 +487,41 @@ def run_gpu(args):
         "leaf": (fam_ms["leaf"] + fam_ms["subtree"], 17.0 * m * n,
                  fam_n["leaf"] + fam_n["subtree"]),
     }
+    # the band products against the FP32-effective tensor rate (tile products
+    # in the band, 2 * 32^3 flops each)
+    tc_ms, tc_work, tc_n = groups["tc"]
+    tc_roof = None
+    if tc_ms > 0:
+        tc_ach = tc_work / (tc_ms / 1e3) / 1e12
+        tc_roof = {"kernel": "k_tc_band: band products on tcgen05, 3xTF32 (stages 1 and 2)",
+                   "bound": "tensor", "achieved": tc_ach, "peak": p_eff, "unit": "TFLOP/s",
+                   "frac": tc_ach / p_eff, "peak_source": p_src,
+                   "algorithmic_per_step": tc_work, "launches_per_step": tc_n,
+                   "ms_per_step": tc_ms, "traffic": _traffic("tc")}
+    # the leaves against their latency floor: the element anti-diagonals
+    # (m + n - 1 dependent rounding steps, Sec. 3.3) at the chain's own
+    # measured step time, one tile alone on the GPU
+    leaf_ms, leaf_bytes, leaf_n = groups["leaf"]
+    cyc = P.bakron_diag_leaf_chain()
+    mhz = float((clocks or {}).get("sm_mhz") or sm_max)
+    step_ns = cyc / mhz * 1e3
+    floor_ms = (m + n - 1) * step_ns * 1e-6
+    tile_steps = leaf_n * (2 * TILE - 1)
+    leaf_roof = {"kernel": "k_leaf: 32 x 32 tiles, one CTA each, wavefront of 63 in-tile steps",
+                 "bound": "latency", "achieved": (m + n - 1) / (leaf_ms / 1e3),
+                 "peak": 1e9 / step_ns, "unit": "element anti-diagonals/s",
+                 "frac": floor_ms / leaf_ms if leaf_ms > 0 else None,
+                 "peak_source": f"measured: bakron_diag_leaf_chain {cyc:.1f} cycles per chain "
+                                f"step at the sampled {mhz:.0f} MHz",
+                 "floor_ms": floor_ms, "ms_per_step": leaf_ms, "launches_per_step": leaf_n,
+                 "schedule_chain_steps": tile_steps,
+                 "hbm_gbs": leaf_bytes / (leaf_ms / 1e3) / 1e9 if leaf_ms > 0 else None,
+                 "traffic": _traffic("leaf")}
     dom = max(groups, key=lambda g: groups[g][0])
-    g_ms, g_work, g_n = groups[dom]
     if dom == "tc":
-        achieved = g_work / (g_ms / 1e3) / 1e12
-        roof = {"kernel": "k_tc_band: band products on tcgen05, 3xTF32 (stages 1 and 2)",
-                "bound": "tensor", "achieved": achieved, "peak": p_eff, "unit": "TFLOP/s",
-                "frac": achieved / p_eff,
-                "peak_source": p_src,
-                "algorithmic_per_step": g_work, "launches_per_step": g_n,
-                "traffic": _traffic("tc")}
+        roof = dict(tc_roof)
     elif dom == "simt":
+        g_ms, g_work, g_n = groups["simt"]
         achieved = g_work / (g_ms / 1e3) / 1e12
         roof = {"kernel": "k_band1_simt/k_band2_simt/k_band_fused_simt: narrow band products",
                 "bound": "alu", "achieved": achieved, "peak": fp32_simt_peak, "unit": "TFLOP/s",
@@ -491,13 +530,10 @@ def run_gpu(args):
                 "algorithmic_per_step": g_work, "launches_per_step": g_n,
                 "traffic": _traffic("simt")}
     else:
-        achieved = g_work / (g_ms / 1e3) / 1e9
-        roof = {"kernel": "k_leaf / k_subtree: anti-diagonal wavefront of 32x32 tiles "
-                          "(k_subtree: persistent launches of the narrow ranges, leaves plus "
-                          "their band products)", "bound": "hbm",
-                "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                "peak_source": "of measured: hbm_gbs", "algorithmic_per_step": g_work,
-                "launches_per_step": g_n, "traffic": _traffic("leaf")}
+        roof = dict(leaf_roof)
+    roof["timing"] = ("family times partition the graph-replayed step (timeline stamps, "
+                      f"{prof_steps} replays)")
+    roof["timeline_ms_per_step"] = timeline_ms
     roof["groups_ms_per_step"] = {k: v[0] for k, v in groups.items()}
     roof["family_ms_per_step"] = fam_ms
     roof["family_launches_per_step"] = fam_n
@@ -505,7 +541,8 @@ def run_gpu(args):
     # whole-solve roofline: F_alg at the FP32-effective tensor rate plus the
     # leaves' bytes at HBM rate
     t_roof = F_alg / (p_eff * 1e12) + 17.0 * m * n / (hbm * 1e9)
-    solve_roof = {"fp32_effective_tflops": p_eff, "f_alg_flops": F_alg,
+    solve_roof = {"tc_roofline": tc_roof, "leaf_roofline": leaf_roof,
+                  "fp32_effective_tflops": p_eff, "f_alg_flops": F_alg,
                   "leaf_bytes": 17.0 * m * n, "hbm_gbs": hbm,
                   "roofline_ms": 1e3 * t_roof, "frac": 1e3 * t_roof / ms,
                   "peak_source": p_src,

@@ -354,25 +354,40 @@ int bakron_read_status(void* workspace, void* stream);
 
 /*
  * Instrumentation for benchmarks (no counterpart in the paper).
- * bakron_profile_enable(1) makes every later bakron_solve bracket each of its
- * kernel launches with CUDA events on `stream` and accumulate, per kernel
- * family, the number of launches, their device time and their algorithmic
- * floating-point work.  Families:
+ * bakron_profile_enable(1) (event mode) makes every later bakron_solve
+ * bracket each of its kernel launches with CUDA events on `stream` and
+ * accumulate, per kernel family, the number of launches, their device time
+ * and their algorithmic floating-point work.  The events serialise the
+ * launches, so these times add up to more than a solve takes.
+ * bakron_profile_enable(2) (timeline mode) instead has every kernel of a
+ * solve stamp, on the device, when its CTAs start their dependent work and
+ * when the last one ends (global nanosecond timer), with no events between
+ * the launches.  The launch sequence of the last bakron_solve enqueued (for
+ * example while a CUDA graph of it is captured) is recorded; after each run
+ * of that sequence (a graph replay), bakron_profile_collect(stream)
+ * synchronises `stream`, turns the stamps into a partition of the run's
+ * device time -- launch i owns the time from the end of launch i - 1 to its
+ * own end -- adds it to the family totals and clears the stamps.  Timeline
+ * mode allocates its stamp buffer (512 KiB) at the first enable(2).  It
+ * records one solve at a time (a batched solve's heads overwrite each other).
+ * Families:
  *   0 grid + workspace init, 1 leaf wavefront (2*32^3 flops per tile),
  *   2 / 3 band product stage 1 (M = L^B E) / stage 2 (X += M L^A^T) on CUDA
  *   cores, 4 output copy, 5 / 6 stage 1 / stage 2 on the tensor cores,
  *   7 both stages of a narrow node fused in one launch on CUDA cores,
  *   8 one persistent launch running a narrow range of the recursion (its
- *   leaves and band products, separated by grid-wide barriers).
+ *   leaves and band products, separated by grid-wide barriers; not stamped).
  *   A band stage counts 2*32^3 flops per 32x32 tile product it must form
  *   (tile pairs inside the band, triangular diagonal blocks counted whole).
  * bakron_profile_read synchronises the device, then returns the totals since
  * the last bakron_profile_enable (launches, milliseconds, flops; `flops` may
- * be NULL).
+ * be NULL); family -1 returns, in timeline mode, the number of collected runs
+ * and the sum of their spans (first start to last end).
  * bakron_last_launches returns the number of kernels the last bakron_solve
  * call on this host thread enqueued.
  */
 int bakron_profile_enable(int on);
+int bakron_profile_collect(void* stream);
 int bakron_profile_read(int family, int* launches, double* ms, double* flops);
 int bakron_last_launches(void);
 
@@ -399,6 +414,20 @@ int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C, int M,
  */
 int bakron_diag_mma_rate(int stages, void* workspace, size_t workspace_bytes,
                          double* tflops, double* cycles_per_mma, void* stream);
+
+/*
+ * Diagnostic (no counterpart in the paper): the cycles one step of the leaf's
+ * dependent chain takes, alone on the GPU.  Solves the 32 x 32 problem W
+ * (device, row stride 32, fp32 or bf16) with `factors` (a factor buffer of a
+ * 32 x 32 problem) as one leaf tile (4-bit grid into codes, scales, zeros),
+ * and returns in *cycles_per_step the chain warp's clock64 cycles over its
+ * 63 in-tile steps divided by 63.  workspace >= bakron_workspace_bytes(32,
+ * 32) + 256 bytes.  Synchronous; returns the device status.
+ */
+int bakron_diag_leaf_chain(const void* W, int wdtype, const void* factors,
+                           uint8_t* codes, float* scales, float* zeros,
+                           void* workspace, size_t workspace_bytes,
+                           double* cycles_per_step, void* stream);
 
 /* Static description of a status code. */
 const char* bakron_strerror(int status);

@@ -79,6 +79,11 @@ def lib() -> ctypes.CDLL:
     L.bakron_read_status.restype = i32
     L.bakron_profile_enable.argtypes = [i32]
     L.bakron_profile_enable.restype = i32
+    L.bakron_profile_collect.argtypes = [vp]
+    L.bakron_profile_collect.restype = i32
+    L.bakron_diag_leaf_chain.argtypes = [vp, i32, vp, vp, vp, vp, vp, ctypes.c_size_t,
+                                         ctypes.POINTER(ctypes.c_double), vp]
+    L.bakron_diag_leaf_chain.restype = i32
     L.bakron_profile_read.argtypes = [i32, ctypes.POINTER(i32), ctypes.POINTER(ctypes.c_double),
                                       ctypes.POINTER(ctypes.c_double)]
     L.bakron_profile_read.restype = i32
@@ -459,8 +464,24 @@ def bakron_read_status_noalloc(stream=None) -> int:
 PROFILE_FAMILIES = ("init", "leaf", "band1", "band2", "copy", "tc1", "tc2", "fused", "subtree")
 
 
-def bakron_profile_enable(on: bool = True) -> None:
-    _check(lib().bakron_profile_enable(1 if on else 0), "bakron_profile_enable")
+def bakron_profile_enable(on=True) -> None:
+    """on: False (off), True or 1 (event mode), 2 (timeline mode)."""
+    mode = 2 if on == 2 else (1 if on else 0)
+    _check(lib().bakron_profile_enable(mode), "bakron_profile_enable")
+
+
+def bakron_profile_collect(stream=None) -> None:
+    """Timeline mode: fold the stamps of the last run of the recorded solve
+    (e.g. one graph replay) into the family totals."""
+    _check(lib().bakron_profile_collect(_stream(stream)), "bakron_profile_collect")
+
+
+def bakron_profile_timeline() -> tuple:
+    """Timeline mode: (runs collected, summed span of those runs in ms)."""
+    n, ms = ctypes.c_int(0), ctypes.c_double(0.0)
+    _check(lib().bakron_profile_read(-1, ctypes.byref(n), ctypes.byref(ms), None),
+           "bakron_profile_read")
+    return n.value, ms.value
 
 
 def bakron_profile_read() -> dict:
@@ -474,6 +495,23 @@ def bakron_profile_read() -> dict:
                "bakron_profile_read")
         out[name] = (n.value, ms.value, fl.value)
     return out
+
+
+def bakron_diag_leaf_chain(seed: int = 0, device=None) -> float:
+    """Cycles of one step of the leaf's dependent chain, one tile alone on the
+    GPU (a random 32 x 32 problem with identity factors)."""
+    dev = device or torch.device("cuda")
+    g = torch.Generator(device=dev).manual_seed(seed)
+    W = 0.02 * torch.randn(32, 32, generator=g, device=dev)
+    f = bakron_set_factors(torch.eye(32, device=dev), torch.eye(32, device=dev))
+    codes = torch.empty(32, 32, dtype=torch.uint8, device=dev)
+    sz = torch.empty(2, 32, 1, dtype=torch.float32, device=dev)
+    ws = torch.empty(workspace_bytes(32, 32) + 256, dtype=torch.uint8, device=dev)
+    cyc = ctypes.c_double(0.0)
+    _check(lib().bakron_diag_leaf_chain(_ptr(W), F32, _ptr(f.buf), _ptr(codes), _ptr(sz[0]),
+                                        _ptr(sz[1]), _ptr(ws), ws.numel(), ctypes.byref(cyc),
+                                        _stream(None)), "bakron_diag_leaf_chain")
+    return cyc.value
 
 
 def bakron_last_launches() -> int:

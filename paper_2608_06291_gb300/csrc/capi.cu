@@ -4,6 +4,8 @@
 #include <stdint.h>
 #include <stdlib.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "tune.cuh"
 #include "solve.cuh"
@@ -168,6 +170,31 @@ int bakron_read_status(void* workspace, void* stream) {
   BK_CUDA_OK(cudaMemsetAsync(workspace, 0, sizeof(int), s));
   BK_CUDA_OK(cudaGetLastError());
   return h;
+}
+
+int bakron_diag_leaf_chain(const void* W, int wdtype, const void* factors, uint8_t* codes,
+                           float* scales, float* zeros, void* workspace, size_t workspace_bytes,
+                           double* cycles_per_step, void* stream) {
+  if (!W || !factors || !codes || !scales || !zeros || !workspace || !cycles_per_step)
+    return BAKRON_ERR_INVALID_ARG;
+  if (wdtype != BAKRON_F32 && wdtype != BAKRON_BF16) return BAKRON_ERR_INVALID_ARG;
+  const size_t need = SolveLayout(TILE, TILE).bytes;
+  if (workspace_bytes < need + 256) return BAKRON_ERR_WORKSPACE;
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lk(mu);
+  cudaStream_t s = (cudaStream_t)stream;
+  long long* clk = (long long*)((char*)workspace + need);
+  BK_CUDA_OK(cudaMemsetAsync(clk, 0, 2 * sizeof(long long), s));
+  g_diag_leaf_clk = clk;
+  const int rc = solve_impl(W, wdtype, TILE, TILE, TILE, factors, 15, 0, codes, scales, zeros,
+                            nullptr, workspace, s, nullptr, false, false);
+  g_diag_leaf_clk = nullptr;
+  if (rc != BAKRON_OK) return rc;
+  long long h[2] = {0, 0};
+  BK_CUDA_OK(cudaMemcpyAsync(h, clk, sizeof(h), cudaMemcpyDeviceToHost, s));
+  BK_CUDA_OK(cudaStreamSynchronize(s));
+  *cycles_per_step = (double)(h[1] - h[0]) / (2 * TILE - 1);
+  return bakron_read_status(workspace, stream);
 }
 
 const char* bakron_strerror(int status) {

@@ -148,6 +148,23 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
+// Timeline stamps of one kernel launch (benchmark instrumentation; kernels
+// receive a null slot unless bakron_profile_enable(2) is on): slot[0] takes
+// the earliest time a CTA of the launch started its dependent work (after its
+// pdl_wait), slot[1] the latest time a CTA finished, in %globaltimer
+// nanoseconds.  Thread 0 of each CTA stamps.
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void stamp_begin(unsigned long long* slot) {
+  if (slot != nullptr && threadIdx.x == 0) atomicMin(slot, global_ns());
+}
+__device__ __forceinline__ void stamp_end(unsigned long long* slot) {
+  if (slot != nullptr && threadIdx.x == 0) atomicMax(slot + 1, global_ns());
+}
+
 // Device status word (first int of every workspace).  Kernels only ever raise
 // it with atomicMax-free writes of a nonzero code; the host reads and clears.
 __device__ inline void raise_status(int* status, int code) {

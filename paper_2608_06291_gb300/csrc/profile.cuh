@@ -17,8 +17,11 @@ enum {
   kFamilies = 9
 };
 
-// Counts one kernel launch; when profiling is on, records an event on the
-// stream at construction and another at destruction (wrap exactly one launch).
+// Counts one kernel launch.  Event mode (bakron_profile_enable(1)): records
+// an event on the stream at construction and another at destruction (wrap
+// exactly one launch).  Timeline mode (bakron_profile_enable(2)): takes the
+// next stamp slot of the current solve, which the launch passes to its kernel
+// (stamp(); null in the other modes).
 class LaunchScope {
  public:
   // `flops`: algorithmic floating-point work of the launch (0 if not tracked)
@@ -26,15 +29,17 @@ class LaunchScope {
   ~LaunchScope();
   LaunchScope(const LaunchScope&) = delete;
   LaunchScope& operator=(const LaunchScope&) = delete;
+  unsigned long long* stamp() const { return stamp_; }
 
  private:
   int family_;
   cudaStream_t s_;
   void* a_;
   double flops_;
+  unsigned long long* stamp_;
 };
 
-void reset_launch_count();
+void reset_launch_count();    // also starts a new solve's stamp slots
 int launch_count();            // kernels enqueued on this host thread since the reset
 void set_launch_count(int n);
 bool profiling_on();

@@ -36,9 +36,10 @@ namespace bakron {
 // ([-1, 1] if both are 0), s = (xmax - xmin) / qmax, z = rint(-xmin / s),
 // all in IEEE fp32 so the scales equal the oracle's bit for bit.
 __global__ void k_grid(const void* W, int wdt, int m, int n, int64_t ldw, int gsz, int G,
-                       int qmax, float* scales, float* zeros) {
+                       int qmax, float* scales, float* zeros, unsigned long long* stamp) {
   const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
+  stamp_begin(stamp);
   if (warp >= (int64_t)m * G) return;
   const int row = (int)(warp / G), grp = (int)(warp % G);
   const int c0 = grp * gsz, c1 = c0 + gsz;
@@ -61,6 +62,7 @@ __global__ void k_grid(const void* W, int wdt, int m, int n, int64_t ldw, int gs
     scales[(int64_t)row * G + grp] = s;
     zeros[(int64_t)row * G + grp] = rintf(__fdiv_rn(-xmin, s));
   }
+  stamp_end(stamp);
 }
 
 // Symmetric alphabet {-l, ..., +l} of the paper's experiments (Appendix
@@ -147,9 +149,10 @@ int launch_grid_sym(const void* W, int wdt, int m, int n, int64_t ldw, int level
 // Grid-stride over chunks of 8 entries of a row (np is a multiple of 128, so
 // a chunk never straddles a row), stored as two 16-byte vectors.
 __global__ void k_init(const void* W, int wdt, int m, int n, int64_t ldw, float* X,
-                       int64_t mp, int64_t np) {
+                       int64_t mp, int64_t np, unsigned long long* stamp) {
   pdl_wait();
   pdl_trigger();
+  stamp_begin(stamp);
   const int64_t chunks = mp * np / 8;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < chunks;
        i += (int64_t)gridDim.x * blockDim.x) {
@@ -167,6 +170,7 @@ __global__ void k_init(const void* W, int wdt, int m, int n, int64_t ldw, float*
     o[0] = make_float4(v[0], v[1], v[2], v[3]);
     o[1] = make_float4(v[4], v[5], v[6], v[7]);
   }
+  stamp_end(stamp);
 }
 
 __global__ void k_copy_out(const float* X, int64_t np, int m, int n, float* out) {
@@ -271,6 +275,8 @@ struct LeafArgs {
   int G, gsz, qmax;
   uint8_t* codes;
   int* status;
+  unsigned long long* stamp;   // timeline stamp slot of the launch (null: none)
+  long long* clk;              // diagnostic: the chain's clock64 around its steps (null: none)
 };
 
 constexpr int KM = 36;   // row stride of k-major product operands: float4 rows
@@ -493,6 +499,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     pdl_wait();
     pdl_trigger();
   }
+  stamp_begin(a.stamp);
   // X at this thread's product positions: rows pr .. pr+3, columns pc, pc+1
   float xv[4][2];
 #pragma unroll
@@ -599,6 +606,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     float4 g0 = S.Srzl[(0 - q) & (TILE - 1)][q], g1 = S.Srzl[(1 - q) & (TILE - 1)][q];
     float4 lb0 = S.Lsub[(0 - q) & (TILE - 1)], lb1 = S.Lsub[(1 - q) & (TILE - 1)];
     leaf_sync();   // the helpers' pre of steps 0 and 1
+    if (a.clk != nullptr && lane == 0) a.clk[0] = clock64();
 #pragma unroll 1
     for (int k = 0; k < TILE; ++k) {
       const int d0 = 2 * k, d1 = 2 * k + 1;
@@ -617,6 +625,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
       if (d1 < 2 * TILE - 1) step(d1, true, pre1, g1c, lb1c);
       leaf_sync();
     }
+    if (a.clk != nullptr && lane == 0) a.clk[1] = clock64();
   } else {
     // ------------------------------------------------ helpers: rows i0..i0+11
     const int g = w - 1, i0 = LEAF_ROWS_PER_HELPER * g;
@@ -740,6 +749,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
   }
   if (bad) raise_status(a.status, BAKRON_ERR_NONFINITE);
   leaf_sync();   // shared memory free for the next tile of this CTA
+  stamp_end(a.stamp);
 }
 
 // leaf_tile<false, P> for a window known at run time (0 <= h <= LEAF_WINDOW)
@@ -834,6 +844,7 @@ struct BandArgs {
   int64_t ldm;
   float* X;
   int64_t ldx;
+  unsigned long long* stamp;   // timeline stamp slot of the launch (null: none)
 };
 
 // Unit (x, y) of stage 1: M tile (I, J') with I = row_lo + y, J' = max(0, k - I) + x.
@@ -984,25 +995,31 @@ __device__ __forceinline__ void fused_unit(const Band& bd, const BandArgs& a, in
 __global__ void __launch_bounds__(SIMT_THREADS) k_band1_simt(Band bd, BandArgs a) {
   pdl_wait();
   pdl_trigger();
+  stamp_begin(a.stamp);
   __shared__ BandSmem S;
   int I, Jp;
   if (band1_index(bd, blockIdx.x, blockIdx.y, I, Jp)) band1_unit(bd, a, I, Jp, S);
+  stamp_end(a.stamp);
 }
 
 __global__ void __launch_bounds__(SIMT_THREADS) k_band2_simt(Band bd, BandArgs a) {
   pdl_wait();
   pdl_trigger();
+  stamp_begin(a.stamp);
   __shared__ BandSmem S;
   int I, J;
   if (band2_index(bd, blockIdx.x, blockIdx.y, I, J)) band2_unit(bd, a, I, J, S);
+  stamp_end(a.stamp);
 }
 
 __global__ void __launch_bounds__(SIMT_THREADS) k_band_fused_simt(Band bd, BandArgs a) {
   pdl_wait();
   pdl_trigger();
+  stamp_begin(a.stamp);
   __shared__ BandSmem S;
   int I, J;
   if (band2_index(bd, blockIdx.x, blockIdx.y, I, J)) fused_unit(bd, a, I, J, S);
+  stamp_end(a.stamp);
 }
 
 // ------------------------------------------------- persistent subtree
@@ -1201,7 +1218,9 @@ static void leaf(SolveArgs& a, int K, int window) {
                  2.0 * TILE * TILE * TILE * (1 + window_products(window)) * (ihi - ilo + 1));
   const dim3 grid(ihi - ilo + 1), block(LEAF_THREADS);
   const size_t sm = sizeof(LeafSmem);
-  note(a, launch_leaf_window(window, grid, block, sm, a.s, K, a.la));
+  LeafArgs la = a.la;
+  la.stamp = ls.stamp();
+  note(a, launch_leaf_window(window, grid, block, sm, a.s, K, la));
 }
 
 // Dynamic shared memory of the leaf and subtree kernels above the 48 KB
@@ -1226,12 +1245,12 @@ static void band(SolveArgs& a, int k, int h, int l) {
   if (a.tc_ready && l - k >= a.tc_min_band) {
     {
       LaunchScope ls(kFamTc1, a.s, f * p1);
-      int rc = tc_band_stage(1, a.tcm, a.tco, k, h, l, a.s);
+      int rc = tc_band_stage(1, a.tcm, a.tco, k, h, l, a.s, ls.stamp());
       if (rc != BAKRON_OK) a.rc = rc;
     }
     {
       LaunchScope ls(kFamTc2, a.s, f * p2);
-      int rc = tc_band_stage(2, a.tcm, a.tco, k, h, l, a.s);
+      int rc = tc_band_stage(2, a.tcm, a.tco, k, h, l, a.s, ls.stamp());
       if (rc != BAKRON_OK) a.rc = rc;
     }
     return;
@@ -1242,18 +1261,22 @@ static void band(SolveArgs& a, int k, int h, int l) {
   Band bd{k, h, l, a.Mt, a.Nt, row_lo};
   // J' span per row <= min(h, l - k); output J span <= l - h
   dim3 g1(min(h, l - k), row_hi - row_lo + 1), g2(l - h, row_hi - row_lo + 1);
+  BandArgs ba = a.ba;
   if (l - k <= a.fused_max_band) {
     LaunchScope ls(kFamFused, a.s, f * (p1 + p2));
-    note(a, launch_pdl(k_band_fused_simt, g2, dim3(SIMT_THREADS), 0, a.s, bd, a.ba));
+    ba.stamp = ls.stamp();
+    note(a, launch_pdl(k_band_fused_simt, g2, dim3(SIMT_THREADS), 0, a.s, bd, ba));
     return;
   }
   {
     LaunchScope ls(kFamBand1, a.s, f * p1);
-    note(a, launch_pdl(k_band1_simt, g1, dim3(SIMT_THREADS), 0, a.s, bd, a.ba));
+    ba.stamp = ls.stamp();
+    note(a, launch_pdl(k_band1_simt, g1, dim3(SIMT_THREADS), 0, a.s, bd, ba));
   }
   {
     LaunchScope ls(kFamBand2, a.s, f * p2);
-    note(a, launch_pdl(k_band2_simt, g2, dim3(SIMT_THREADS), 0, a.s, bd, a.ba));
+    ba.stamp = ls.stamp();
+    note(a, launch_pdl(k_band2_simt, g2, dim3(SIMT_THREADS), 0, a.s, bd, ba));
   }
 }
 
@@ -1335,6 +1358,10 @@ static void rec(SolveArgs& a, int k, int l) {
   rec(a, h, l);
 }
 
+// Diagnostic only (bakron_diag_leaf_chain): where the leaves of the next
+// solve record the chain's clock64 before and after its steps.
+long long* g_diag_leaf_clk = nullptr;
+
 // `force`: thresholds to use instead of tuning_for(m, n) (the autotuner's candidates).
 // `grid_given`: scales and zeros hold the caller's grid (read only); otherwise
 // the min-max grid over qmax + 1 codes is computed into them first.
@@ -1372,9 +1399,10 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
   // the leaves' fp32 E^T and final G share the M planes (see SolveLayout)
   a.la = LeafArgs{a.Mt, a.Nt, m, n, a.X, a.np, a.EtH, a.EtL, a.MH, a.ML, a.mp,
                   (const float*)(f + fl.off_LBblk), (const float*)(f + fl.off_LAblk),
-                  scales, zeros, a.G, a.gsz, a.qmax, codes, a.status};
+                  scales, zeros, a.G, a.gsz, a.qmax, codes, a.status, nullptr,
+                  g_diag_leaf_clk};
   a.ba = BandArgs{a.LBH, a.LBL, a.mp, a.EtH, a.EtL, a.mp, a.LAH, a.LAL, a.np,
-                  a.MH, a.ML, a.np, a.X, a.np};
+                  a.MH, a.ML, a.np, a.X, a.np, nullptr};
   a.profiling = profiling_on();
   {
     if (ensure_leaf_attrs() != cudaSuccess) return BAKRON_ERR_CUDA;
@@ -1408,14 +1436,15 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
     const int64_t warps = (int64_t)m * a.G;
     LaunchScope ls(kFamInit, s);
     k_grid<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(W, wdt, m, n, ldw, a.gsz, a.G,
-                                                                 a.qmax, scales, zeros);
+                                                                 a.qmax, scales, zeros,
+                                                                 ls.stamp());
   }
   {
     const int64_t chunks = a.mp * a.np / 8;
     LaunchScope ls(kFamInit, s);
     const unsigned blocks = (unsigned)std::min<int64_t>((chunks + 255) / 256, 152 * 8);
     note(a, launch_pdl(k_init, dim3(blocks), dim3(256), 0, s, W, wdt, m, n, ldw, a.X, a.mp,
-                       a.np));
+                       a.np, ls.stamp()));
   }
   rec(a, 0, a.Mt + a.Nt - 1);
   if (prerounding) {

@@ -20,4 +20,8 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
                void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
                bool keep_status);
 
+// Diagnostic only (bakron_diag_leaf_chain): when set, the leaves of the next
+// solve record the chain warp's clock64 before and after its 63 steps there.
+extern long long* g_diag_leaf_clk;
+
 }  // namespace bakron

@@ -84,6 +84,7 @@ struct TcParams {
   float alpha, beta;
   int dreal;
   int a_exact, b_exact;
+  unsigned long long* stamp;   // timeline stamp slot of the launch (null: none)
 };
 
 // Kernel variants (compile time, so that the band products' issue loop
@@ -428,6 +429,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   // the rest waits for the previous kernel
   pdl_wait();
   pdl_trigger();
+  stamp_begin(P.stamp);
   const long long drain = 4000000000LL;   // ~2 s at 2 GHz: wind-down bound
   const int nk = blk.nk;
   constexpr int kgroup = V == V_GRAM_BF16 ? GRAM_KGROUP : 1;
@@ -706,6 +708,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
+  stamp_end(P.stamp);
   if (warp == 1) {
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                  "r"(TMEM_COLS)
@@ -936,9 +939,10 @@ bool tc_band_maps(TcMaps& maps, const TcOperands& op) {
 }
 
 int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, int h, int l,
-                  cudaStream_t s) {
+                  cudaStream_t s, unsigned long long* stamp) {
   if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
   TcParams P{};
+  P.stamp = stamp;
   P.mode = stage == 1 ? MODE_STAGE1 : MODE_STAGE2;
   P.k = k; P.h = h; P.l = l;
   P.Mt = op.Mt; P.Nt = op.Nt;

@@ -31,7 +31,8 @@ long long spin_cycles_from_env();
 
 // Stage 1 (M = L^B E on the band [k, h)) or stage 2 (X += M L^A^T on the
 // band [h, l)) of one Alg. 5 node, over 128 x 128 output blocks.
+// `stamp`: the launch's timeline stamp slot (null: none).
 int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, int h, int l,
-                  cudaStream_t s);
+                  cudaStream_t s, unsigned long long* stamp = nullptr);
 
 }  // namespace bakron
