@@ -629,7 +629,8 @@ def run_extra(args):
                one bakron_solve_batched call over 16 lanes per step (CUDA graph
                replay; the same call on one lane is timed for context);
       gptq     the 4096 x 4096 solve with B = I (GPTQ, the method's special
-               case) under the layer's input-side factor, graph replay."""
+               case) under the layer's input-side factor, bakron_solve_gptq,
+               graph replay."""
     import torch
 
     import paper_2608_06291_gb300 as P
@@ -680,11 +681,11 @@ def run_extra(args):
         outg = (torch.empty(m, n, dtype=torch.uint8, device=dev),
                 torch.empty(m, 1, dtype=torch.float32, device=dev),
                 torch.empty(m, 1, dtype=torch.float32, device=dev), None)
-        P.bakron_solve(W, fac, cfg2.bits, 0, workspace=wsb, out=outg)
+        P.bakron_solve_gptq(W, fac, cfg2.bits, 0, workspace=wsb, out=outg)
         launches_per = P.bakron_last_launches()
         gr = torch.cuda.CUDAGraph()
         with torch.cuda.graph(gr):
-            P.bakron_solve(W, fac, cfg2.bits, 0, workspace=wsb, sync=False, out=outg)
+            P.bakron_solve_gptq(W, fac, cfg2.bits, 0, workspace=wsb, sync=False, out=outg)
 
         def step():
             gr.replay()
@@ -823,8 +824,9 @@ def run_extra(args):
         roof = {"bound": "tensor", "achieved": F_alg / (ms / 1e3) / 1e12, "peak": p_eff,
                 "unit": "TFLOP/s", "frac": 1e3 * t_roof / ms, "traffic": None,
                 "peak_source": roof_src, "roofline_ms": 1e3 * t_roof,
-                "note": "whole-solve roofline as for the general solve (the kernels do not "
-                        "specialise L^B = I)"}
+                "note": "bakron_solve_gptq (column recursion, row-parallel leaves): F_alg of "
+                        "B = I, m n (n - 1) flops, at the FP32-effective tensor rate plus "
+                        "17 B/entry at HBM rate"}
     elif args.workload == "batched":
         if P.lib().bakron_read_status_batched(wsS.data_ptr(), mh, n, lanes, None) != 0:
             raise RuntimeError("device status set during the timed steps")

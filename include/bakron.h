@@ -131,6 +131,25 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw,
                  int sync, void* stream);
 
 /*
+ * bakron_solve_gptq -- the solve with B = I, i.e. GPTQ (paper, Sec. 1: GPTQ
+ * is BaKron with an identity output-side factor; Alg. 1 applied to every row
+ * under H = A).  The rows are independent, so the recursion splits columns
+ * only: one launch rounds up to four 32-column tiles of every row (one warp
+ * per 32-row strip, 32 dependent steps per tile) and the errors of each
+ * finished column range reach the columns after it as one tensor-core
+ * product E L^A^T (3xTF32).  Arguments, outputs and errors as bakron_solve;
+ * only the L^A part of `factors` is read (its L^B may be anything, e.g. from
+ * bakron_prepare with B = I).  group_size must be 0 or a multiple of 32 (a
+ * group covers whole tiles); BAKRON_ERR_INVALID_ARG otherwise.  The result
+ * is the textbook GPTQ loop's (Alg. 1) on every row, up to fp32 rounding.
+ */
+int bakron_solve_gptq(const void* W, int wdtype, int m, int n, int64_t ldw,
+                      const void* factors, int bits, int group_size,
+                      uint8_t* codes, float* scales, float* zeros,
+                      float* prerounding, void* workspace,
+                      size_t workspace_bytes, int sync, void* stream);
+
+/*
  * bakron_grid_symmetric -- the quantisation grid of the paper's experiments
  * (Appendix "Experiments"): the symmetric alphabet {-l, ..., +l}, one scale
  * per row (group_size 0) or per (row, group of group_size columns), chosen

@@ -52,6 +52,9 @@ def lib() -> ctypes.CDLL:
     L.bakron_get_factors.restype = i32
     L.bakron_solve.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, vp, sz, i32, vp]
     L.bakron_solve.restype = i32
+    L.bakron_solve_gptq.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp, vp, sz,
+                                    i32, vp]
+    L.bakron_solve_gptq.restype = i32
     L.bakron_grid_symmetric.argtypes = [vp, i32, i32, i32, i64, i32, i32, i32, vp, vp, vp]
     L.bakron_grid_symmetric.restype = i32
     L.bakron_solve_with_grid.argtypes = [vp, i32, i32, i32, i64, vp, i32, i32, vp, vp, vp, vp,
@@ -222,6 +225,32 @@ def bakron_solve(W, f: Factors, bits: int, group_size: int = 0, workspace=None,
                             int(group_size), _ptr(codes), _ptr(scales), _ptr(zeros), _ptr(xpre),
                             _ptr(ws), ws.numel(), 1 if sync else 0, _stream(stream))
     _check(rc, "bakron_solve")
+    return (codes, scales, zeros, xpre) if prerounding else (codes, scales, zeros)
+
+
+def bakron_solve_gptq(W, f: Factors, bits: int, group_size: int = 0, workspace=None,
+                      prerounding: bool = False, sync: bool = True, out=None, stream=None):
+    """The solve with B = I (GPTQ on every row under L^A of `f`); arguments
+    and results as bakron_solve, group_size 0 or a multiple of 32."""
+    dt = _w_dtype(W)
+    m, n = W.shape
+    if (f.m, f.n) != (m, n):
+        raise ValueError("factor buffer was built for a different shape")
+    G = 1 if group_size == 0 else n // group_size
+    dev = W.device
+    if out is None:
+        codes = torch.empty(m, n, dtype=torch.uint8, device=dev)
+        scales = torch.empty(m, G, dtype=torch.float32, device=dev)
+        zeros = torch.empty(m, G, dtype=torch.float32, device=dev)
+        xpre = torch.empty(m, n, dtype=torch.float32, device=dev) if prerounding else None
+    else:
+        codes, scales, zeros, xpre = out
+    ws = workspace if workspace is not None else alloc_workspace(m, n, dev)
+    rc = lib().bakron_solve_gptq(_ptr(W), dt, m, n, W.stride(0), _ptr(f.buf), int(bits),
+                                 int(group_size), _ptr(codes), _ptr(scales), _ptr(zeros),
+                                 _ptr(xpre), _ptr(ws), ws.numel(), 1 if sync else 0,
+                                 _stream(stream))
+    _check(rc, "bakron_solve_gptq")
     return (codes, scales, zeros, xpre) if prerounding else (codes, scales, zeros)
 
 

@@ -130,6 +130,24 @@ int bakron_solve(const void* W, int wdtype, int m, int n, int64_t ldw, const voi
   return bakron_read_status(workspace, stream);
 }
 
+int bakron_solve_gptq(const void* W, int wdtype, int m, int n, int64_t ldw, const void* factors,
+                      int bits, int group_size, uint8_t* codes, float* scales, float* zeros,
+                      float* prerounding, void* workspace, size_t workspace_bytes, int sync,
+                      void* stream) {
+  if (!W || !factors || !codes || !scales || !zeros || !workspace || !dims_ok(m, n))
+    return BAKRON_ERR_INVALID_ARG;
+  if (wdtype != BAKRON_F32 && wdtype != BAKRON_BF16) return BAKRON_ERR_INVALID_ARG;
+  if (ldw < n || bits < 1 || bits > 8) return BAKRON_ERR_INVALID_ARG;
+  if (group_size < 0 || (group_size > 0 && (n % group_size != 0 || group_size % TILE != 0)))
+    return BAKRON_ERR_INVALID_ARG;
+  if (workspace_bytes < SolveLayout(m, n).bytes) return BAKRON_ERR_WORKSPACE;
+  cudaStream_t s = (cudaStream_t)stream;
+  int rc = gptq_impl(W, wdtype, m, n, ldw, factors, (1 << bits) - 1, group_size, codes, scales,
+                     zeros, prerounding, workspace, s);
+  if (rc != BAKRON_OK || !sync) return rc;
+  return bakron_read_status(workspace, stream);
+}
+
 int bakron_grid_symmetric(const void* W, int wdtype, int m, int n, int64_t ldw, int levels,
                           int group_size, int shrink_steps, float* scales, float* zeros,
                           void* stream) {

@@ -1,0 +1,249 @@
+// The B = I case of the solve (GPTQ, Sec. 1 and Alg. 1): with L^B = I the
+// rows of W are independent, entry (p, q) depends only on the entries left of
+// it in its own row, and the two-sided recursion collapses to column splits
+// (Alg. 4 splitting columns only):
+//
+//   rec(c0, c1): a range of at most GQ_BLOCK tile columns is a leaf launch;
+//                otherwise h = (c0 + c1) / 2, rec(c0, h),
+//                X[:, h..c1) += E[:, c0..h) L^A[h..c1, c0..h)^T  (tensor cores),
+//                rec(h, c1).
+//
+// A leaf launch gives one warp to each 32-row strip of W (lane p = row p), and
+// the warp walks the range's columns in order.  Column q of a tile is one
+// step: every lane rounds its row's entry, x_pq -> code, e_pq = s (c - z) - x,
+// then adds e_pq L^A[q'][q] to the pre-rounding values of the later columns
+// q' of the tile, which it keeps in registers.  A later tile of the range
+// starts from X plus the errors of the range's earlier tiles times the
+// matching blocks of L^A (the Alg. 4 nodes inside the range).  So a tile of
+// 32 x 32 entries takes 32 dependent steps, and all strips run side by side.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdlib>
+#include <mutex>
+
+#include "common.cuh"
+#include "profile.cuh"
+#include "tc_gemm.cuh"
+#include "tune.cuh"
+
+namespace bakron {
+
+constexpr int GQ_BLOCK = 4;                               // tile columns per leaf launch
+constexpr int GQ_LA_BLOCKS = GQ_BLOCK * (GQ_BLOCK + 1) / 2;   // L^A blocks one launch reads
+
+struct GptqArgs {
+  int Mt, Nt, m, n;
+  float* X;                     // pre-rounding values, in place (mp x np, row stride ldx)
+  int64_t ldx;
+  float *EH, *EL;               // E as tf32 hi / lo, row-major like X (the column band's A)
+  const float* LAblk;           // the factor buffer's L^A leaf blocks
+  const float *scales, *zeros;
+  int G, gsz, qmax;
+  uint8_t* codes;
+  int* status;
+  unsigned long long* stamp;
+};
+
+struct GptqSmem {
+  // L^A[J, J - g] of every tile J of the range and g = 0 .. J - c0, k-major
+  // ([j][q] = L^A[J, J-g][q][j]), in the order (J - c0) (J - c0 + 1) / 2 + g
+  __align__(16) float LA[GQ_LA_BLOCKS][TILE][LEAF_BLOCK_LD];
+  float Xs[TILE][GQ_BLOCK * TILE + 1];   // X of the strip's range in, pre-rounding values out
+  float Es[GQ_BLOCK][TILE][TILE + 1];    // errors of the range's tiles, [p][j]
+  uint8_t Cs[TILE][GQ_BLOCK * TILE + 4]; // codes (rows 132 bytes apart: no bank conflicts)
+};
+
+__device__ __forceinline__ void gq_cp_async16(void* dst, const void* src) {
+  const unsigned d = (unsigned)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(src) : "memory");
+}
+
+// Tiles c0 .. c0 + nt - 1 (nt <= GQ_BLOCK) of the strip of tile row blockIdx.x.
+__global__ void __launch_bounds__(32) k_gptq_leaf(int c0, int nt, GptqArgs a) {
+  extern __shared__ __align__(16) unsigned char gq_smem[];
+  GptqSmem& S = *reinterpret_cast<GptqSmem*>(gq_smem);
+  const int p = threadIdx.x;            // row of the strip
+  const int I = blockIdx.x;
+  const int64_t r0 = (int64_t)I * TILE, cbase = (int64_t)c0 * TILE;
+  // factor blocks (read-only during the solve) before waiting for the
+  // previous kernel
+  for (int t = 0; t < nt; ++t)
+    for (int g = 0; g <= t; ++g) {
+      const float* src = a.LAblk + ((int64_t)(c0 + t) * LEAF_BLOCKS + g) * LEAF_BLOCK_FLOATS;
+      float* dst = &S.LA[t * (t + 1) / 2 + g][0][0];
+      for (int c = p; c < LEAF_BLOCK_FLOATS / 4; c += 32) gq_cp_async16(dst + 4 * c, src + 4 * c);
+    }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+  // this row's grid on each tile (a group covers whole tiles: gsz % 32 == 0)
+  const int64_t row = r0 + p;
+  const bool row_real = row < a.m;
+  float sv[GQ_BLOCK], iv[GQ_BLOCK], zv[GQ_BLOCK];
+#pragma unroll
+  for (int t = 0; t < GQ_BLOCK; ++t) {
+    const int64_t col = cbase + (int64_t)t * TILE;
+    const bool ok = row_real && t < nt && col < a.n;
+    const float s = ok ? a.scales[row * a.G + col / a.gsz] : 1.f;
+    sv[t] = s;
+    iv[t] = 1.f / s;
+    zv[t] = ok ? a.zeros[row * a.G + col / a.gsz] : 0.f;
+  }
+  pdl_wait();
+  pdl_trigger();
+  stamp_begin(a.stamp);
+  // X of the strip's range (coalesced: lane = column)
+  for (int i = 0; i < TILE; ++i)
+    for (int c = p; c < nt * TILE; c += 32) S.Xs[i][c] = __ldcg(a.X + (r0 + i) * a.ldx + cbase + c);
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  __syncwarp();
+
+  constexpr float R = 12582912.f;   // 1.5 * 2^23: fl(v + R) - R rounds v to an integer
+  const float fq = (float)a.qmax;
+  bool bad = false;
+  for (int t = 0; t < nt; ++t) {
+    const int64_t col0 = cbase + (int64_t)t * TILE;
+    float acc[TILE];
+#pragma unroll
+    for (int q = 0; q < TILE; ++q) acc[q] = S.Xs[p][t * TILE + q];
+    // the range's earlier tiles: x += E[I, J-g] L^A[J, J-g]^T
+    for (int g = 1; g <= t; ++g) {
+      const float(*Lg)[LEAF_BLOCK_LD] = S.LA[t * (t + 1) / 2 + g];
+      const float(*Eg)[TILE + 1] = S.Es[t - g];
+#pragma unroll 4
+      for (int j = 0; j < TILE; ++j) {
+        const float e = Eg[p][j];
+#pragma unroll
+        for (int q4 = 0; q4 < TILE / 4; ++q4) {
+          const float4 l = *reinterpret_cast<const float4*>(&Lg[j][4 * q4]);
+          acc[4 * q4] = fmaf(e, l.x, acc[4 * q4]);
+          acc[4 * q4 + 1] = fmaf(e, l.y, acc[4 * q4 + 1]);
+          acc[4 * q4 + 2] = fmaf(e, l.z, acc[4 * q4 + 2]);
+          acc[4 * q4 + 3] = fmaf(e, l.w, acc[4 * q4 + 3]);
+        }
+      }
+    }
+    // the tile's 32 steps; the unit diagonal of L^A[J, J] is this entry's own
+    const float(*L0)[LEAF_BLOCK_LD] = S.LA[t * (t + 1) / 2];
+    const float s = sv[t], inv = iv[t], mz = -zv[t];
+#pragma unroll
+    for (int q = 0; q < TILE; ++q) {
+      const float x = acc[q];
+      const float tc = fminf(fmaxf(fmaf(x, inv, R), R + mz), R + fq + mz);
+      const float mk = (row_real && col0 + q < a.n) ? 1.f : 0.f;
+      const float e = fmaf(s * mk, tc - R, x * -mk);   // s (c - z) - x, rounded once
+      bad |= !isfinite(x);
+      S.Xs[p][t * TILE + q] = x;
+      S.Es[t][p][q] = e;
+      S.Cs[p][t * TILE + q] = (uint8_t)(int)(tc - (R + mz));
+#pragma unroll
+      for (int q4 = (q + 1) / 4; q4 < TILE / 4; ++q4) {
+        const float4 l = *reinterpret_cast<const float4*>(&L0[q][4 * q4]);
+        if (4 * q4 > q) acc[4 * q4] = fmaf(e, l.x, acc[4 * q4]);
+        if (4 * q4 + 1 > q) acc[4 * q4 + 1] = fmaf(e, l.y, acc[4 * q4 + 1]);
+        if (4 * q4 + 2 > q) acc[4 * q4 + 2] = fmaf(e, l.z, acc[4 * q4 + 2]);
+        if (4 * q4 + 3 > q) acc[4 * q4 + 3] = fmaf(e, l.w, acc[4 * q4 + 3]);
+      }
+    }
+  }
+  __syncwarp();
+  // outputs, coalesced (lane = column): pre-rounding values, codes, and E as
+  // an exact tf32 hi/lo pair for the column band
+  for (int i = 0; i < TILE; ++i) {
+    const int64_t r = r0 + i;
+    for (int c = p; c < nt * TILE; c += 32) {
+      const int64_t o = r * a.ldx + cbase + c;
+      a.X[o] = S.Xs[i][c];
+      const float e = S.Es[c / TILE][i][c % TILE];
+      const float hi = tf32_hi(e);
+      a.EH[o] = hi;
+      a.EL[o] = e - hi;
+      if (r < a.m && cbase + c < a.n) a.codes[r * a.n + cbase + c] = S.Cs[i][c];
+    }
+  }
+  if (bad) raise_status(a.status, BAKRON_ERR_NONFINITE);
+  stamp_end(a.stamp);
+}
+
+namespace {
+struct GqRun {
+  GptqArgs la;
+  TcMaps tcm;
+  TcOperands tco;
+  cudaStream_t s;
+  int rc;
+};
+
+void gq_leaf(GqRun& r, int c0, int c1) {
+  LaunchScope ls(kFamLeaf, r.s, 2.0 * TILE * TILE * TILE * r.la.Mt * (c1 - c0) * (c1 - c0 + 1) / 2);
+  GptqArgs la = r.la;
+  la.stamp = ls.stamp();
+  if (launch_pdl(k_gptq_leaf, dim3(r.la.Mt), dim3(32), sizeof(GptqSmem), r.s, c0, c1 - c0, la) !=
+      cudaSuccess)
+    r.rc = BAKRON_ERR_CUDA;
+}
+
+void gq_rec(GqRun& r, int c0, int c1) {
+  if (c1 - c0 <= GQ_BLOCK) {
+    gq_leaf(r, c0, c1);
+    return;
+  }
+  const int h = (c0 + c1) / 2;
+  gq_rec(r, c0, h);
+  {
+    LaunchScope ls(kFamTc2, r.s, 2.0 * TILE * TILE * TILE * r.la.Mt * (h - c0) * (c1 - h));
+    const int rc = tc_cols_stage(r.tcm, r.tco, c0, h, c1, r.s, ls.stamp());
+    if (rc != BAKRON_OK) r.rc = rc;
+  }
+  gq_rec(r, h, c1);
+}
+}  // namespace
+
+int launch_solve_prologue(const void* W, int wdt, int m, int n, int64_t ldw, int gsz, int G,
+                          int qmax, float* scales, float* zeros, float* X, int64_t mp, int64_t np,
+                          char* status_area, cudaStream_t s);
+int launch_copy_out(const float* X, int64_t np, int m, int n, float* out, cudaStream_t s);
+
+int gptq_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
+              int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
+              void* workspace, cudaStream_t s) {
+  FactorLayout fl(m, n);
+  SolveLayout sl(m, n);
+  char* ws = (char*)workspace;
+  const char* f = (const char*)factors;
+  static std::once_flag attr_once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(attr_once, [] {
+    attr_err = cudaFuncSetAttribute(k_gptq_leaf, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)sizeof(GptqSmem));
+  });
+  if (attr_err != cudaSuccess) return BAKRON_ERR_CUDA;
+  GqRun r;
+  r.s = s;
+  r.rc = BAKRON_OK;
+  const int Mt = ceil_div(m, TILE), Nt = ceil_div(n, TILE);
+  const int gsz = group_size == 0 ? n : group_size;
+  float* X = (float*)(ws + sl.off_X);
+  float* MH = (float*)(ws + sl.off_MH);
+  float* ML = (float*)(ws + sl.off_ML);
+  int* status = (int*)(ws + sl.off_status);
+  r.la = GptqArgs{Mt, Nt, m, n, X, sl.np, MH, ML, (const float*)(f + fl.off_LAblk), scales,
+                  zeros, n / gsz, gsz, qmax, codes, status, nullptr};
+  r.tco = TcOperands{sl.mp, sl.np, Mt, Nt,
+                     (const float*)(f + fl.off_LBH), (const float*)(f + fl.off_LBL),
+                     (const float*)(f + fl.off_LAH), (const float*)(f + fl.off_LAL),
+                     (float*)(ws + sl.off_EtH), (float*)(ws + sl.off_EtL), MH, ML, X, status};
+  if (!tc_band_maps(r.tcm, r.tco)) return BAKRON_ERR_CUDA;
+  reset_launch_count();
+  int rc = launch_solve_prologue(W, wdt, m, n, ldw, gsz, n / gsz, qmax, scales, zeros, X, sl.mp,
+                                 sl.np, ws + sl.off_status, s);
+  if (rc != BAKRON_OK) return rc;
+  gq_rec(r, 0, Nt);
+  if (prerounding) {
+    rc = launch_copy_out(X, sl.np, m, n, prerounding, s);
+    if (rc != BAKRON_OK) return rc;
+  }
+  BK_CUDA_OK(cudaGetLastError());
+  return r.rc;
+}
+
+}  // namespace bakron

@@ -1358,6 +1358,12 @@ static void rec(SolveArgs& a, int k, int l) {
   rec(a, h, l);
 }
 
+void launch_grid(const void* W, int wdt, int m, int n, int64_t ldw, int gsz, int G, int qmax,
+                 float* scales, float* zeros, cudaStream_t s);
+int launch_init(const void* W, int wdt, int m, int n, int64_t ldw, float* X, int64_t mp,
+                int64_t np, cudaStream_t s);
+int launch_copy_out(const float* X, int64_t np, int m, int n, float* out, cudaStream_t s);
+
 // Diagnostic only (bakron_diag_leaf_chain): where the leaves of the next
 // solve record the chain's clock64 before and after its steps.
 long long* g_diag_leaf_clk = nullptr;
@@ -1432,29 +1438,55 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
     BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_status + 64, 0, 256 - 64, s));
   else
     BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_status, 0, 256, s));
-  if (!grid_given) {
-    const int64_t warps = (int64_t)m * a.G;
-    LaunchScope ls(kFamInit, s);
-    k_grid<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(W, wdt, m, n, ldw, a.gsz, a.G,
-                                                                 a.qmax, scales, zeros,
-                                                                 ls.stamp());
-  }
+  if (!grid_given) launch_grid(W, wdt, m, n, ldw, a.gsz, a.G, a.qmax, scales, zeros, s);
   {
-    const int64_t chunks = a.mp * a.np / 8;
-    LaunchScope ls(kFamInit, s);
-    const unsigned blocks = (unsigned)std::min<int64_t>((chunks + 255) / 256, 152 * 8);
-    note(a, launch_pdl(k_init, dim3(blocks), dim3(256), 0, s, W, wdt, m, n, ldw, a.X, a.mp,
-                       a.np, ls.stamp()));
+    const int rc = launch_init(W, wdt, m, n, ldw, a.X, a.mp, a.np, s);
+    if (rc != BAKRON_OK) a.rc = rc;
   }
   rec(a, 0, a.Mt + a.Nt - 1);
   if (prerounding) {
-    const int64_t tot = (int64_t)m * n;
-    LaunchScope ls(kFamCopy, s);
-    note(a, launch_pdl(k_copy_out, dim3((unsigned)((tot + 255) / 256)), dim3(256), 0, s,
-                       (const float*)a.X, a.np, m, n, prerounding));
+    const int rc = launch_copy_out(a.X, a.np, m, n, prerounding, s);
+    if (rc != BAKRON_OK) a.rc = rc;
   }
   BK_CUDA_OK(cudaGetLastError());
   return a.rc;
+}
+
+// The first kernels of a solve: the min-max grid (k_grid) and X from W (k_init).
+void launch_grid(const void* W, int wdt, int m, int n, int64_t ldw, int gsz, int G, int qmax,
+                 float* scales, float* zeros, cudaStream_t s) {
+  const int64_t warps = (int64_t)m * G;
+  LaunchScope ls(kFamInit, s);
+  k_grid<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(W, wdt, m, n, ldw, gsz, G, qmax,
+                                                               scales, zeros, ls.stamp());
+}
+
+int launch_init(const void* W, int wdt, int m, int n, int64_t ldw, float* X, int64_t mp,
+                int64_t np, cudaStream_t s) {
+  const int64_t chunks = mp * np / 8;
+  LaunchScope ls(kFamInit, s);
+  const unsigned blocks = (unsigned)std::min<int64_t>((chunks + 255) / 256, 152 * 8);
+  return launch_pdl(k_init, dim3(blocks), dim3(256), 0, s, W, wdt, m, n, ldw, X, mp, np,
+                    ls.stamp()) == cudaSuccess
+             ? BAKRON_OK
+             : BAKRON_ERR_CUDA;
+}
+
+int launch_solve_prologue(const void* W, int wdt, int m, int n, int64_t ldw, int gsz, int G,
+                          int qmax, float* scales, float* zeros, float* X, int64_t mp, int64_t np,
+                          char* status_area, cudaStream_t s) {
+  BK_CUDA_OK(cudaMemsetAsync(status_area, 0, 256, s));
+  launch_grid(W, wdt, m, n, ldw, gsz, G, qmax, scales, zeros, s);
+  return launch_init(W, wdt, m, n, ldw, X, mp, np, s);
+}
+
+int launch_copy_out(const float* X, int64_t np, int m, int n, float* out, cudaStream_t s) {
+  const int64_t tot = (int64_t)m * n;
+  LaunchScope ls(kFamCopy, s);
+  return launch_pdl(k_copy_out, dim3((unsigned)((tot + 255) / 256)), dim3(256), 0, s, X, np, m,
+                    n, out) == cudaSuccess
+             ? BAKRON_OK
+             : BAKRON_ERR_CUDA;
 }
 
 }  // namespace bakron

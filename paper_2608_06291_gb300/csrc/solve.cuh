@@ -20,6 +20,14 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
                void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
                bool keep_status);
 
+// The B = I (GPTQ) solve (gptq.cu): grid, X from W, then the column
+// recursion.  Workspace and factor buffer as the general solve (only L^A's
+// planes and leaf blocks are read; the M planes hold E row-major).  Requires
+// group_size == 0 or a multiple of 32 (a group covers whole tiles).
+int gptq_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
+              int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
+              void* workspace, cudaStream_t s);
+
 // Diagnostic only (bakron_diag_leaf_chain): when set, the leaves of the next
 // solve record the chain warp's clock64 before and after its 63 steps there.
 extern long long* g_diag_leaf_clk;

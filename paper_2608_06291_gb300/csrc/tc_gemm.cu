@@ -64,7 +64,11 @@ constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*ba
 constexpr int NACC = 4;                         // TMEM accumulators, rotating per K stage
 constexpr uint32_t TMEM_COLS = NACC * BN;       // all 512 columns: one CTA per SM (shared memory)
 
-enum Mode { MODE_DENSE = 0, MODE_STAGE1 = 1, MODE_STAGE2 = 2, MODE_GRAM = 3 };
+// MODE_COLS: the column-band update of the B = I (GPTQ) schedule,
+// X[:, S2] += E[:, S1] L^A[S2, S1]^T with S1 = tile columns [k, h) and S2 =
+// [h, l); it reads and writes like stage 2 (A = E in the M planes, B = L^A,
+// TMA reduce-add into X).
+enum Mode { MODE_DENSE = 0, MODE_STAGE1 = 1, MODE_STAGE2 = 2, MODE_GRAM = 3, MODE_COLS = 4 };
 
 struct TcParams {
   int mode;
@@ -279,6 +283,11 @@ __host__ __device__ inline bool band_row_span(int mode, int k, int h, int l, int
                                               int& cb_lo, int& cb_hi) {
   const int I0 = 4 * rb;                     // first 32-tile row of the block
   if (I0 >= Mt) return false;
+  if (mode == MODE_COLS) {                   // every row; output tile columns [h, l)
+    cb_lo = h / 4;
+    cb_hi = (l - 1) / 4;
+    return true;
+  }
   // output 32-tiles (I, J) of the band S2 = [h, l) in rows I0..I0+3
   const int Ilast = min(I0 + 3, Mt - 1);
   const int jout_lo = max(0, h - Ilast);
@@ -325,6 +334,11 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
   if (!band_row_span(P.mode, P.k, P.h, P.l, P.Mt, P.Nt, b.rb, cb_lo, cb_hi)) return false;
   b.cb = P.mode == MODE_STAGE2 ? cb_hi - (int)blockIdx.x : cb_lo + (int)blockIdx.x;
   if (b.cb > cb_hi || b.cb < cb_lo) return false;
+  if (P.mode == MODE_COLS) {   // K = the tile columns of S1, the same for every block
+    b.k0 = P.k;
+    b.nk = P.h - P.k;
+    return true;
+  }
   const int I0 = 4 * b.rb, Ilast = min(I0 + 3, P.Mt - 1);
   const int J0 = 4 * b.cb;
   if (P.mode == MODE_STAGE1) {
@@ -408,7 +422,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   // during the solve: its part of the first ring slots is loaded before the
   // wait for the previous kernel, whose output (E^T or M) is the other one.
   const int npre = blk.nk < STAGES ? blk.nk : STAGES;
-  const bool a_static = P.mode != MODE_STAGE2;
+  const bool a_static = P.mode != MODE_STAGE2 && P.mode != MODE_COLS;
   constexpr bool bf16_ops = V == V_GRAM_BF16;
   if (warp == 0 && lane == 0) {
     for (int i = 0; i < npre; ++i) {
@@ -697,7 +711,9 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
           for (int ti = 0; ti < 4; ++ti) {
             for (int c = 0; c < 4; ++c) {
               const int I = 4 * blk.rb + ti, J = 4 * blk.cb + c;
-              if (I >= P.Mt || J >= P.Nt || I + J < P.h || I + J >= P.l) continue;
+              if (I >= P.Mt || J >= P.Nt) continue;
+              if (P.mode == MODE_COLS ? (J < P.h || J >= P.l) : (I + J < P.h || I + J >= P.l))
+                continue;
               tma_reduce_add_2d(&mapOh, smem + c * TILE_BYTES + ti * 4096, 32 * J, 32 * I);
             }
           }
@@ -973,6 +989,28 @@ int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, in
     e = launch_pdl(k_tc_band<V_BAND>, grid, dim3(THREADS), SMEM_BYTES, s, maps.M2, maps.LA2,
                    maps.Eth,
                    maps.Etl, maps.X32, maps.X32, P);
+  return e == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
+}
+
+int tc_cols_stage(const TcMaps& maps, const TcOperands& op, int k, int h, int l, cudaStream_t s,
+                  unsigned long long* stamp) {
+  if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
+  if (k >= h || h >= l) return BAKRON_OK;
+  TcParams P{};
+  P.stamp = stamp;
+  P.mode = MODE_COLS;
+  P.k = k; P.h = h; P.l = l;
+  P.Mt = op.Mt; P.Nt = op.Nt;
+  P.out_hi = op.MH; P.out_lo = op.ML; P.X = op.X;
+  P.ldo = op.np;
+  P.status = op.status;
+  P.spin_cycles = spin_cycles_from_env();
+  const int rows = (op.Mt + 3) / 4;              // 128-row blocks holding real tiles
+  const int cols = (l - 1) / 4 - h / 4 + 1;      // 128-column blocks covering S2
+  P.row0 = 0;
+  const cudaError_t e =
+      launch_pdl(k_tc_band<V_BAND>, dim3(cols, rows), dim3(THREADS), SMEM_BYTES, s, maps.M2,
+                 maps.LA2, maps.Eth, maps.Etl, maps.X32, maps.X32, P);
   return e == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
 }
 

@@ -35,4 +35,10 @@ long long spin_cycles_from_env();
 int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, int h, int l,
                   cudaStream_t s, unsigned long long* stamp = nullptr);
 
+// The column-band update of the B = I (GPTQ) schedule over 128 x 128 output
+// blocks: X[:, S2] += E[:, S1] L^A[S2, S1]^T, S1 = tile columns [k, h), S2 =
+// [h, l), with E in the M planes (row-major hi/lo).
+int tc_cols_stage(const TcMaps& maps, const TcOperands& op, int k, int h, int l, cudaStream_t s,
+                  unsigned long long* stamp = nullptr);
+
 }  // namespace bakron
