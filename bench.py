@@ -827,6 +827,23 @@ def run_extra(args):
                 "note": "bakron_solve_gptq (column recursion, row-parallel leaves): F_alg of "
                         "B = I, m n (n - 1) flops, at the FP32-effective tensor rate plus "
                         "17 B/entry at HBM rate"}
+        # family times of the replayed step (timeline stamps), as for the solve
+        P.bakron_profile_enable(2)
+        pg = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(pg):
+            P.bakron_solve_gptq(W, fac, cfg2.bits, 0, workspace=wsb, sync=False, out=outg)
+        for i in range(5):
+            flush.fill_(i & 0xFF)
+            pg.replay()
+            P.bakron_profile_collect()
+        fam = P.bakron_profile_read()
+        P.bakron_profile_enable(False)
+        roof["family_ms_per_step"] = {k: v[1] / 5 for k, v in fam.items() if v[0]}
+        roof["family_launches_per_step"] = {k: v[0] // 5 for k, v in fam.items() if v[0]}
+        tc_ms = roof["family_ms_per_step"].get("tc2", 0.0)
+        if tc_ms > 0:
+            tc_fl = fam["tc2"][2] / 5
+            roof["tc_frac"] = tc_fl / (tc_ms / 1e3) / 1e12 / p_eff
     elif args.workload == "batched":
         if P.lib().bakron_read_status_batched(wsS.data_ptr(), mh, n, lanes, None) != 0:
             raise RuntimeError("device status set during the timed steps")

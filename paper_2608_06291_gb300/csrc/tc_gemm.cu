@@ -56,12 +56,18 @@ namespace {
 constexpr int BM = 128, BN = 128, BK = 32;     // output block and K stage (fp32 elements)
 constexpr int STAGES = 3;
 constexpr int EPI_WARPS = 8;                   // two per TMEM lane quarter
-constexpr int THREADS = 32 * (2 + EPI_WARPS);
+// Threads issuing MMAs: warp 1 takes the even accumulator groups, warp
+// 2 + EPI_WARPS the odd ones, so that one issuer's barrier waits and
+// descriptor work overlap the other's MMAs (a single issuing thread spent
+// about a third of each K stage outside tcgen05.mma).
+constexpr int MMA_ISSUERS = 2;
+constexpr int THREADS = 32 * (2 + EPI_WARPS + (MMA_ISSUERS - 1));
 constexpr int EPI_COLS = BN / 2;               // columns summed by one epilogue warp
 constexpr uint32_t TILE_BYTES = BM * BK * 4;   // 16 KiB: one operand plane of one stage
 constexpr uint32_t STAGE_BYTES = 4 * TILE_BYTES;  // A hi, A lo, B hi, B lo
 constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
 constexpr int NACC = 4;                         // TMEM accumulators, rotating per K stage
+static_assert(NACC % MMA_ISSUERS == 0, "each issuer keeps its own accumulators");
 constexpr uint32_t TMEM_COLS = NACC * BN;       // all 512 columns: one CTA per SM (shared memory)
 
 // MODE_COLS: the column-band update of the B = I (GPTQ) schedule,
@@ -399,7 +405,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(accum, 1);
+    mbar_init(accum, MMA_ISSUERS);
     for (int a = 0; a < NACC; ++a) {
       mbar_init(&accF[a], 1);
       mbar_init(&accE[a], EPI_WARPS);  // lane 0 of each epilogue warp
@@ -544,17 +550,23 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
           raise_status(P.status, BAKRON_ERR_TIMEOUT);
       }
     }
-  } else if (warp == 1) {
-    // --------------------------------------------------------- MMA issuer
+  } else if (warp == 1 || warp == 2 + EPI_WARPS) {
+    // -------------------------------------------------------- MMA issuers
     // Each group of kgroup K stages (one stage in the band products, four of
     // exact bf16 products in the Gram) accumulates afresh into accumulator
     // (group mod NACC); the epilogue adds the groups in fp32 registers.  The
     // tensor core's accumulation is not round-to-nearest, and its error grows
     // with the number of MMAs summed in place; restarting every group bounds it.
+    // Issuer u takes the groups g with g mod MMA_ISSUERS == u (so the
+    // accumulators g mod NACC of the two never coincide).
+    const int u = warp == 1 ? 0 : 1;
     if (lane == 0) {
       const uint32_t idesc = idesc_tf32(BM, BN), idesc_b = idesc_bf16(BM, BN);
       const uint64_t desc0 = smem_desc(smem_u32(smem));   // stage 0, A hi, K step 0
+      bool issued_any = false;
       for (int i = 0; i < nk; ++i) {
+        if ((i / kgroup) % MMA_ISSUERS != u) continue;
+        if (*abort_flag) break;
         const int s = i % STAGES;
         const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
         const int g = i / kgroup, a = g % NACC;     // accumulator group of this slot
@@ -592,8 +604,9 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
         }
         if constexpr (kgroup > 1) mma_commit(&empty[s]);   // the slot back to the producer
         if (last) mma_commit(&accF[a]);  // the group's sum to the epilogue (kgroup 1: and the slot)
+        issued_any = true;
       }
-      if (nk > 0) mma_commit(accum);  // tracks every MMA issued above
+      if (issued_any) mma_commit(accum);  // tracks every MMA this thread issued
       else mbar_arrive(accum);
       // wind-down guard: all issued MMAs complete before anyone frees TMEM
       if (!mbar_wait(accum, 0, drain)) raise_status(P.status, BAKRON_ERR_TIMEOUT);
