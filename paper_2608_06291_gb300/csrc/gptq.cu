@@ -49,7 +49,11 @@ struct GptqSmem {
   // L^A[J, J - g] of every tile J of the range and g = 0 .. J - c0, k-major
   // ([j][q] = L^A[J, J-g][q][j]), in the order (J - c0) (J - c0 + 1) / 2 + g
   __align__(16) float LA[GQ_LA_BLOCKS][TILE][LEAF_BLOCK_LD];
-  float Xs[TILE][GQ_BLOCK * TILE + 1];   // X of the strip's range in, pre-rounding values out
+  // X of the strip's range, copied in with 16-byte asynchronous copies (rows
+  // 132 floats apart: 16-byte aligned, and the float4 reads of 8 lanes of
+  // different rows fall in different banks)
+  __align__(16) float Xin[TILE][GQ_BLOCK * TILE + 4];
+  float Xo[TILE][GQ_BLOCK * TILE + 1];   // pre-rounding values out
   float Es[GQ_BLOCK][TILE][TILE + 1];    // errors of the range's tiles, [p][j]
   uint8_t Cs[TILE][GQ_BLOCK * TILE + 4]; // codes (rows 132 bytes apart: no bank conflicts)
 };
@@ -91,9 +95,13 @@ __global__ void __launch_bounds__(32) k_gptq_leaf(int c0, int nt, GptqArgs a) {
   pdl_wait();
   pdl_trigger();
   stamp_begin(a.stamp);
-  // X of the strip's range (coalesced: lane = column)
-  for (int i = 0; i < TILE; ++i)
-    for (int c = p; c < nt * TILE; c += 32) S.Xs[i][c] = __ldcg(a.X + (r0 + i) * a.ldx + cbase + c);
+  // X of the strip's range: all its 16-byte chunks in flight at once
+  const int chunks_per_row = nt * TILE / 4;
+  for (int c = p; c < TILE * chunks_per_row; c += 32) {
+    const int i = c / chunks_per_row, k = c % chunks_per_row;
+    gq_cp_async16(&S.Xin[i][4 * k], a.X + (r0 + i) * a.ldx + cbase + 4 * k);
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
   asm volatile("cp.async.wait_group 0;" ::: "memory");
   __syncwarp();
 
@@ -104,7 +112,13 @@ __global__ void __launch_bounds__(32) k_gptq_leaf(int c0, int nt, GptqArgs a) {
     const int64_t col0 = cbase + (int64_t)t * TILE;
     float acc[TILE];
 #pragma unroll
-    for (int q = 0; q < TILE; ++q) acc[q] = S.Xs[p][t * TILE + q];
+    for (int q4 = 0; q4 < TILE / 4; ++q4) {
+      const float4 v = *reinterpret_cast<const float4*>(&S.Xin[p][t * TILE + 4 * q4]);
+      acc[4 * q4] = v.x;
+      acc[4 * q4 + 1] = v.y;
+      acc[4 * q4 + 2] = v.z;
+      acc[4 * q4 + 3] = v.w;
+    }
     // the range's earlier tiles: x += E[I, J-g] L^A[J, J-g]^T
     for (int g = 1; g <= t; ++g) {
       const float(*Lg)[LEAF_BLOCK_LD] = S.LA[t * (t + 1) / 2 + g];
@@ -132,7 +146,7 @@ __global__ void __launch_bounds__(32) k_gptq_leaf(int c0, int nt, GptqArgs a) {
       const float mk = (row_real && col0 + q < a.n) ? 1.f : 0.f;
       const float e = fmaf(s * mk, tc - R, x * -mk);   // s (c - z) - x, rounded once
       bad |= !isfinite(x);
-      S.Xs[p][t * TILE + q] = x;
+      S.Xo[p][t * TILE + q] = x;
       S.Es[t][p][q] = e;
       S.Cs[p][t * TILE + q] = (uint8_t)(int)(tc - (R + mz));
 #pragma unroll
@@ -152,7 +166,7 @@ __global__ void __launch_bounds__(32) k_gptq_leaf(int c0, int nt, GptqArgs a) {
     const int64_t r = r0 + i;
     for (int c = p; c < nt * TILE; c += 32) {
       const int64_t o = r * a.ldx + cbase + c;
-      a.X[o] = S.Xs[i][c];
+      a.X[o] = S.Xo[i][c];
       const float e = S.Es[c / TILE][i][c % TILE];
       const float hi = tf32_hi(e);
       a.EH[o] = hi;

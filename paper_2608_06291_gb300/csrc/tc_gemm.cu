@@ -56,18 +56,12 @@ namespace {
 constexpr int BM = 128, BN = 128, BK = 32;     // output block and K stage (fp32 elements)
 constexpr int STAGES = 3;
 constexpr int EPI_WARPS = 8;                   // two per TMEM lane quarter
-// Threads issuing MMAs: warp 1 takes the even accumulator groups, warp
-// 2 + EPI_WARPS the odd ones, so that one issuer's barrier waits and
-// descriptor work overlap the other's MMAs (a single issuing thread spent
-// about a third of each K stage outside tcgen05.mma).
-constexpr int MMA_ISSUERS = 2;
-constexpr int THREADS = 32 * (2 + EPI_WARPS + (MMA_ISSUERS - 1));
+constexpr int THREADS = 32 * (2 + EPI_WARPS);
 constexpr int EPI_COLS = BN / 2;               // columns summed by one epilogue warp
 constexpr uint32_t TILE_BYTES = BM * BK * 4;   // 16 KiB: one operand plane of one stage
 constexpr uint32_t STAGE_BYTES = 4 * TILE_BYTES;  // A hi, A lo, B hi, B lo
 constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
 constexpr int NACC = 4;                         // TMEM accumulators, rotating per K stage
-static_assert(NACC % MMA_ISSUERS == 0, "each issuer keeps its own accumulators");
 constexpr uint32_t TMEM_COLS = NACC * BN;       // all 512 columns: one CTA per SM (shared memory)
 
 // MODE_COLS: the column-band update of the B = I (GPTQ) schedule,
@@ -375,8 +369,8 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint64_t* bars = (uint64_t*)(smem + STAGES * STAGE_BYTES);
   uint64_t* full = bars;                 // [STAGES] smem stage loaded
-  uint64_t* empty = bars + STAGES;       // [STAGES] slot free again: its MMAs are complete
-                                         // (owner's commit) and every issuer has passed it
+  uint64_t* empty = bars + STAGES;       // [STAGES] slot read by its MMAs (kgroup > 1 only;
+                                         // otherwise the slot's accF commit frees it)
   uint64_t* accum = bars + 2 * STAGES;   // [1] every MMA of the CTA complete
   uint64_t* accF = accum + 1;            // [NACC] accumulator holds a finished K stage
   uint64_t* accE = accum + 1 + NACC;     // [NACC] accumulator read out by the epilogue
@@ -403,9 +397,9 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], MMA_ISSUERS);
+      mbar_init(&empty[s], 1);
     }
-    mbar_init(accum, MMA_ISSUERS);
+    mbar_init(accum, 1);
     for (int a = 0; a < NACC; ++a) {
       mbar_init(&accF[a], 1);
       mbar_init(&accE[a], EPI_WARPS);  // lane 0 of each epilogue warp
@@ -461,12 +455,15 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
     for (int i = 0; i < nk; ++i) {
       const int s = i % STAGES;
       bool ok = true;
-      // slot s was last used by stage j = i - STAGES: its MMAs are complete
-      // (the owning issuer's commit) and the other issuer has passed it, so
-      // no issuer can still be waiting on that phase of full[s]
+      // slot s was last read by the MMAs of stage j = i - STAGES, which are
+      // complete when their accumulator's commit arrives (accF); that barrier
+      // cannot have moved on to stage j + NACC yet, which needs this load
       if (lane == 0 && i >= STAGES) {
         const int j = i - STAGES;
-        ok = mbar_wait(&empty[s], (uint32_t)(j / STAGES) & 1u, P.spin_cycles);
+        if constexpr (kgroup > 1)
+          ok = mbar_wait(&empty[s], (uint32_t)(j / STAGES) & 1u, P.spin_cycles);
+        else
+          ok = mbar_wait(&accF[j % NACC], (uint32_t)(j / NACC) & 1u, P.spin_cycles);
       }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok || *abort_flag) {
@@ -547,45 +544,31 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
           raise_status(P.status, BAKRON_ERR_TIMEOUT);
       }
     }
-  } else if (warp == 1 || warp == 2 + EPI_WARPS) {
-    // -------------------------------------------------------- MMA issuers
+  } else if (warp == 1) {
+    // --------------------------------------------------------- MMA issuer
     // Each group of kgroup K stages (one stage in the band products, four of
     // exact bf16 products in the Gram) accumulates afresh into accumulator
     // (group mod NACC); the epilogue adds the groups in fp32 registers.  The
     // tensor core's accumulation is not round-to-nearest, and its error grows
     // with the number of MMAs summed in place; restarting every group bounds it.
-    // Issuer u owns the groups g with g mod MMA_ISSUERS == u (so the
-    // accumulators g mod NACC of the two never coincide), but walks every
-    // stage in order: it waits for each stage's data (an mbarrier parity wait
-    // is only sound one phase at a time) and, for a stage it does not own,
-    // arrives on the slot's empty barrier, which the producer waits on before
-    // reloading the slot.  So neither issuer can fall two phases behind.
-    const int u = warp == 1 ? 0 : 1;
     if (lane == 0) {
       const uint32_t idesc = idesc_tf32(BM, BN), idesc_b = idesc_bf16(BM, BN);
       const uint64_t desc0 = smem_desc(smem_u32(smem));   // stage 0, A hi, K step 0
-      bool issued_any = false;
       for (int i = 0; i < nk; ++i) {
-        if (*abort_flag) break;
         const int s = i % STAGES;
         const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
         const int g = i / kgroup, a = g % NACC;     // accumulator group of this slot
-        const bool mine = g % MMA_ISSUERS == u;
         const bool first = i % kgroup == 0;
         const bool last = i % kgroup == kgroup - 1 || i == nk - 1;
         // accumulator a was last used by group g - NACC: wait until it was read
         // out (the producer's and the epilogue's aborts surface here as time-outs)
         const bool ok = mbar_wait(&full[s], ph, P.spin_cycles) &&
-                        (!mine || !first || g < NACC ||
+                        (!first || g < NACC ||
                          mbar_wait(&accE[a], (uint32_t)(g / NACC - 1) & 1u, P.spin_cycles));
         if (!ok) {
           raise_status(P.status, BAKRON_ERR_TIMEOUT);
           *abort_flag = 1;
           break;
-        }
-        if (!mine) {
-          mbar_arrive(&empty[s]);
-          continue;
         }
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         // descriptors of this stage's four planes; K steps of 32 bytes add 2 to
@@ -607,11 +590,10 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
             if (V == V_BAND || !P.a_exact) mma_tf32(d, dal + o, dbh + o, idesc, 1u);
           }
         }
-        mma_commit(&empty[s]);           // the slot back to the producer once read
-        if (last) mma_commit(&accF[a]);  // the group's sum to the epilogue
-        issued_any = true;
+        if constexpr (kgroup > 1) mma_commit(&empty[s]);   // the slot back to the producer
+        if (last) mma_commit(&accF[a]);  // the group's sum to the epilogue (kgroup 1: and the slot)
       }
-      if (issued_any) mma_commit(accum);  // tracks every MMA this thread issued
+      if (nk > 0) mma_commit(accum);  // tracks every MMA issued above
       else mbar_arrive(accum);
       // wind-down guard: all issued MMAs complete before anyone frees TMEM
       if (!mbar_wait(accum, 0, drain)) raise_status(P.status, BAKRON_ERR_TIMEOUT);
