@@ -55,12 +55,89 @@ struct GptqSmem {
   __align__(16) float Xin[TILE][GQ_BLOCK * TILE + 4];
   float Xo[TILE][GQ_BLOCK * TILE + 1];   // pre-rounding values out
   float Es[GQ_BLOCK][TILE][TILE + 1];    // errors of the range's tiles, [p][j]
+  float T1[TILE][TILE + 1];              // the window's sum for the current tile, [p][q]
   uint8_t Cs[TILE][GQ_BLOCK * TILE + 4]; // codes (rows 132 bytes apart: no bank conflicts)
 };
 
 __device__ __forceinline__ void gq_cp_async16(void* dst, const void* src) {
   const unsigned d = (unsigned)__cvta_generic_to_shared(dst);
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(src) : "memory");
+}
+
+// tf32 split of an fp32 value: hi = x rounded to tf32, lo = the rest rounded
+// to tf32 (the 3xTF32 scheme: products hi*hi + hi*lo + lo*hi keep fp32
+// accuracy; the dropped lo*lo term is below 2^-22 relative).
+__device__ __forceinline__ void tf32_split(float x, uint32_t& hi, uint32_t& lo) {
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(hi) : "f"(x));
+  const float rest = x - __uint_as_float(hi);
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(lo) : "f"(rest));
+}
+
+// D += A B on the warp's tensor cores: A 16 x 8 (row-major fragment a[4]),
+// B 8 x 8 (b[2]), D 16 x 8 fp32 (d[4]), tf32 inputs.
+__device__ __forceinline__ void mma_tf32_16x8x8(float (&d)[4], const uint32_t (&a)[4],
+                                                const uint32_t (&b)[2]) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+// The window of tile t of the range, T1 = sum_{g=1..t} E[I, J-g] L^A[J, J-g]^T
+// (32 x 32, fp32-accurate by the 3xTF32 split), into S.T1 ([p][q]).  With
+// lane = 4 gid + tig, an m16n8k8 fragment holds A(gid (+8), tig (+4)),
+// B(k = tig (+4), n = gid) and D(gid (+8), 2 tig (+1)).
+__device__ __forceinline__ void gptq_window(GptqSmem& S, int t, int lane) {
+  const int gid = lane >> 2, tig = lane & 3;
+  float d[2][4][4];
+#pragma unroll
+  for (int mi = 0; mi < 2; ++mi)
+#pragma unroll
+    for (int ni = 0; ni < 4; ++ni)
+#pragma unroll
+      for (int r = 0; r < 4; ++r) d[mi][ni][r] = 0.f;
+  for (int g = 1; g <= t; ++g) {
+    const float(*Lg)[LEAF_BLOCK_LD] = S.LA[t * (t + 1) / 2 + g];   // B(k = j, n = q) = Lg[j][q]
+    const float(*Eg)[TILE + 1] = S.Es[t - g];                       // A(p, j) = Eg[p][j]
+#pragma unroll
+    for (int kk = 0; kk < TILE / 8; ++kk) {
+      uint32_t ah[2][4], al[2][4], bh[4][2], bl[4][2];
+#pragma unroll
+      for (int mi = 0; mi < 2; ++mi) {
+        const int r = 16 * mi + gid, c = 8 * kk + tig;
+        tf32_split(Eg[r][c], ah[mi][0], al[mi][0]);
+        tf32_split(Eg[r + 8][c], ah[mi][1], al[mi][1]);
+        tf32_split(Eg[r][c + 4], ah[mi][2], al[mi][2]);
+        tf32_split(Eg[r + 8][c + 4], ah[mi][3], al[mi][3]);
+      }
+#pragma unroll
+      for (int ni = 0; ni < 4; ++ni) {
+        const int k = 8 * kk + tig, n = 8 * ni + gid;
+        tf32_split(Lg[k][n], bh[ni][0], bl[ni][0]);
+        tf32_split(Lg[k + 4][n], bh[ni][1], bl[ni][1]);
+      }
+#pragma unroll
+      for (int mi = 0; mi < 2; ++mi)
+#pragma unroll
+        for (int ni = 0; ni < 4; ++ni) {
+          mma_tf32_16x8x8(d[mi][ni], al[mi], bh[ni]);
+          mma_tf32_16x8x8(d[mi][ni], ah[mi], bl[ni]);
+          mma_tf32_16x8x8(d[mi][ni], ah[mi], bh[ni]);
+        }
+    }
+  }
+#pragma unroll
+  for (int mi = 0; mi < 2; ++mi)
+#pragma unroll
+    for (int ni = 0; ni < 4; ++ni) {
+      const int r = 16 * mi + gid, c = 8 * ni + 2 * tig;
+      S.T1[r][c] = d[mi][ni][0];
+      S.T1[r][c + 1] = d[mi][ni][1];
+      S.T1[r + 8][c] = d[mi][ni][2];
+      S.T1[r + 8][c + 1] = d[mi][ni][3];
+    }
+  __syncwarp();
 }
 
 // Tiles c0 .. c0 + nt - 1 (nt <= GQ_BLOCK) of the strip of tile row blockIdx.x.
@@ -119,22 +196,13 @@ __global__ void __launch_bounds__(32) k_gptq_leaf(int c0, int nt, GptqArgs a) {
       acc[4 * q4 + 2] = v.z;
       acc[4 * q4 + 3] = v.w;
     }
-    // the range's earlier tiles: x += E[I, J-g] L^A[J, J-g]^T
-    for (int g = 1; g <= t; ++g) {
-      const float(*Lg)[LEAF_BLOCK_LD] = S.LA[t * (t + 1) / 2 + g];
-      const float(*Eg)[TILE + 1] = S.Es[t - g];
-#pragma unroll 4
-      for (int j = 0; j < TILE; ++j) {
-        const float e = Eg[p][j];
+    // the range's earlier tiles: x += sum_g E[I, J-g] L^A[J, J-g]^T
+    if (t > 0) {
+      __syncwarp();                     // this warp's errors of tile t - 1 are in S.Es
+      gptq_window(S, t, p);
 #pragma unroll
-        for (int q4 = 0; q4 < TILE / 4; ++q4) {
-          const float4 l = *reinterpret_cast<const float4*>(&Lg[j][4 * q4]);
-          acc[4 * q4] = fmaf(e, l.x, acc[4 * q4]);
-          acc[4 * q4 + 1] = fmaf(e, l.y, acc[4 * q4 + 1]);
-          acc[4 * q4 + 2] = fmaf(e, l.z, acc[4 * q4 + 2]);
-          acc[4 * q4 + 3] = fmaf(e, l.w, acc[4 * q4 + 3]);
-        }
-      }
+      for (int q = 0; q < TILE; ++q) acc[q] += S.T1[p][q];
+      __syncwarp();                     // S.T1 read before the next tile writes it
     }
     // the tile's 32 steps; the unit diagonal of L^A[J, J] is this entry's own
     const float(*L0)[LEAF_BLOCK_LD] = S.LA[t * (t + 1) / 2];
