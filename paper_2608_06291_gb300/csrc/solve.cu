@@ -289,6 +289,14 @@ static_assert(KM == LEAF_BLOCK_LD, "the factor buffer's leaf blocks are copied a
 constexpr int LEAF_WINDOW = 15;
 static_assert(LEAF_WINDOW + 1 == LEAF_BLOCKS, "a window needs the blocks L[I, I-1 .. I-LEAF_WINDOW]");
 
+// Rounding to the nearest integer (ties to even) by the shift LEAF_R =
+// 1.5 * 2^23: for |v| < 2^22, fl(v + LEAF_R) - LEAF_R is v rounded to an
+// integer, and the clamp to integer bounds commutes with it, so
+//     c - z = clamp(fl(x * fl(1/s) + LEAF_R), LEAF_R - z, LEAF_R + qmax - z) - LEAF_R
+// (one fused multiply-add: the product x * fl(1/s) is rounded once, to the
+// integer).  Larger |v| fall outside the bounds and are clamped.
+constexpr float LEAF_R = 12582912.f;
+
 // 32^3 products a window-P leaf forms before its wavefront (T1 and U).
 __host__ __device__ constexpr int window_products(int P) { return 2 * P; }
 
@@ -300,7 +308,7 @@ struct LeafSmem {
   __align__(16) float Ebr[4][LEAF_ROWS_PADDED];   // errors of a step, by row (ring of 4 steps)
   float Part[4][LEAF_HELPERS][TILE];              // partial pre of a step (ring of 4 steps)
   float4 Lsub[TILE];                              // (L^B[p][p-1], L^B[p][p-2], L^B[p][p-3], 0)
-  __align__(16) float4 Srzl[TILE][TILE];          // (s, 1/s, -z, 0) per entry
+  __align__(16) float4 Srzl[TILE][TILE];          // (s, 1/s, R - z, R + qmax - z) per entry
   union {
     struct {   // prologue of a window-P leaf: its window, staged one d at a time
       // buffer b holds the operands of one d: [0] E[I, J-d] k-major
@@ -471,7 +479,10 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
 #pragma unroll
   for (int k = 0; k < LEAF_PER_THREAD; ++k) {
     const int e = t + k * LEAF_THREADS;
-    S.Srzl[e / TILE][e % TILE] = make_float4(scv[k], 1.f / scv[k], -zv[k], 0.f);
+    // the clamp bounds of the shifted rounding (LEAF_R - z, LEAF_R + qmax - z:
+    // integers below 2^24, exact in fp32)
+    S.Srzl[e / TILE][e % TILE] = make_float4(scv[k], 1.f / scv[k], LEAF_R - zv[k],
+                                             LEAF_R + (float)a.qmax - zv[k]);
   }
   for (int e = t; e < 4 * LEAF_ROWS_PADDED; e += LEAF_THREADS) (&S.Ebr[0][0])[e] = 0.f;
   if (P >= 2) {
@@ -550,17 +561,12 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     // ------------------------------------------------ the chain
     const bool col_real = (c0 + q) < a.n;
     const int rows_real = a.m - (int)r0;     // rows p < rows_real are inside W
+    // entry (p, q) is real iff 0 <= p < plim (one unsigned compare per step)
+    const unsigned plim = col_real ? (unsigned)min(max(rows_real, 0), TILE) : 0u;
     const float la1 = q >= 1 ? S.LA0[q - 1][q] : 0.f;
     const float la2 = q >= 2 ? S.LA0[q - 2][q] : 0.f;
     const float la3 = q >= 3 ? S.LA0[q - 3][q] : 0.f;
-    const float fq = (float)a.qmax;
-    // Rounding to the nearest integer (ties to even) by the shift R = 1.5 * 2^23:
-    // for |v| < 2^22, fl(v + R) - R is v rounded to an integer, and the clamp
-    // to integer bounds commutes with it, so
-    //     c - z = clamp(fl(x * fl(1/s) + R), R - z, R + qmax - z) - R
-    // (one fused multiply-add: the product x * fl(1/s) is rounded once, to
-    // the integer).  Larger |v| fall outside the bounds and are clamped.
-    constexpr float R = 12582912.f;
+    constexpr float R = LEAF_R;
     float E1 = 0.f, E2 = 0.f, E3 = 0.f;
     float L1_1 = 0.f, L1_2 = 0.f, L1_3 = 0.f, L2_2 = 0.f, L2_3 = 0.f, L3_3 = 0.f;
     // One step.  Of the explicit terms only E1 (own column, last step) and
@@ -571,7 +577,7 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     // factor mk).
     auto step = [&](int d, bool odd, float pre, const float4& g, const float4& lb) {
       const int p = d - q;
-      const bool on_tile = p >= 0 && p < TILE;
+      const bool on_tile = (unsigned)p < (unsigned)TILE;
       float A = fmaf(la2, L2_2, pre);
       const float A2 = fmaf(lb.y, E2, (lb.x * la1) * L1_2);
       if (odd) {
@@ -583,9 +589,9 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
       const float nL3_3 = __shfl_up_sync(0xffffffffu, L2_2, 1);   // column q-3, this step's d-2
       const float x = fmaf(la1, L1_1, fmaf(lb.x, E1, A));
       const float nL2_2 = __shfl_up_sync(0xffffffffu, L1_1, 1);   // column q-2, step d-1
-      const float tc = fminf(fmaxf(fmaf(x, g.y, R), R + g.z), R + fq + g.z);
-      const float mk = (on_tile && p < rows_real && col_real) ? 1.f : 0.f;
-      const float e = fmaf(g.x * mk, tc - R, x * -mk);   // s (c - z) - x, rounded once
+      const float tc = fminf(fmaxf(fmaf(x, g.y, R), g.z), g.w);
+      const float mk = (unsigned)p < plim ? 1.f : 0.f;
+      const float e = fmaf(g.x, tc - R, -x) * mk;   // s (c - z) - x, rounded once
       L1_3 = L1_2;
       L1_2 = L1_1;
       L2_3 = L2_2;
@@ -597,17 +603,18 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
       L1_1 = __shfl_up_sync(0xffffffffu, e, 1);                    // column q-1, step d
       if (on_tile) {
         S.u.w.XE[p][q] = make_float2(x, e);
-        S.u.w.Cs[p][q] = (uint8_t)(int)(tc - (R + g.z));
+        S.u.w.Cs[p][q] = (uint8_t)(int)(tc - g.z);
       }
       S.Ebr[d & 3][p & (TILE - 1)] = e;    // rows off the tile get a zero
     };
-    // (s, 1/s, -z) and the sub-diagonal L^B of the next interval's entries are
-    // loaded one interval ahead
+    // the grid and the sub-diagonal L^B of the next interval's entries are
+    // loaded one interval ahead; three intervals per loop iteration, so that
+    // the three-step histories (E*, L*_*) rotate by renaming
     float4 g0 = S.Srzl[(0 - q) & (TILE - 1)][q], g1 = S.Srzl[(1 - q) & (TILE - 1)][q];
     float4 lb0 = S.Lsub[(0 - q) & (TILE - 1)], lb1 = S.Lsub[(1 - q) & (TILE - 1)];
     leaf_sync();   // the helpers' pre of steps 0 and 1
     if (a.clk != nullptr && lane == 0) a.clk[0] = clock64();
-#pragma unroll 1
+#pragma unroll 3
     for (int k = 0; k < TILE; ++k) {
       const int d0 = 2 * k, d1 = 2 * k + 1;
       const float* pa = &S.Part[d0 & 3][0][q];
