@@ -407,6 +407,12 @@ int bakron_read_status(void* workspace, void* stream);
  */
 int bakron_profile_enable(int on);
 int bakron_profile_collect(void* stream);
+/* Timeline mode: the launches of the last collected run, in enqueue order --
+ * family, algorithmic flops, and start / end (us from the run's first start;
+ * -1 for a launch without stamps).  Fills at most `max` entries of each
+ * (host) array and returns the number of launches, or a negative status. */
+int bakron_profile_launch_stamps(int max, int* family, double* flops,
+                                 double* start_us, double* end_us);
 int bakron_profile_read(int family, int* launches, double* ms, double* flops);
 int bakron_last_launches(void);
 

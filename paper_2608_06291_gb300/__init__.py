@@ -13,6 +13,7 @@ from .bakron import (BakronError, Factors, alloc_workspace, bakron_diag_gemm_tf3
                      bakron_batched_workspace_bytes,
                      bakron_last_launches, bakron_prepare, bakron_profile_enable,
                      bakron_profile_read, bakron_profile_collect, bakron_profile_timeline,
+                     bakron_profile_launch_stamps,
                      bakron_read_status, bakron_set_factors, bakron_solve, bakron_solve_gptq,
                      bakron_solve_noalloc, bakron_read_status_noalloc,
                      dequantize, factors_bytes, lib, library_path, strerror, workspace_bytes)

@@ -84,6 +84,9 @@ def lib() -> ctypes.CDLL:
     L.bakron_profile_enable.restype = i32
     L.bakron_profile_collect.argtypes = [vp]
     L.bakron_profile_collect.restype = i32
+    dp = ctypes.POINTER(ctypes.c_double)
+    L.bakron_profile_launch_stamps.argtypes = [i32, ctypes.POINTER(i32), dp, dp, dp]
+    L.bakron_profile_launch_stamps.restype = i32
     L.bakron_diag_leaf_chain.argtypes = [vp, i32, vp, vp, vp, vp, vp, ctypes.c_size_t,
                                          ctypes.POINTER(ctypes.c_double), vp]
     L.bakron_diag_leaf_chain.restype = i32
@@ -511,6 +514,18 @@ def bakron_profile_timeline() -> tuple:
     _check(lib().bakron_profile_read(-1, ctypes.byref(n), ctypes.byref(ms), None),
            "bakron_profile_read")
     return n.value, ms.value
+
+
+def bakron_profile_launch_stamps(max_launches: int = 1 << 15) -> list:
+    """Timeline mode: [(family name, flops, start_us, end_us)] of the last
+    collected run, in enqueue order."""
+    n = max_launches
+    fam = (ctypes.c_int * n)()
+    fl, st, en = (ctypes.c_double * n)(), (ctypes.c_double * n)(), (ctypes.c_double * n)()
+    k = lib().bakron_profile_launch_stamps(n, fam, fl, st, en)
+    if k < 0:
+        _check(-k, "bakron_profile_launch_stamps")
+    return [(PROFILE_FAMILIES[fam[i]], fl[i], st[i], en[i]) for i in range(min(k, n))]
 
 
 def bakron_profile_read() -> dict:

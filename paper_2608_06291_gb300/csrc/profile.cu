@@ -41,6 +41,7 @@ double g_timeline_ms = 0.0;          // sum over collected replays of (last end 
 int g_replays = 0;
 unsigned long long* g_stamps = nullptr;   // device, 2 per slot
 std::vector<std::pair<int, double>> g_slots;   // (family, flops) of the recorded solve
+std::vector<unsigned long long> g_last;         // stamps of the last collected run
 thread_local int t_launch_count = 0;
 
 cudaEvent_t take_event() {
@@ -152,6 +153,7 @@ extern "C" int bakron_profile_collect(void* stream) {
   BK_CUDA_OK(cudaStreamSynchronize(s));
   if (n) BK_CUDA_OK(cudaMemcpy(h.data(), g_stamps, sizeof(unsigned long long) * 2 * n,
                                cudaMemcpyDeviceToHost));
+  g_last.assign(h.begin(), h.begin() + 2 * n);
   // launches in enqueue order; a launch without stamps (its kernel takes no
   // stamp slot, or none of its CTAs had work) owns no time
   unsigned long long first = 0, prev_end = 0;
@@ -196,3 +198,22 @@ extern "C" int bakron_profile_read(int family, int* launches, double* ms, double
 }
 
 extern "C" int bakron_last_launches(void) { return t_launch_count; }
+
+extern "C" int bakron_profile_launch_stamps(int max, int* family, double* flops,
+                                            double* start_us, double* end_us) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (max < 0 || !family || !flops || !start_us || !end_us) return -BAKRON_ERR_INVALID_ARG;
+  const size_t n = std::min(g_slots.size(), g_last.size() / 2);
+  unsigned long long t0 = ~0ull;
+  for (size_t i = 0; i < n; ++i)
+    if (g_last[2 * i + 1] != 0) t0 = std::min(t0, g_last[2 * i]);
+  const int k = (int)std::min<size_t>(n, (size_t)max);
+  for (int i = 0; i < k; ++i) {
+    family[i] = g_slots[i].first;
+    flops[i] = g_slots[i].second;
+    const unsigned long long b = g_last[2 * i], e = g_last[2 * i + 1];
+    start_us[i] = e ? 1e-3 * (double)(b - t0) : -1.0;
+    end_us[i] = e ? 1e-3 * (double)(e - t0) : -1.0;
+  }
+  return (int)n;
+}
