@@ -165,6 +165,27 @@ __device__ __forceinline__ void stamp_end(unsigned long long* slot) {
   if (slot != nullptr && threadIdx.x == 0) atomicMax(slot + 1, global_ns());
 }
 
+// tf32 split of an fp32 value: hi = x rounded to tf32, lo = the rest rounded
+// to tf32 (the 3xTF32 scheme: products hi*hi + hi*lo + lo*hi keep fp32
+// accuracy; the dropped lo*lo term is below 2^-22 relative).
+__device__ __forceinline__ void tf32_split(float x, uint32_t& hi, uint32_t& lo) {
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(hi) : "f"(x));
+  const float rest = x - __uint_as_float(hi);
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(lo) : "f"(rest));
+}
+
+// D += A B on the warp's tensor cores (mma.sync; used for the small 32^3
+// products of the leaves): A 16 x 8 (row-major fragment a[4]),
+// B 8 x 8 (b[2]), D 16 x 8 fp32 (d[4]), tf32 inputs.
+__device__ __forceinline__ void mma_tf32_16x8x8(float (&d)[4], const uint32_t (&a)[4],
+                                                const uint32_t (&b)[2]) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
 // Device status word (first int of every workspace).  Kernels only ever raise
 // it with atomicMax-free writes of a nonzero code; the host reads and clears.
 __device__ inline void raise_status(int* status, int code) {

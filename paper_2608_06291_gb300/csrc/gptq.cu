@@ -64,26 +64,6 @@ __device__ __forceinline__ void gq_cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(src) : "memory");
 }
 
-// tf32 split of an fp32 value: hi = x rounded to tf32, lo = the rest rounded
-// to tf32 (the 3xTF32 scheme: products hi*hi + hi*lo + lo*hi keep fp32
-// accuracy; the dropped lo*lo term is below 2^-22 relative).
-__device__ __forceinline__ void tf32_split(float x, uint32_t& hi, uint32_t& lo) {
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(hi) : "f"(x));
-  const float rest = x - __uint_as_float(hi);
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(lo) : "f"(rest));
-}
-
-// D += A B on the warp's tensor cores: A 16 x 8 (row-major fragment a[4]),
-// B 8 x 8 (b[2]), D 16 x 8 fp32 (d[4]), tf32 inputs.
-__device__ __forceinline__ void mma_tf32_16x8x8(float (&d)[4], const uint32_t (&a)[4],
-                                                const uint32_t (&b)[2]) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
-      "{%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
-}
-
 // The window of tile t of the range, T1 = sum_{g=1..t} E[I, J-g] L^A[J, J-g]^T
 // (32 x 32, fp32-accurate by the 3xTF32 split), into S.T1 ([p][q]).  With
 // lane = 4 gid + tig, an m16n8k8 fragment holds A(gid (+8), tig (+4)),
