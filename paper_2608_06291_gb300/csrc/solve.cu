@@ -419,19 +419,12 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
   // 2P products of 32^3, taken one d at a time.  For d >= 2 the tiles were
   // written by kernels that had completed when this one was launched: their
   // part runs before the wait for the previous kernel (overlapping it), its
-  // operands double-buffered; E[I, J-1] and G[I-1, J] come after.  The
-  // products run on the warps' tensor cores (mma.sync m16n8k8, tf32 operands
-  // split 3xTF32 so the sums keep fp32 accuracy): warp w forms rows
-  // 16 (w >> 1) .. +15 and columns 16 (w & 1) .. +15 of T1 and U as two
-  // 16 x 8 fragments each.  Thread t loads X at rows pr .. pr+3, columns pc,
-  // pc+1.
+  // operands double-buffered; E[I, J-1] and G[I-1, J] come after.  Thread t
+  // forms rows pr .. pr+3, columns pc, pc+1 of T1 and U.
   const int pr = 4 * (t >> 4), pc = 2 * (t & 15);
-  const int gid = lane >> 2, tig = lane & 3, fm0 = 16 * (w >> 1), fn0 = 16 * (w & 1);
-  float t1f[2][4], uf[2][4];
+  float t1[4][2], u[4][2];
 #pragma unroll
-  for (int j = 0; j < 2; ++j)
-#pragma unroll
-    for (int r = 0; r < 4; ++r) t1f[j][r] = uf[j][r] = 0.f;
+  for (int i = 0; i < 4; ++i) t1[i][0] = t1[i][1] = u[i][0] = u[i][1] = 0.f;
   auto fetch_factors = [&](int d, int b) {
     copy_block(&S.u.pro.B[b][2][0][0], lak + d * LEAF_BLOCK_FLOATS, t);
     copy_block(&S.u.pro.B[b][3][0][0], lbk + d * LEAF_BLOCK_FLOATS, t);
@@ -452,39 +445,21 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
                  vg ? a.Gout + (r0 - (int64_t)TILE * d + j) * a.ldx + c0 + i4 : a.Gout, vg);
     }
   };
-  // T1 += E[I, J-d] L^A[J, J-d]^T and U += L^B[I, I-d] G[I-d, J] from buffer b:
-  // T1 = A B with A(p, k) = E^T buffer [k][p], B(k, q) = L^A buffer [k][q];
-  // U likewise with A(p, k) = L^B buffer [k][p], B(k, q) = G buffer [k][q].
-  // Fragment rows gid (+8), A columns / B rows tig (+4), B columns gid.
+  // T1 += E[I, J-d] L^A[J, J-d]^T and U += L^B[I, I-d] G[I-d, J] from buffer b
   auto products = [&](int b) {
+#pragma unroll 2
+    for (int k = 0; k < TILE; ++k) {
+      const float4 ae = *reinterpret_cast<const float4*>(&S.u.pro.B[b][0][k][pr]);
+      const float be0 = S.u.pro.B[b][2][k][pc], be1 = S.u.pro.B[b][2][k][pc + 1];
+      const float4 ab = *reinterpret_cast<const float4*>(&S.u.pro.B[b][3][k][pr]);
+      const float bn0 = S.u.pro.B[b][1][k][pc], bn1 = S.u.pro.B[b][1][k][pc + 1];
+      const float ea[4] = {ae.x, ae.y, ae.z, ae.w}, ba[4] = {ab.x, ab.y, ab.z, ab.w};
 #pragma unroll
-    for (int kk = 0; kk < TILE / 8; ++kk) {
-      const int k0 = 8 * kk;
-      uint32_t eh[4], el[4], lh[4], ll[4];
-      const float(*Be)[KM] = S.u.pro.B[b][0];
-      const float(*Bl)[KM] = S.u.pro.B[b][3];
-      tf32_split(Be[k0 + tig][fm0 + gid], eh[0], el[0]);
-      tf32_split(Be[k0 + tig][fm0 + gid + 8], eh[1], el[1]);
-      tf32_split(Be[k0 + tig + 4][fm0 + gid], eh[2], el[2]);
-      tf32_split(Be[k0 + tig + 4][fm0 + gid + 8], eh[3], el[3]);
-      tf32_split(Bl[k0 + tig][fm0 + gid], lh[0], ll[0]);
-      tf32_split(Bl[k0 + tig][fm0 + gid + 8], lh[1], ll[1]);
-      tf32_split(Bl[k0 + tig + 4][fm0 + gid], lh[2], ll[2]);
-      tf32_split(Bl[k0 + tig + 4][fm0 + gid + 8], lh[3], ll[3]);
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const int n = fn0 + 8 * j + gid;
-        uint32_t ah[2], al[2], gh[2], gl[2];
-        tf32_split(S.u.pro.B[b][2][k0 + tig][n], ah[0], al[0]);
-        tf32_split(S.u.pro.B[b][2][k0 + tig + 4][n], ah[1], al[1]);
-        tf32_split(S.u.pro.B[b][1][k0 + tig][n], gh[0], gl[0]);
-        tf32_split(S.u.pro.B[b][1][k0 + tig + 4][n], gh[1], gl[1]);
-        mma_tf32_16x8x8(t1f[j], el, ah);
-        mma_tf32_16x8x8(t1f[j], eh, al);
-        mma_tf32_16x8x8(t1f[j], eh, ah);
-        mma_tf32_16x8x8(uf[j], ll, gh);
-        mma_tf32_16x8x8(uf[j], lh, gl);
-        mma_tf32_16x8x8(uf[j], lh, gh);
+      for (int i = 0; i < 4; ++i) {
+        t1[i][0] = fmaf(ea[i], be0, t1[i][0]);
+        t1[i][1] = fmaf(ea[i], be1, t1[i][1]);
+        u[i][0] = fmaf(ba[i], bn0, u[i][0]);
+        u[i][1] = fmaf(ba[i], bn1, u[i][1]);
       }
     }
   };
@@ -548,27 +523,21 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
   cp_async_commit();
   cp_async_wait_group<0>();
   leaf_sync();   // factor blocks and the last window tiles in shared memory
-  if (P >= 1) products(2);
+  if (P >= 1) {
+    products(2);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      S.T1s[pr + i][pc] = t1[i][0];
+      S.T1s[pr + i][pc + 1] = t1[i][1];
+      xv[i][0] += u[i][0];
+      xv[i][1] += u[i][1];
+    }
+  }
   leaf_sync();   // the wavefront's arrays overlay the prologue's
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     S.Xs[pr + i][pc] = xv[i][0];
     S.Xs[pr + i][pc + 1] = xv[i][1];
-  }
-  if (P >= 1) {
-    leaf_sync();   // X in place: add U to it, T1 is G's initial value
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      const int r = fm0 + gid, c = fn0 + 8 * j + 2 * tig;
-      S.T1s[r][c] = t1f[j][0];
-      S.T1s[r][c + 1] = t1f[j][1];
-      S.T1s[r + 8][c] = t1f[j][2];
-      S.T1s[r + 8][c + 1] = t1f[j][3];
-      S.Xs[r][c] += uf[j][0];
-      S.Xs[r][c + 1] += uf[j][1];
-      S.Xs[r + 8][c] += uf[j][2];
-      S.Xs[r + 8][c + 1] += uf[j][3];
-    }
   }
 
   if (t < TILE)
