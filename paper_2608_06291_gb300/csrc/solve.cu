@@ -506,19 +506,27 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
       }
     }
   }
+  // X at this thread's product positions: rows pr .. pr+3, columns pc, pc+1.
+  // Inside a block only the leaves run, each writing its own anti-diagonal's
+  // tiles, so for P >= 1 this tile's X was last written by the band product
+  // before the block, two or more kernels ago: it is loaded before the wait.
+  float xv[4][2];
+  auto load_x = [&]() {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 x2 =
+          __ldcg(reinterpret_cast<const float2*>(a.X + (r0 + pr + i) * a.ldx + c0 + pc));
+      xv[i][0] = x2.x;
+      xv[i][1] = x2.y;
+    }
+  };
+  if (P >= 1 || !PDL) load_x();
   if (PDL) {
     pdl_wait();
     pdl_trigger();
   }
   stamp_begin(a.stamp);
-  // X at this thread's product positions: rows pr .. pr+3, columns pc, pc+1
-  float xv[4][2];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float2 x2 = __ldcg(reinterpret_cast<const float2*>(a.X + (r0 + pr + i) * a.ldx + c0 + pc));
-    xv[i][0] = x2.x;
-    xv[i][1] = x2.y;
-  }
+  if (P == 0 && PDL) load_x();
   if (P >= 1) fetch_tiles(1, 2);
   cp_async_commit();
   cp_async_wait_group<0>();
