@@ -333,10 +333,11 @@ void bakron_autotune_clear(void);
  *
  * Scratch: a fixed array of BAKRON_NOALLOC_SCRATCH_BYTES (64 MiB) inside the
  * library, on every GPU that loads it, held until the process exits.  A
- * problem fits when the solve's scratch, 256 + 20 * mp * np bytes (mp, np: m
- * and n rounded up to multiples of 128), is at most 64 MiB -- e.g. 1792 x
- * 1792 or 2048 x 1536; larger problems are rejected with BAKRON_ERR_WORKSPACE
- * before anything is enqueued (sides above 131072 with BAKRON_ERR_INVALID_ARG,
+ * problem fits when the solve's scratch, bakron_workspace_bytes(m, n)'s solve
+ * part -- 20 * mp * np bytes (mp, np: m and n rounded up to multiples of 128)
+ * plus 4 bytes per 32 x 32 tile and 33 KiB of counters and status -- is at
+ * most 64 MiB: e.g. 1792 x 1792 or 2048 x 1536; larger problems are rejected
+ * with BAKRON_ERR_WORKSPACE before anything is enqueued (sides above 131072 with BAKRON_ERR_INVALID_ARG,
  * as bakron_solve does).  The call allocates nothing: no cudaMalloc/cudaFree,
  * no allocating library routine.
  *

@@ -457,7 +457,7 @@ def bakron_solve_noalloc(W, f: Factors, bits: int, group_size: int = 0,
                          prerounding: bool = False, sync: bool = True, out=None, stream=None):
     """bakron_solve without a workspace argument, for callers that cannot
     allocate device scratch: the library's fixed 64 MiB array is used instead
-    (problems whose scratch, 20 * mp * np + 256 bytes, fits).  Outputs are
+    (problems whose solve scratch, about 20 * mp * np bytes, fits).  Outputs are
     allocated here unless ``out`` is given."""
     if not W.is_cuda or W.dim() != 2 or W.stride(1) != 1:
         raise ValueError("W must be a 2-D CUDA tensor with unit column stride")

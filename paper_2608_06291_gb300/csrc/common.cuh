@@ -87,9 +87,13 @@ int build_leaf_blocks(const FactorLayout& fl, char* factors, cudaStream_t s);
 // M = L^B E; M is the stage-1 band product.  The M hi plane doubles as E^T in
 // fp32 for the leaves: a leaf block reads back only E tiles written inside the
 // block, and M is written only by band products, which run between blocks.
+// Then the leaves' dataflow words (one launch per block of leaves): a tile
+// counter per block, indexed by the block's first anti-diagonal, and a
+// readiness flag per padded tile; zeroed at the start of every solve.
+constexpr int FLOW_COUNTERS = 8192;   // > the anti-diagonals of the largest problem (2 * 4096)
 struct SolveLayout {
   int64_t mp, np;
-  size_t off_status, off_X, off_EtH, off_EtL, off_MH, off_ML, bytes;
+  size_t off_status, off_X, off_EtH, off_EtL, off_MH, off_ML, off_flow, flow_bytes, bytes;
   SolveLayout(int m, int n) {
     mp = round_up(m, PAD);
     np = round_up(n, PAD);
@@ -100,7 +104,9 @@ struct SolveLayout {
     off_EtL = align256(off_EtH + plane);
     off_MH = align256(off_EtL + plane);
     off_ML = align256(off_MH + plane);
-    bytes = align256(off_ML + plane);
+    off_flow = align256(off_ML + plane);
+    flow_bytes = size_t(FLOW_COUNTERS + (mp / TILE) * (np / TILE)) * 4;
+    bytes = align256(off_flow + flow_bytes);
   }
 };
 

@@ -378,6 +378,53 @@ __device__ __forceinline__ void copy_block(float* dst, const float* src, int t) 
   for (int c = t; c < CHUNKS; c += LEAF_THREADS) cp_async16(dst + 4 * c, src + 4 * c, true);
 }
 
+// How a leaf learns that its inputs are ready.
+//   LEAF_PDL   one launch per anti-diagonal: programmatic dependent launch
+//              (everything the previous leaf wrote is ready at pdl_wait);
+//   LEAF_PLAIN inside a persistent subtree, after a grid-wide barrier;
+//   LEAF_FLOW  one launch per block of anti-diagonals, persistent CTAs: a tile
+//              waits only for the tiles its window reads, through per-tile
+//              flags that each tile sets as soon as its fp32 errors and final
+//              G are in memory (before the rest of its epilogue).
+constexpr int LEAF_PDL = 0, LEAF_PLAIN = 1, LEAF_FLOW = 2;
+
+// Per-tile readiness flags of a block launch (LEAF_FLOW).
+struct FlowCtx {
+  unsigned* done;        // per padded tile I * ntp + J: nonzero once published
+  int ntp;
+  long long spin_cycles; // bound of every wait
+};
+
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Thread 0 waits, for at most fc.spin_cycles, until tiles (I1, J1) and
+// (I2, J2) are published (a tile with a negative coordinate does not exist
+// and counts as published), then the leaf's threads meet at its barrier.
+// A wait that runs out records BAKRON_ERR_TIMEOUT and the leaf goes on.
+__device__ __forceinline__ void flow_wait(const FlowCtx& fc, int I1, int J1, int I2, int J2,
+                                          int* status) {
+  if (threadIdx.x == 0) {
+    const int is[2] = {I1, I2}, js[2] = {J1, J2};
+    for (int u = 0; u < 2; ++u) {
+      if (is[u] < 0 || js[u] < 0) continue;
+      const unsigned* f = fc.done + (int64_t)is[u] * fc.ntp + js[u];
+      if (ld_acquire_u32(f)) continue;
+      const long long t0 = clock64();
+      while (!ld_acquire_u32(f)) {
+        if (clock64() - t0 > fc.spin_cycles) {
+          raise_status(status, BAKRON_ERR_TIMEOUT);
+          break;
+        }
+      }
+    }
+  }
+  leaf_sync();
+}
+
 // Rounds tile (I, J); run by threads 0 .. LEAF_THREADS-1 of the CTA.  With
 // PDL, the factor blocks and the grid (read-only during the solve, the grid
 // written by the solve's first kernel, more than one kernel ago), and the
@@ -395,9 +442,15 @@ __device__ __forceinline__ void copy_block(float* dst, const float* src, int t) 
 //     U = sum_dp L^B[I,I-dp] N_dp,   N_dp = sum_g E[I-dp,J-g] L^A[J,J-g]^T,
 // and N_dp is the final G of tile (I - dp, J), which that tile's leaf leaves
 // behind (its window is P - dp).  Tiles outside the matrix are zeros.
-template <bool PDL, int P>
-__device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafSmem& S) {
+// In LEAF_FLOW mode the window's tiles come from the same launch: the tiles
+// two anti-diagonals back are waited for before the products of d >= 2, the
+// two neighbours before those of d = 1, and `first` (the CTA's first tile)
+// also waits for the previous kernel.
+template <int MODE, int P>
+__device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafSmem& S,
+                                          const FlowCtx* fc = nullptr, bool first = false) {
   static_assert(P >= 0 && P <= LEAF_WINDOW, "window");
+  constexpr bool PDL = MODE == LEAF_PDL;
   static_assert(LEAF_PER_THREAD * LEAF_THREADS == TILE * TILE, "whole tile per pass");
   const int t = threadIdx.x, w = t >> 5, lane = t & 31;
   const int64_t r0 = (int64_t)I * TILE, c0 = (int64_t)J * TILE;
@@ -485,6 +538,13 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
                                              LEAF_R + (float)a.qmax - zv[k]);
   }
   for (int e = t; e < 4 * LEAF_ROWS_PADDED; e += LEAF_THREADS) (&S.Ebr[0][0])[e] = 0.f;
+  if constexpr (MODE == LEAF_FLOW) {
+    if (first) {   // X was written by the kernel before this launch
+      pdl_wait();
+      pdl_trigger();
+    }
+    if (P >= 2) flow_wait(*fc, I, J - 2, I - 2, J, a.status);
+  }
   if (P >= 2) {
 #pragma unroll
     for (int d = 2; d <= P && d <= 3; ++d) {
@@ -521,9 +581,11 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     }
   };
   if (P >= 1 || !PDL) load_x();
-  if (PDL) {
+  if constexpr (PDL) {
     pdl_wait();
     pdl_trigger();
+  } else if constexpr (MODE == LEAF_FLOW) {
+    if (P >= 1) flow_wait(*fc, I, J - 1, I - 1, J, a.status);
   }
   stamp_begin(a.stamp);
   if (P == 0 && PDL) load_x();
@@ -748,6 +810,19 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     S.u.w.EsT[c][r] = S.u.w.XE[r][c].y;
   }
   leaf_sync();
+  if constexpr (MODE == LEAF_FLOW) {
+    // what the tiles right of and below this one read (E^T in fp32; the final
+    // G the helpers stored above), then the flag, then the rest
+    for (int e = t; e < TILE * TILE; e += LEAF_THREADS) {
+      const int r = e / TILE, c = e % TILE;
+      a.EtF[(c0 + r) * a.ldt + r0 + c] = S.u.w.EsT[r][c];
+    }
+    leaf_sync();
+    if (t == 0) {
+      __threadfence();
+      atomicExch(fc->done + (int64_t)I * fc->ntp + J, 1u);
+    }
+  }
   bool bad = false;
   for (int e = t; e < TILE * TILE; e += LEAF_THREADS) {
     const int r = e / TILE, c = e % TILE;
@@ -760,21 +835,22 @@ __device__ __forceinline__ void leaf_tile(const LeafArgs& a, int I, int J, LeafS
     const int64_t o = (c0 + r) * a.ldt + r0 + c;
     a.EtH[o] = hi;
     a.EtL[o] = ev - hi;
-    a.EtF[o] = ev;
+    if constexpr (MODE != LEAF_FLOW) a.EtF[o] = ev;
   }
   if (bad) raise_status(a.status, BAKRON_ERR_NONFINITE);
   leaf_sync();   // shared memory free for the next tile of this CTA
   stamp_end(a.stamp);
 }
 
-// leaf_tile<false, P> for a window known at run time (0 <= h <= LEAF_WINDOW)
-template <int P>
-__device__ __forceinline__ void leaf_tile_window(int h, const LeafArgs& a, int I, int J, LeafSmem& S) {
+// leaf_tile<MODE, P> for a window known at run time (0 <= h <= LEAF_WINDOW)
+template <int MODE, int P>
+__device__ __forceinline__ void leaf_tile_window(int h, const LeafArgs& a, int I, int J, LeafSmem& S,
+                                                 const FlowCtx* fc = nullptr, bool first = false) {
   if (h == P || P == LEAF_WINDOW) {
-    leaf_tile<false, P>(a, I, J, S);
+    leaf_tile<MODE, P>(a, I, J, S, fc, first);
     return;
   }
-  if constexpr (P < LEAF_WINDOW) leaf_tile_window<P + 1>(h, a, I, J, S);
+  if constexpr (P < LEAF_WINDOW) leaf_tile_window<MODE, P + 1>(h, a, I, J, S, fc, first);
 }
 
 // One CTA per tile of tile anti-diagonal K; P: the leaf's window.
@@ -783,7 +859,43 @@ __global__ void __launch_bounds__(LEAF_THREADS) k_leaf(int K, LeafArgs a) {
   extern __shared__ __align__(16) unsigned char leaf_smem[];
   LeafSmem& S = *reinterpret_cast<LeafSmem*>(leaf_smem);
   const int I = max(0, K - (a.Nt - 1)) + blockIdx.x;
-  leaf_tile<true, P>(a, I, K - I, S);
+  leaf_tile<LEAF_PDL, P>(a, I, K - I, S);
+}
+
+// A whole block of leaves [k, l) in one launch (LEAF_FLOW).  The block's
+// tiles are numbered by anti-diagonal, then row; CTAs take them in that order
+// from a counter, and a tile waits only for tiles numbered before it, which
+// CTAs already running hold: the lowest unfinished tile can always proceed.
+struct FlowArgs {
+  LeafArgs leaf;
+  FlowCtx fc;
+  int k, l;
+  unsigned* claim;   // this launch's tile counter (zero before the launch)
+};
+
+__global__ void __launch_bounds__(LEAF_THREADS) k_leaf_flow(const __grid_constant__ FlowArgs F) {
+  extern __shared__ __align__(16) unsigned char leaf_smem[];
+  LeafSmem& S = *reinterpret_cast<LeafSmem*>(leaf_smem);
+  __shared__ int tile_s;
+  const int Mt = F.leaf.Mt, Nt = F.leaf.Nt;
+  bool first = true;
+  for (;;) {
+    if (threadIdx.x == 0) tile_s = (int)atomicAdd(F.claim, 1u);
+    leaf_sync();
+    int rem = tile_s, K = F.k, I = -1;
+    leaf_sync();   // every thread has read tile_s before the next claim
+    for (; K < F.l; ++K) {
+      const int ilo = max(0, K - (Nt - 1)), cnt = min(K, Mt - 1) - ilo + 1;
+      if (rem < cnt) {
+        I = ilo + rem;
+        break;
+      }
+      rem -= cnt;
+    }
+    if (I < 0) break;
+    leaf_tile_window<LEAF_FLOW, 0>(K - F.k, F.leaf, I, K - I, S, &F.fc, first);
+    first = false;
+  }
 }
 
 // ------------------------------------------------------- band products (SIMT)
@@ -1113,7 +1225,7 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_subtree(const __grid_constant_
       const int ilo = max(0, P.k - (Nt - 1)), ihi = min(P.k, Mt - 1);
       if (threadIdx.x < LEAF_THREADS)
         for (int I = ilo + (int)blockIdx.x; I <= ihi; I += gridDim.x) {
-          leaf_tile_window<0>(P.h, A.leaf, I, P.k - I, S.leaf);
+          leaf_tile_window<LEAF_PLAIN, 0>(P.h, A.leaf, I, P.k - I, S.leaf);
         }
     } else {
       const int row_lo = max(0, P.h - (Nt - 1)), row_hi = min(Mt - 1, P.l - 1);
@@ -1175,6 +1287,11 @@ struct SolveArgs {
   int subtree_max;      // ranges spanning <= this many: one persistent cooperative launch
   int leaf_block;       // ranges spanning <= this many: a block of leaves (1 .. LEAF_WINDOW + 1)
   int subtree_grid;     // CTAs a cooperative launch may hold (resident at once)
+  bool leaf_flow;       // a block of leaves is one dataflow launch (k_leaf_flow)
+  int flow_grid;        // CTAs of k_leaf_flow resident at once
+  unsigned* flow_claim; // per block (by first anti-diagonal): tile counter
+  unsigned* flow_done;  // per padded tile: published flag
+  int ntp;              // padded tile columns
   long long spin_cycles;
   bool tc_ready;
   bool profiling;
@@ -1249,6 +1366,8 @@ static cudaError_t ensure_leaf_attrs() {
   cudaError_t e = set_leaf_smem<0>(sm);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(k_subtree, cudaFuncAttributeMaxDynamicSharedMemorySize, ss);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_leaf_flow, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
   if (e == cudaSuccess) done = true;
   return e;
 }
@@ -1356,7 +1475,56 @@ static void subtree(SolveArgs& a, int k, int l) {
   note(a, cudaLaunchKernelEx(&cfg, k_subtree, A));
 }
 
+// CTAs of k_leaf_flow resident at once on the current device (occupancy x
+// SMs), queried once per device; -1 on a CUDA error.
+static int flow_capacity() {
+  static std::mutex mu;
+  static int cap[64];
+  static bool done[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return -1;
+  std::lock_guard<std::mutex> lk(mu);
+  if (dev < 64 && done[dev]) return cap[dev];
+  int sms = 0, per_sm = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return -1;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_leaf_flow, LEAF_THREADS,
+                                                    sizeof(LeafSmem)) != cudaSuccess)
+    return -1;
+  const int c = sms * (per_sm > 0 ? per_sm : 1);
+  if (dev < 64) {
+    cap[dev] = c;
+    done[dev] = true;
+  }
+  return c;
+}
+
+// The leaves of anti-diagonals [k, l) as one dataflow launch.
+static void leaf_block_flow(SolveArgs& a, int k, int l) {
+  int tiles = 0;
+  double flops = 0.0;
+  for (int K = k; K < l; ++K) {
+    const int cnt = min(K, a.Mt - 1) - max(0, K - (a.Nt - 1)) + 1;
+    tiles += cnt;
+    flops += 2.0 * TILE * TILE * TILE * (1 + window_products(K - k)) * cnt;
+  }
+  if (tiles <= 0) return;
+  LaunchScope ls(kFamLeaf, a.s, flops);
+  FlowArgs F;
+  F.leaf = a.la;
+  F.leaf.stamp = ls.stamp();
+  F.fc = FlowCtx{a.flow_done, a.ntp, a.spin_cycles};
+  F.k = k;
+  F.l = l;
+  F.claim = a.flow_claim + k;
+  note(a, launch_pdl(k_leaf_flow, dim3(min(tiles, a.flow_grid)), dim3(LEAF_THREADS),
+                     sizeof(LeafSmem), a.s, F));
+}
+
 static void rec(SolveArgs& a, int k, int l) {
+  if (l - k <= a.leaf_block && a.leaf_flow) {
+    leaf_block_flow(a, k, l);
+    return;
+  }
   if (l - k <= a.leaf_block) {
     // a block of leaves: leaf K applies what anti-diagonals k .. K-1 send it
     // (the Alg. 5 nodes inside [k, l)), so no band launch is needed here
@@ -1440,6 +1608,15 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
       a.subtree_grid = cap;
     }
     a.spin_cycles = spin_cycles_from_env();
+    a.leaf_flow = tu.leaf_flow != 0;
+    a.flow_grid = 0;
+    a.flow_claim = (unsigned*)(ws + sl.off_flow);
+    a.flow_done = a.flow_claim + FLOW_COUNTERS;
+    a.ntp = (int)(sl.np / TILE);
+    if (a.leaf_flow) {
+      a.flow_grid = flow_capacity();
+      if (a.flow_grid <= 0) return BAKRON_ERR_CUDA;
+    }
     a.tc_ready = false;
     if (a.tc_min_band > 0) {
       a.tco = TcOperands{a.mp, a.np, a.Mt, a.Nt, a.LBH, a.LBL, a.LAH, a.LAL,
@@ -1453,6 +1630,7 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
     BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_status + 64, 0, 256 - 64, s));
   else
     BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_status, 0, 256, s));
+  if (a.leaf_flow) BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_flow, 0, sl.flow_bytes, s));
   if (!grid_given) launch_grid(W, wdt, m, n, ldw, a.gsz, a.G, a.qmax, scales, zeros, s);
   {
     const int rc = launch_init(W, wdt, m, n, ldw, a.X, a.mp, a.np, s);

@@ -42,6 +42,7 @@ Tuning tuning_for(int m, int n) {
   env_override("BAKRON_FUSED_MAX_BAND", t.fused_max_band);
   env_override("BAKRON_SUBTREE_MAX", t.subtree_max);
   env_override("BAKRON_LEAF_BLOCK", t.leaf_block);
+  env_override("BAKRON_LEAF_FLOW", t.leaf_flow);
   return t;
 }
 
@@ -72,12 +73,13 @@ int bakron_autotune(const void* W, int wdtype, int m, int n, int64_t ldw, const 
     return BAKRON_ERR_CUDA;
   }
   Tuning best = kDefaultTuning;
+  env_override("BAKRON_LEAF_FLOW", best.leaf_flow);   // not tuned: the default or the environment
   float best_t = -1.f;
   int rc = BAKRON_OK;
   for (int tc : kTc) {
     for (int fu : kFused) {
      for (int lb : kBlock) {
-      const Tuning cand{tc, fu, 0, lb};
+      const Tuning cand{tc, fu, 0, lb, best.leaf_flow};
       float t_min = -1.f;
       for (int rep = 0; rep < 3 && rc == BAKRON_OK; ++rep) {   // rep 0 warms up
         if (cudaEventRecord(e0, s) != cudaSuccess) { rc = BAKRON_ERR_CUDA; break; }

@@ -55,12 +55,12 @@ def test_noalloc_scratch_limit():
     L = P.lib()
     t = torch.zeros(16, dtype=torch.uint8, device="cuda")
     p = t.data_ptr()
-    # 4096 x 4096 needs 20 * 4096^2 + 256 bytes > 64 MiB: refused on the host
+    # 4096 x 4096 needs more than 20 * 4096^2 bytes > 64 MiB: refused on the host
     rc = L.bakron_solve_noalloc(p, 0, 4096, 4096, 4096, p, 4, 0, p, p, p, None, 1, None)
     assert rc == 5
     assert P.strerror(rc) == "workspace too small"
-    # 1792 x 1792 (20 * 1792^2 + 256 bytes) fits and runs; one more column pads
-    # n to 1920 and no longer fits
+    # 1792 x 1792 (20 * 1792^2 bytes plus the tile flags and counters) fits and
+    # runs; one more column pads n to 1920 and no longer fits
     W, fac, bits, group = _problem(1792, 1792, 73, 4, 0)
     _same_solve(W, fac, bits, group)
     rc = L.bakron_solve_noalloc(p, 0, 1792, 1793, 1793, p, 4, 0, p, p, p, None, 1, None)
