@@ -419,6 +419,7 @@ __device__ __forceinline__ void flow_wait(const FlowCtx& fc, int I1, int J1, int
           raise_status(status, BAKRON_ERR_TIMEOUT);
           break;
         }
+        __nanosleep(64);   // leave the issue slots to the wavefronts sharing the SM
       }
     }
   }

@@ -307,11 +307,26 @@ __host__ __device__ inline bool band_row_span(int mode, int k, int h, int l, int
   return true;
 }
 
+// CTAs run in launch order, so consecutive ones should share operands in L2:
+// the band stages walk their grid in groups of RASTER_ROWS row blocks, column
+// by column inside a group (an A row block is then reused by the ~150
+// resident CTAs of its group, and a B column block by RASTER_ROWS of them,
+// instead of every B block coming from DRAM once per row block).
+constexpr int RASTER_ROWS = 8;
+
 // Returns false if the block has no work at all (beyond its row's span).
 __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
   // the blocks with the longest K ranges first (they sit at high rows, and
   // in stage 2 at high columns): less of a tail when the grid runs in waves
-  b.rb = P.row0 + (P.mode == MODE_DENSE ? blockIdx.y : gridDim.y - 1 - blockIdx.y);
+  int bx = (int)blockIdx.x, by = (int)blockIdx.y;
+  if (P.mode != MODE_DENSE && P.mode != MODE_GRAM) {
+    const int W = (int)gridDim.x, H = (int)gridDim.y;
+    const int L = by * W + bx, grp = L / (RASTER_ROWS * W), in = L - grp * RASTER_ROWS * W;
+    const int gh = min(RASTER_ROWS, H - grp * RASTER_ROWS);   // rows of this group
+    by = grp * RASTER_ROWS + in % gh;
+    bx = in / gh;
+  }
+  b.rb = P.row0 + (P.mode == MODE_DENSE ? by : (int)gridDim.y - 1 - by);
   if (P.mode == MODE_DENSE) {
     b.cb = blockIdx.x;
     b.k0 = 0;
@@ -332,7 +347,7 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
   }
   int cb_lo, cb_hi;
   if (!band_row_span(P.mode, P.k, P.h, P.l, P.Mt, P.Nt, b.rb, cb_lo, cb_hi)) return false;
-  b.cb = P.mode == MODE_STAGE2 ? cb_hi - (int)blockIdx.x : cb_lo + (int)blockIdx.x;
+  b.cb = P.mode == MODE_STAGE2 ? cb_hi - bx : cb_lo + bx;
   if (b.cb > cb_hi || b.cb < cb_lo) return false;
   if (P.mode == MODE_COLS) {   // K = the tile columns of S1, the same for every block
     b.k0 = P.k;

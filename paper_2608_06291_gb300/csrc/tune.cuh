@@ -16,7 +16,7 @@ struct Tuning {
 // Defaults: 4096 x 4096 solves are fastest with blocks of up to 8 leaves
 // (no node narrower than 9 anti-diagonals is left) and tensor cores for
 // every node above them.
-constexpr Tuning kDefaultTuning{6, 2, 0, 8, 1};
+constexpr Tuning kDefaultTuning{6, 2, 0, 8, 0};
 
 // Thresholds for an m x n solve on the current device: the table entry if
 // bakron_autotune stored one, else the defaults; each BAKRON_TC_MIN_BAND,
