@@ -253,3 +253,12 @@ def test_deterministic_and_async():
     assert P.bakron_read_status(ws) == 0
     assert torch.equal(a, b)
     np.testing.assert_array_equal(a.cpu().numpy(), r1["codes"])
+
+
+def test_dataflow_leaf_blocks_match_oracle(monkeypatch):
+    """The dataflow mode of the leaves (one launch per block of leaves, tiles
+    waiting on per-tile flags; off by default) gives the oracle's codes too."""
+    monkeypatch.setenv("BAKRON_LEAF_FLOW", "1")
+    for block in ("4", "8", "16"):
+        monkeypatch.setenv("BAKRON_LEAF_BLOCK", block)
+        _assert_parity(_solve_small(97, 131, 41 + int(block), bits=4))
