@@ -89,6 +89,7 @@ struct TcParams {
   int dreal;
   int a_exact, b_exact;
   unsigned long long* stamp;   // timeline stamp slot of the launch (null: none)
+  int raster;                  // band stages: row blocks per launch-order group (>= 1)
 };
 
 // Kernel variants (compile time, so that the band products' issue loop
@@ -312,7 +313,7 @@ __host__ __device__ inline bool band_row_span(int mode, int k, int h, int l, int
 // by column inside a group (an A row block is then reused by the ~150
 // resident CTAs of its group, and a B column block by RASTER_ROWS of them,
 // instead of every B block coming from DRAM once per row block).
-constexpr int RASTER_ROWS = 8;
+constexpr int RASTER_ROWS = 8;   // default group height (BAKRON_TC_RASTER overrides it)
 
 // Returns false if the block has no work at all (beyond its row's span).
 __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
@@ -321,9 +322,10 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
   int bx = (int)blockIdx.x, by = (int)blockIdx.y;
   if (P.mode != MODE_DENSE && P.mode != MODE_GRAM) {
     const int W = (int)gridDim.x, H = (int)gridDim.y;
-    const int L = by * W + bx, grp = L / (RASTER_ROWS * W), in = L - grp * RASTER_ROWS * W;
-    const int gh = min(RASTER_ROWS, H - grp * RASTER_ROWS);   // rows of this group
-    by = grp * RASTER_ROWS + in % gh;
+    const int R = P.raster > 0 ? P.raster : RASTER_ROWS;
+    const int L = by * W + bx, grp = L / (R * W), in = L - grp * R * W;
+    const int gh = min(R, H - grp * R);   // rows of this group
+    by = grp * R + in % gh;
     bx = in / gh;
   }
   b.rb = P.row0 + (P.mode == MODE_DENSE ? by : (int)gridDim.y - 1 - by);
@@ -969,11 +971,19 @@ bool tc_band_maps(TcMaps& maps, const TcOperands& op) {
   return ok;
 }
 
+// Group height of the band stages' launch order (BAKRON_TC_RASTER, read per call).
+static int raster_rows() {
+  const char* e = getenv("BAKRON_TC_RASTER");
+  const int v = e ? atoi(e) : 0;
+  return v >= 1 ? v : RASTER_ROWS;
+}
+
 int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, int h, int l,
                   cudaStream_t s, unsigned long long* stamp) {
   if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
   TcParams P{};
   P.stamp = stamp;
+  P.raster = raster_rows();
   P.mode = stage == 1 ? MODE_STAGE1 : MODE_STAGE2;
   P.k = k; P.h = h; P.l = l;
   P.Mt = op.Mt; P.Nt = op.Nt;
@@ -1013,6 +1023,7 @@ int tc_cols_stage(const TcMaps& maps, const TcOperands& op, int k, int h, int l,
   if (k >= h || h >= l) return BAKRON_OK;
   TcParams P{};
   P.stamp = stamp;
+  P.raster = raster_rows();
   P.mode = MODE_COLS;
   P.k = k; P.h = h; P.l = l;
   P.Mt = op.Mt; P.Nt = op.Nt;
