@@ -458,6 +458,14 @@ int bakron_diag_leaf_chain(const void* W, int wdtype, const void* factors,
 /* Static description of a status code. */
 const char* bakron_strerror(int status);
 
+/* bakron_last_cuda_error -- the CUDA runtime error behind the last
+ * BAKRON_ERR_CUDA that a call of this library returned on the calling host
+ * thread (0 if none).  Where the pointers are non-null, *name receives the
+ * error's name (static storage), *where the library source file and *line the
+ * line that saw it.  Host-only, never fails; the record is overwritten by the
+ * next failure and not cleared by successes. */
+int bakron_last_cuda_error(const char** name, const char** where, int* line);
+
 #ifdef __cplusplus
 }
 #endif

@@ -16,5 +16,6 @@ from .bakron import (BakronError, Factors, alloc_workspace, bakron_diag_gemm_tf3
                      bakron_profile_launch_stamps,
                      bakron_read_status, bakron_set_factors, bakron_solve, bakron_solve_gptq,
                      bakron_solve_noalloc, bakron_read_status_noalloc,
-                     dequantize, factors_bytes, lib, library_path, strerror, workspace_bytes)
+                     bakron_last_cuda_error, dequantize, factors_bytes, lib, library_path,
+                     strerror, workspace_bytes)
 from .buildlib import build  # noqa: F401

@@ -22,7 +22,12 @@ _lib = None
 class BakronError(RuntimeError):
     def __init__(self, status: int, what: str):
         self.status = status
-        super().__init__(f"{what}: {strerror(status)} (status {status})")
+        detail = ""
+        if status == ERR_CUDA and _lib is not None:
+            code, name, where, line = last_cuda_error()
+            if code:
+                detail = f" [{name} at {where}:{line}]"
+        super().__init__(f"{what}: {strerror(status)} (status {status}){detail}")
 
 
 def library_path() -> str:
@@ -111,12 +116,26 @@ def lib() -> ctypes.CDLL:
     L.bakron_diag_mma_rate.restype = i32
     L.bakron_strerror.argtypes = [i32]
     L.bakron_strerror.restype = ctypes.c_char_p
+    L.bakron_last_cuda_error.argtypes = [ctypes.POINTER(ctypes.c_char_p),
+                                         ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(i32)]
+    L.bakron_last_cuda_error.restype = i32
     _lib = L
     return L
 
 
 def strerror(status: int) -> str:
     return lib().bakron_strerror(int(status)).decode()
+
+
+def bakron_last_cuda_error():
+    """(code, name, source file, line) of the CUDA error behind the last
+    ERR_CUDA this thread got from the library (code 0: none)."""
+    name, where, line = ctypes.c_char_p(), ctypes.c_char_p(), ctypes.c_int32()
+    code = lib().bakron_last_cuda_error(ctypes.byref(name), ctypes.byref(where), ctypes.byref(line))
+    return (int(code), (name.value or b"").decode(), (where.value or b"").decode(), int(line.value))
+
+
+last_cuda_error = bakron_last_cuda_error
 
 
 def _ptr(t):

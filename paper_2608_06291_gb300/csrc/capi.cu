@@ -51,6 +51,20 @@ __global__ void k_export(const float* hi, const float* lo, int64_t Lp, int d, fl
 
 static unsigned nblocks(int64_t work, int threads) { return (unsigned)((work + threads - 1) / threads); }
 
+thread_local cudaError_t t_cuda_err = cudaSuccess;
+thread_local const char* t_cuda_file = nullptr;
+thread_local int t_cuda_line = 0;
+
+int cuda_fail(cudaError_t e, const char* file, int line) {
+  t_cuda_err = e;
+  const char* base = file;
+  for (const char* c = file; c && *c; ++c)
+    if (*c == '/') base = c + 1;
+  t_cuda_file = base;
+  t_cuda_line = line;
+  return BAKRON_ERR_CUDA;
+}
+
 }  // namespace bakron
 
 using namespace bakron;
@@ -213,6 +227,14 @@ int bakron_diag_leaf_chain(const void* W, int wdtype, const void* factors, uint8
   BK_CUDA_OK(cudaStreamSynchronize(s));
   *cycles_per_step = (double)(h[1] - h[0]) / (2 * TILE - 1);
   return bakron_read_status(workspace, stream);
+}
+
+int bakron_last_cuda_error(const char** name, const char** where, int* line) {
+  const int code = (int)t_cuda_err;
+  if (name) *name = cudaGetErrorName(t_cuda_err);
+  if (where) *where = t_cuda_file ? t_cuda_file : "";
+  if (line) *line = t_cuda_line;
+  return code;
 }
 
 const char* bakron_strerror(int status) {

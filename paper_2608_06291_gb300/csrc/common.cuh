@@ -200,8 +200,22 @@ __device__ inline void raise_status(int* status, int code) {
 
 }  // namespace bakron
 
-#define BK_CUDA_OK(expr)                                   \
-  do {                                                     \
-    cudaError_t err__ = (expr);                            \
-    if (err__ != cudaSuccess) return BAKRON_ERR_CUDA;      \
+namespace bakron {
+// Records, for the calling host thread, the CUDA runtime error behind a
+// BAKRON_ERR_CUDA and where the library saw it (bakron_last_cuda_error);
+// returns BAKRON_ERR_CUDA.
+int cuda_fail(cudaError_t e, const char* file, int line);
+}  // namespace bakron
+
+#define BK_CUDA_OK(expr)                                                      \
+  do {                                                                        \
+    cudaError_t err__ = (expr);                                               \
+    if (err__ != cudaSuccess) return ::bakron::cuda_fail(err__, __FILE__, __LINE__); \
   } while (0)
+
+// BAKRON_OK, or BAKRON_ERR_CUDA with the error recorded.
+#define BK_CUDA_RC(expr)                                                      \
+  ([&]() -> int {                                                             \
+    cudaError_t err__ = (expr);                                               \
+    return err__ == cudaSuccess ? BAKRON_OK : ::bakron::cuda_fail(err__, __FILE__, __LINE__); \
+  }())

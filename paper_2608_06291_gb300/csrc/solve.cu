@@ -1317,7 +1317,7 @@ static void band_tile_products(const SolveArgs& a, int k, int h, int l, double& 
 }
 
 static void note(SolveArgs& a, cudaError_t e) {
-  if (e != cudaSuccess) a.rc = BAKRON_ERR_CUDA;
+  if (e != cudaSuccess) a.rc = cuda_fail(e, __FILE__, __LINE__);
 }
 
 // Leaf of anti-diagonal K; `window`: how many anti-diagonals before it (in
@@ -1595,7 +1595,7 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
                   a.MH, a.ML, a.np, a.X, a.np, nullptr};
   a.profiling = profiling_on();
   {
-    if (ensure_leaf_attrs() != cudaSuccess) return BAKRON_ERR_CUDA;
+    BK_CUDA_OK(ensure_leaf_attrs());
     const Tuning tu = force ? *force : tuning_for(m, n);
     a.tc_min_band = tu.tc_min_band;         // 0 or less: tensor cores off
     a.fused_max_band = tu.fused_max_band;
@@ -1660,10 +1660,8 @@ int launch_init(const void* W, int wdt, int m, int n, int64_t ldw, float* X, int
   const int64_t chunks = mp * np / 8;
   LaunchScope ls(kFamInit, s);
   const unsigned blocks = (unsigned)std::min<int64_t>((chunks + 255) / 256, 152 * 8);
-  return launch_pdl(k_init, dim3(blocks), dim3(256), 0, s, W, wdt, m, n, ldw, X, mp, np,
-                    ls.stamp()) == cudaSuccess
-             ? BAKRON_OK
-             : BAKRON_ERR_CUDA;
+  return BK_CUDA_RC(launch_pdl(k_init, dim3(blocks), dim3(256), 0, s, W, wdt, m, n, ldw, X, mp,
+                               np, ls.stamp()));
 }
 
 int launch_solve_prologue(const void* W, int wdt, int m, int n, int64_t ldw, int gsz, int G,
@@ -1677,10 +1675,8 @@ int launch_solve_prologue(const void* W, int wdt, int m, int n, int64_t ldw, int
 int launch_copy_out(const float* X, int64_t np, int m, int n, float* out, cudaStream_t s) {
   const int64_t tot = (int64_t)m * n;
   LaunchScope ls(kFamCopy, s);
-  return launch_pdl(k_copy_out, dim3((unsigned)((tot + 255) / 256)), dim3(256), 0, s, X, np, m,
-                    n, out) == cudaSuccess
-             ? BAKRON_OK
-             : BAKRON_ERR_CUDA;
+  return BK_CUDA_RC(launch_pdl(k_copy_out, dim3((unsigned)((tot + 255) / 256)), dim3(256), 0, s,
+                               X, np, m, n, out));
 }
 
 }  // namespace bakron

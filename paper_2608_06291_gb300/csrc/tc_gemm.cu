@@ -64,6 +64,21 @@ constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*ba
 constexpr int NACC = 4;                         // TMEM accumulators, rotating per K stage
 constexpr uint32_t TMEM_COLS = NACC * BN;       // all 512 columns: one CTA per SM (shared memory)
 
+// Paired variant (V_PAIR): two CTAs of a cluster compute the 128 x 128 blocks
+// of two adjacent row blocks at the same column block with one M = 256
+// MMA (cta_group::2).  Each CTA holds its own 128 rows of A and one half (64
+// rows) of the shared B; the tensor cores of both SMs read both halves.  Per
+// SM and 32-deep K stage that is 48 KiB written into shared memory by TMA and
+// 72 KiB read by the MMAs, against 64 + 96 KiB for one CTA alone: shared
+// memory bandwidth (about 128 B per cycle), not the tensor pipe, bounds the
+// single-CTA kernel.  Four ring slots of 48 KiB.
+constexpr int PAIR_STAGES = 4;
+constexpr int BN_HALF = BN / 2;
+constexpr uint32_t PAIR_STAGE_BYTES = 2 * TILE_BYTES + 2 * (TILE_BYTES / 2);
+constexpr uint32_t PAIR_SMEM_BYTES = PAIR_STAGES * PAIR_STAGE_BYTES + 1024 + 256;
+static_assert(PAIR_STAGES <= NACC, "a slot is freed by the commit of its accumulator");
+static_assert(PAIR_STAGES * PAIR_STAGE_BYTES >= 8 * TILE_BYTES, "the epilogue stages 8 boxes in the ring");
+
 // MODE_COLS: the column-band update of the B = I (GPTQ) schedule,
 // X[:, S2] += E[:, S1] L^A[S2, S1]^T with S1 = tile columns [k, h) and S2 =
 // [h, l); it reads and writes like stage 2 (A = E in the M planes, B = L^A,
@@ -103,7 +118,16 @@ struct TcParams {
 //               MMAs are kind::f16 (bf16 x bf16 products exact in fp32), and
 //               GRAM_KGROUP slots are summed in place per accumulator, each
 //               slot freed by its own commit to `empty`
-enum Variant { V_BAND = 0, V_GRAM_TF32 = 1, V_GRAM_BF16 = 2 };
+//   V_PAIR      band products and the dense diagnostic on CTA pairs (above)
+enum Variant { V_BAND = 0, V_GRAM_TF32 = 1, V_GRAM_BF16 = 2, V_PAIR = 3 };
+
+template <int V>
+struct Ring {
+  static constexpr bool pair = V == V_PAIR;
+  static constexpr int stages = pair ? PAIR_STAGES : STAGES;
+  static constexpr uint32_t b_plane = pair ? TILE_BYTES / 2 : TILE_BYTES;   // one B plane
+  static constexpr uint32_t stage_bytes = 2 * TILE_BYTES + 2 * b_plane;
+};
 constexpr int GRAM_KGROUP = 4;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -252,6 +276,103 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
       : "memory");
 }
 
+// ---- CTA-pair forms (cluster of two along y; rank 0 issues the MMAs)
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+// Address, in the cluster's shared window, of the same variable in rank 0.
+__device__ __forceinline__ uint32_t at_rank0(const void* p) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, 0;" : "=r"(r) : "r"(smem_u32(p)));
+  return r;
+}
+
+__device__ __forceinline__ void cmbar_arrive_expect_tx(uint32_t cbar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.release.cluster.shared::cluster.b64 _, [%0], %1;" ::"r"(
+                   cbar),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cmbar_expect_tx_only(uint32_t cbar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cluster.shared::cluster.b64 [%0], %1;" ::"r"(cbar),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cmbar_arrive(uint32_t cbar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cbar)
+               : "memory");
+}
+
+// Bounded wait with cluster-scope acquire (arrivals from the other CTA).
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity, long long limit) {
+  const long long t0 = clock64();
+  while (true) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    if (ok) return true;
+    if (clock64() - t0 > limit) return false;
+  }
+}
+
+// TMA loads into this CTA's shared memory whose completion is counted on an
+// mbarrier of rank 0 (cta_group::2: the barrier may sit in the peer CTA).
+__device__ __forceinline__ void tma_load_pair_c2(void* dst, const CUtensorMap* map, uint32_t cbar,
+                                                 int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(cbar), "r"(x), "r"(y), "r"(0)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_2d_c2(void* dst, const CUtensorMap* map, uint32_t cbar,
+                                               int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(cbar), "r"(x), "r"(y)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_tf32_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                              uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrives on the barrier at this offset in both CTAs of the pair once every
+// MMA issued so far has completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"((unsigned short)3)
+      : "memory");
+}
+
+// Sets the int at this offset in the other CTA of the pair.
+__device__ __forceinline__ void st_peer_flag(const void* local, int rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(local)), "r"(rank ^ 1));
+  asm volatile("st.relaxed.cluster.shared::cluster.u32 [%0], %1;" ::"r"(r), "r"(1u) : "memory");
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+
 // 32 lanes x 32 consecutive fp32 columns of TMEM into v (one per column) of
 // each thread; the values are valid only after tmem_wait_ld().
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
@@ -274,7 +395,9 @@ __device__ __forceinline__ void tmem_wait_ld() {
 // Output block and K range of this CTA.
 struct Block {
   int rb, cb;         // output block (128-row block, 128-col block)
-  int k0, nk;         // first K tile (32 wide) and number of K tiles
+  int k0, nk;         // first K tile (32 wide) and number of K tiles the MMAs run
+  int ok0, onk;       // the K tiles this block's own rows need (pairs: a subrange)
+  bool own;           // the block is written (pairs: this CTA's row block has work)
 };
 
 // Column blocks [cb_lo, cb_hi] of 128-row block rb that have work in a band
@@ -315,6 +438,31 @@ __host__ __device__ inline bool band_row_span(int mode, int k, int h, int l, int
 // instead of every B block coming from DRAM once per row block).
 constexpr int RASTER_ROWS = 8;   // default group height (BAKRON_TC_RASTER overrides it)
 
+// K tiles of band block (rb, cb): stage 1 those I' with some (I', J') in S1,
+// J' in the column block, I' <= I; stage 2 from where stage 1's M coverage
+// of these rows starts (M tiles of real rows below k - I are exact zeros
+// there); column bands the tile columns of S1, the same for every block.
+__device__ __forceinline__ void band_k_range(const TcParams& P, int rb, int cb, int& k0, int& nk) {
+  if (P.mode == MODE_COLS) {
+    k0 = P.k;
+    nk = P.h - P.k;
+    return;
+  }
+  const int I0 = 4 * rb, Ilast = min(I0 + 3, P.Mt - 1);
+  const int J0 = 4 * cb;
+  if (P.mode == MODE_STAGE1) {
+    const int ilo = max(0, P.k - (J0 + 3));
+    const int ihi = min(I0 + 3, P.h - 1 - J0);
+    k0 = ilo;
+    nk = ihi >= ilo ? ihi - ilo + 1 : 0;
+    return;
+  }
+  const int jlo = max(0, P.k - Ilast);
+  const int jhi = min(J0 + 3, P.h - 1);
+  k0 = jlo;
+  nk = jhi >= jlo ? jhi - jlo + 1 : 0;
+}
+
 // Returns false if the block has no work at all (beyond its row's span).
 __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
   // the blocks with the longest K ranges first (they sit at high rows, and
@@ -329,10 +477,11 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
     bx = in / gh;
   }
   b.rb = P.row0 + (P.mode == MODE_DENSE ? by : (int)gridDim.y - 1 - by);
+  b.own = true;
   if (P.mode == MODE_DENSE) {
     b.cb = blockIdx.x;
-    b.k0 = 0;
-    b.nk = P.K / BK;
+    b.k0 = b.ok0 = 0;
+    b.nk = b.onk = P.K / BK;
     return true;
   }
   if (P.mode == MODE_GRAM) {
@@ -343,35 +492,66 @@ __device__ __forceinline__ bool block_of(const TcParams& P, Block& b) {
     while (rb * (rb + 1) / 2 > t) --rb;
     b.rb = rb;
     b.cb = t - rb * (rb + 1) / 2;
-    b.k0 = 0;
-    b.nk = P.K / BK;   // K stages; the bf16 variant's K counts 128-byte rows of 64
+    b.k0 = b.ok0 = 0;
+    b.nk = b.onk = P.K / BK;   // K stages; the bf16 variant's K counts 128-byte rows of 64
     return true;
   }
   int cb_lo, cb_hi;
   if (!band_row_span(P.mode, P.k, P.h, P.l, P.Mt, P.Nt, b.rb, cb_lo, cb_hi)) return false;
   b.cb = P.mode == MODE_STAGE2 ? cb_hi - bx : cb_lo + bx;
   if (b.cb > cb_hi || b.cb < cb_lo) return false;
-  if (P.mode == MODE_COLS) {   // K = the tile columns of S1, the same for every block
-    b.k0 = P.k;
-    b.nk = P.h - P.k;
+  band_k_range(P, b.rb, b.cb, b.k0, b.nk);
+  b.ok0 = b.k0;
+  b.onk = b.nk;
+  b.own = true;
+  return true;
+}
+
+// Pairs: clusters of two CTAs along x; CTA `rank` of the cluster at grid
+// position (blockIdx.x / 2, blockIdx.y) takes row block base + rank; both
+// CTAs take the same column block and run the union of their K ranges (this
+// CTA's A is zero outside its own).  The decision that the pair has work is
+// the same in both CTAs.
+__device__ __forceinline__ bool block_of_pair(const TcParams& P, int rank, Block& b) {
+  int bx = (int)blockIdx.x >> 1, by = (int)blockIdx.y;
+  const int W = (int)gridDim.x >> 1, H = (int)gridDim.y;
+  if (P.mode == MODE_DENSE) {
+    b.rb = 2 * by + rank;
+    b.cb = bx;
+    b.k0 = b.ok0 = 0;
+    b.nk = b.onk = P.K / BK;
+    b.own = true;
     return true;
   }
-  const int I0 = 4 * b.rb, Ilast = min(I0 + 3, P.Mt - 1);
-  const int J0 = 4 * b.cb;
-  if (P.mode == MODE_STAGE1) {
-    // K tiles I' with some (I', J') in S1, J' in this column block, I' <= I
-    const int ilo = max(0, P.k - (J0 + 3));
-    const int ihi = min(I0 + 3, P.h - 1 - J0);
-    b.k0 = ilo;
-    b.nk = ihi >= ilo ? ihi - ilo + 1 : 0;
-    return true;
+  {
+    const int R = max(1, (P.raster > 0 ? P.raster : RASTER_ROWS) / 2);   // pairs per group
+    const int L = by * W + bx, grp = L / (R * W), in = L - grp * R * W;
+    const int gh = min(R, H - grp * R);
+    by = grp * R + in % gh;
+    bx = in / gh;
   }
-  // stage 2 (K starts where stage 1's M coverage of these rows starts; M tiles
-  // of real rows below k - I are exact zeros there)
-  const int jlo = max(0, P.k - Ilast);
-  const int jhi = min(J0 + 3, P.h - 1);
-  b.k0 = jlo;
-  b.nk = jhi >= jlo ? jhi - jlo + 1 : 0;
+  const int base = P.row0 + 2 * (H - 1 - by);
+  int lo0 = 0, hi0 = -1, lo1 = 0, hi1 = -1;
+  const bool v0 = band_row_span(P.mode, P.k, P.h, P.l, P.Mt, P.Nt, base, lo0, hi0);
+  const bool v1 = band_row_span(P.mode, P.k, P.h, P.l, P.Mt, P.Nt, base + 1, lo1, hi1);
+  if (!v0 && !v1) return false;
+  const int cb_lo = v0 && v1 ? min(lo0, lo1) : (v0 ? lo0 : lo1);
+  const int cb_hi = v0 && v1 ? max(hi0, hi1) : (v0 ? hi0 : hi1);
+  b.cb = P.mode == MODE_STAGE2 ? cb_hi - bx : cb_lo + bx;
+  if (b.cb > cb_hi || b.cb < cb_lo) return false;
+  const bool s0 = v0 && lo0 <= b.cb && b.cb <= hi0, s1 = v1 && lo1 <= b.cb && b.cb <= hi1;
+  int k00 = 0, nk0 = 0, k01 = 0, nk1 = 0;
+  if (s0) band_k_range(P, base, b.cb, k00, nk0);
+  if (s1) band_k_range(P, base + 1, b.cb, k01, nk1);
+  const bool w0 = s0 && nk0 > 0, w1 = s1 && nk1 > 0;   // rows with K tiles
+  const int u0 = w0 && w1 ? min(k00, k01) : (w0 ? k00 : k01);
+  const int u1 = w0 && w1 ? max(k00 + nk0, k01 + nk1) : (w0 ? k00 + nk0 : k01 + nk1);
+  b.rb = base + rank;
+  b.own = rank ? s1 : s0;
+  b.ok0 = rank ? k01 : k00;
+  b.onk = rank ? nk1 : nk0;
+  b.k0 = w0 || w1 ? u0 : 0;
+  b.nk = w0 || w1 ? u1 - u0 : 0;
   return true;
 }
 
@@ -381,23 +561,32 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
           const __grid_constant__ CUtensorMap mapBh, const __grid_constant__ CUtensorMap mapBl,
           const __grid_constant__ CUtensorMap mapOh, const __grid_constant__ CUtensorMap mapOl,
           const TcParams P) {
+  using RG = Ring<V>;
+  constexpr bool pair = RG::pair;
+  constexpr int NST = RG::stages;
+  constexpr uint32_t SB = RG::stage_bytes;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // 1024-byte alignment for the 128-byte swizzle atoms
   unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint64_t* bars = (uint64_t*)(smem + STAGES * STAGE_BYTES);
-  uint64_t* full = bars;                 // [STAGES] smem stage loaded
-  uint64_t* empty = bars + STAGES;       // [STAGES] slot read by its MMAs (kgroup > 1 only;
+  uint64_t* bars = (uint64_t*)(smem + NST * SB);
+  uint64_t* full = bars;                 // [NST] smem stage loaded
+  uint64_t* empty = bars + NST;          // [NST] slot read by its MMAs (kgroup > 1 only;
                                          // otherwise the slot's accF commit frees it)
-  uint64_t* accum = bars + 2 * STAGES;   // [1] every MMA of the CTA complete
+  uint64_t* accum = bars + 2 * NST;      // [1] every MMA of the CTA complete
   uint64_t* accF = accum + 1;            // [NACC] accumulator holds a finished K stage
   uint64_t* accE = accum + 1 + NACC;     // [NACC] accumulator read out by the epilogue
   uint32_t* tmem_slot = (uint32_t*)(accum + 1 + 2 * NACC);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // pairs: rank 0 (the leader) issues the MMAs; the loads of both CTAs count
+  // on the leader's `full` barriers, the epilogues of both on its `accE`
+  const int rank = pair ? (int)cluster_rank() : 0;
   Block blk;
-  const bool has_block = block_of(P, blk);
-  if (!has_block) {          // uniform over the CTA: nothing allocated yet
+  bool has_block;
+  if constexpr (pair) has_block = block_of_pair(P, rank, blk);
+  else has_block = block_of(P, blk);
+  if (!has_block) {          // uniform over the CTA (and the pair): nothing allocated yet
     pdl_wait();
     pdl_trigger();
     return;
@@ -412,42 +601,79 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapOl)) : "memory");
   }
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&full[s], 1);
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&full[s], pair && rank == 0 ? 2 : 1);   // leader: its producer and the peer's
       mbar_init(&empty[s], 1);
     }
     mbar_init(accum, 1);
     for (int a = 0; a < NACC; ++a) {
       mbar_init(&accF[a], 1);
-      mbar_init(&accE[a], EPI_WARPS);  // lane 0 of each epilogue warp
+      // lane 0 of each epilogue warp (of both CTAs at the leader)
+      mbar_init(&accE[a], pair && rank == 0 ? 2 * EPI_WARPS : EPI_WARPS);
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     smem_u32(tmem_slot)),
-                 "r"(TMEM_COLS)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    if constexpr (pair) {   // one warp of each CTA of the pair, same columns in both
+      asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                       smem_u32(tmem_slot)),
+                   "r"(TMEM_COLS)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    } else {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                       smem_u32(tmem_slot)),
+                   "r"(TMEM_COLS)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-  __syncthreads();
+  if constexpr (pair) cluster_sync_all();   // both CTAs' barriers initialised
+  else __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = *tmem_slot;
+  // the leader's barriers in the cluster's shared window (pairs)
+  uint32_t cfull0 = 0, caccE0 = 0;
+  if constexpr (pair) {
+    cfull0 = at_rank0(full);
+    caccE0 = at_rank0(accE);
+  }
   // The factor operand (stage 1: A = L^B; stage 2: B = L^A) is read-only
   // during the solve: its part of the first ring slots is loaded before the
   // wait for the previous kernel, whose output (E^T or M) is the other one.
-  const int npre = blk.nk < STAGES ? blk.nk : STAGES;
+  // a wait that ran out stops both CTAs of a pair
+  auto abort_all = [&]() {
+    *abort_flag = 1;
+    if constexpr (pair) st_peer_flag((const void*)abort_flag, rank);
+  };
+  const int npre = blk.nk < NST ? blk.nk : NST;
   const bool a_static = P.mode != MODE_STAGE2 && P.mode != MODE_COLS;
   constexpr bool bf16_ops = V == V_GRAM_BF16;
+  // pairs: this CTA's A is zero (a fully out-of-range box) outside its own K
+  // range; its half of B is rows 64 * rank .. of the column block
+  auto a_row = [&](int kt) -> int {
+    if (!pair) return blk.rb * BM;
+    return (blk.own && kt >= blk.ok0 && kt < blk.ok0 + blk.onk) ? blk.rb * BM : -BM;
+  };
+  const int b_row = pair ? blk.cb * BN + BN_HALF * rank : blk.cb * BN;
   if (warp == 0 && lane == 0) {
     for (int i = 0; i < npre; ++i) {
-      unsigned char* st = smem + i * STAGE_BYTES;
+      unsigned char* st = smem + i * SB;
       const int kt = blk.k0 + i;
       if constexpr (bf16_ops) {
         mbar_expect_tx_only(&full[i], TILE_BYTES);
         tma_load_2d(st, &mapA2, &full[i], kt * 2 * BK, blk.rb * BM);
+        continue;
+      }
+      if constexpr (pair) {
+        const uint32_t cb = cfull0 + (uint32_t)(i * 8);
+        cmbar_expect_tx_only(cb, a_static ? 2 * TILE_BYTES : 2 * RG::b_plane);
+        if (a_static)
+          tma_load_pair_c2(st, &mapA2, cb, kt * BK, a_row(kt));
+        else
+          tma_load_pair_c2(st + 2 * TILE_BYTES, &mapB2, cb, kt * BK, b_row);
         continue;
       }
       mbar_expect_tx_only(&full[i], 2 * TILE_BYTES);
@@ -469,31 +695,37 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   if (warp == 0) {
     // ---------------------------------------------------------- producer
     int issued = 0;
+    bool aborted = false;
     for (int i = 0; i < nk; ++i) {
-      const int s = i % STAGES;
+      const int s = i % NST;
       bool ok = true;
-      // slot s was last read by the MMAs of stage j = i - STAGES, which are
+      // slot s was last read by the MMAs of stage j = i - NST, which are
       // complete when their accumulator's commit arrives (accF); that barrier
       // cannot have moved on to stage j + NACC yet, which needs this load
-      if (lane == 0 && i >= STAGES) {
-        const int j = i - STAGES;
+      if (lane == 0 && i >= NST) {
+        const int j = i - NST;
         if constexpr (kgroup > 1)
-          ok = mbar_wait(&empty[s], (uint32_t)(j / STAGES) & 1u, P.spin_cycles);
+          ok = mbar_wait(&empty[s], (uint32_t)(j / NST) & 1u, P.spin_cycles);
         else
           ok = mbar_wait(&accF[j % NACC], (uint32_t)(j / NACC) & 1u, P.spin_cycles);
       }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok || *abort_flag) {
-        if (lane == 0 && !ok) { raise_status(P.status, BAKRON_ERR_TIMEOUT); *abort_flag = 1; }
+        if (lane == 0 && !ok) { raise_status(P.status, BAKRON_ERR_TIMEOUT); abort_all(); }
         // slots loaded in part before the wait: arrive, so that their phase
         // completes once those copies land (the drain below waits for them)
-        if (lane == 0)
-          for (int j = i; j < npre; ++j) mbar_arrive(&full[j]);
+        if (lane == 0) {
+          for (int j = i; j < npre; ++j) {
+            if constexpr (pair) cmbar_arrive(cfull0 + (uint32_t)(j * 8));
+            else mbar_arrive(&full[j]);
+          }
+        }
+        aborted = true;
         break;
       }
-      unsigned char* st = smem + s * STAGE_BYTES;
+      unsigned char* st = smem + s * SB;
       // planes of the slot: A hi, A lo, B hi, B lo (a pair lands as hi then lo)
-      unsigned char *a_hi = st, *b_hi = st + 2 * TILE_BYTES, *b_lo = st + 3 * TILE_BYTES;
+      unsigned char *a_hi = st, *b_hi = st + 2 * TILE_BYTES, *b_lo = b_hi + RG::b_plane;
       const int kt = blk.k0 + i;            // K tile index (32 wide)
       const bool pre = i < npre;            // the factor operand is already on its way
       if constexpr (bf16_ops) {             // one bf16 box per operand, 64 of K
@@ -507,6 +739,38 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
         continue;
       }
       const bool load_a = !(pre && a_static), load_b = !(pre && !a_static);
+      if constexpr (pair) {
+        // every box lands in full (an out-of-range one as zeros), so the
+        // byte count does not depend on the band
+        if (lane == 0) {
+          const uint32_t cb = cfull0 + (uint32_t)(s * 8);
+          cmbar_arrive_expect_tx(cb, (load_a ? 2 * TILE_BYTES : 0u) +
+                                         (load_b ? 2 * RG::b_plane : 0u));
+          if (load_a) tma_load_pair_c2(a_hi, &mapA2, cb, kt * BK, a_row(kt));
+          if (load_b) {
+            unsigned valid = 3u;            // stage 1: this half's two sub-tiles in the band
+            if (P.mode == MODE_STAGE1) {
+              valid = 0;
+              for (int sub = 0; sub < 2; ++sub) {
+                const int Jp = 4 * blk.cb + 2 * rank + sub;
+                if (Jp < P.Nt && kt < P.Mt && kt + Jp >= P.k && kt + Jp < P.h) valid |= 1u << sub;
+              }
+            }
+            if (valid == 3u) {
+              tma_load_pair_c2(b_hi, &mapB2, cb, kt * BK, b_row);   // b_lo follows
+            } else {
+              for (int sub = 0; sub < 2; ++sub) {
+                const int y = (valid & (1u << sub)) ? b_row + 32 * sub : -32;
+                tma_load_2d_c2(b_hi + sub * 4096, &mapBh, cb, kt * BK, y);
+                tma_load_2d_c2(b_lo + sub * 4096, &mapBl, cb, kt * BK, y);
+              }
+            }
+          }
+        }
+        __syncwarp();
+        issued = i + 1;
+        continue;
+      }
       uint32_t bytes = load_a ? 2 * TILE_BYTES : 0u;   // A hi + A lo
       unsigned valid = 0xF;                 // stage 1: B sub-tiles in the band
       if (P.mode == MODE_STAGE1) {
@@ -554,11 +818,22 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
     }
     // drain: every copy this warp issued has landed before the CTA winds down
     if (lane == 0) {
-      const int last = issued > npre ? issued : npre;
-      const int first = last > STAGES ? last - STAGES : 0;
-      for (int i = first; i < last; ++i) {
-        if (!mbar_wait(&full[i % STAGES], (uint32_t)(i / STAGES) & 1u, drain))
-          raise_status(P.status, BAKRON_ERR_TIMEOUT);
+      // pairs: after an abort a leader's phase may lack the peer's arrival,
+      // and the peer cannot watch the leader's barriers; copies in flight land
+      // within microseconds, so both wait about a millisecond instead
+      constexpr long long kPairSettle = 2000000LL;
+      if (pair && (rank != 0 || *abort_flag)) {
+        if (aborted || *abort_flag) {
+          const long long t0 = clock64();
+          while (clock64() - t0 < kPairSettle) __nanosleep(1000);
+        }
+      } else {
+        const int last = issued > npre ? issued : npre;
+        const int first = last > NST ? last - NST : 0;
+        for (int i = first; i < last; ++i) {
+          if (!mbar_wait(&full[i % NST], (uint32_t)(i / NST) & 1u, drain))
+            raise_status(P.status, BAKRON_ERR_TIMEOUT);
+        }
       }
     }
   } else if (warp == 1) {
@@ -568,36 +843,55 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
     // (group mod NACC); the epilogue adds the groups in fp32 registers.  The
     // tensor core's accumulation is not round-to-nearest, and its error grows
     // with the number of MMAs summed in place; restarting every group bounds it.
-    if (lane == 0) {
-      const uint32_t idesc = idesc_tf32(BM, BN), idesc_b = idesc_bf16(BM, BN);
+    if (lane == 0 && pair && rank != 0) {
+      // the peer: the leader's MMAs write this CTA's TMEM and read its shared
+      // memory; its last commit arrives here too once they have completed
+      if (nk == 0) mbar_arrive(accum);
+      if (!mbar_wait(accum, 0, drain)) raise_status(P.status, BAKRON_ERR_TIMEOUT);
+    } else if (lane == 0) {
+      const uint32_t idesc = idesc_tf32(pair ? 2 * BM : BM, BN), idesc_b = idesc_bf16(BM, BN);
       const uint64_t desc0 = smem_desc(smem_u32(smem));   // stage 0, A hi, K step 0
       for (int i = 0; i < nk; ++i) {
-        const int s = i % STAGES;
-        const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
+        const int s = i % NST;
+        const uint32_t ph = (uint32_t)(i / NST) & 1u;
         const int g = i / kgroup, a = g % NACC;     // accumulator group of this slot
         const bool first = i % kgroup == 0;
         const bool last = i % kgroup == kgroup - 1 || i == nk - 1;
         // accumulator a was last used by group g - NACC: wait until it was read
         // out (the producer's and the epilogue's aborts surface here as time-outs)
-        const bool ok = mbar_wait(&full[s], ph, P.spin_cycles) &&
-                        (!first || g < NACC ||
-                         mbar_wait(&accE[a], (uint32_t)(g / NACC - 1) & 1u, P.spin_cycles));
+        bool ok;
+        if constexpr (pair)
+          ok = mbar_wait_cluster(&full[s], ph, P.spin_cycles) &&
+               (!first || g < NACC ||
+                mbar_wait_cluster(&accE[a], (uint32_t)(g / NACC - 1) & 1u, P.spin_cycles));
+        else
+          ok = mbar_wait(&full[s], ph, P.spin_cycles) &&
+               (!first || g < NACC ||
+                mbar_wait(&accE[a], (uint32_t)(g / NACC - 1) & 1u, P.spin_cycles));
         if (!ok) {
           raise_status(P.status, BAKRON_ERR_TIMEOUT);
-          *abort_flag = 1;
+          abort_all();
           break;
         }
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         // descriptors of this stage's four planes; K steps of 32 bytes add 2 to
         // the start-address field (16-byte units, no carry within a stage)
-        const uint64_t dah = desc0 + (uint64_t)((s * STAGE_BYTES) >> 4);
+        const uint64_t dah = desc0 + (uint64_t)((s * SB) >> 4);
         const uint64_t dal = dah + (TILE_BYTES >> 4), dbh = dah + (2 * TILE_BYTES >> 4),
-                       dbl = dah + (3 * TILE_BYTES >> 4);
+                       dbl = dbh + (RG::b_plane >> 4);
         const uint32_t d = tmem + (uint32_t)(a * BN);
         if constexpr (bf16_ops) {
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)            // 16 bf16 = 32 bytes along K per MMA
             mma_bf16(d, dah + 2 * kk, dbh + 2 * kk, idesc_b, (kk > 0 || !first) ? 1u : 0u);
+        } else if constexpr (pair) {
+#pragma unroll
+          for (int kk = 0; kk < BK / 8; ++kk) {
+            const uint64_t o = (uint64_t)(2 * kk);
+            mma_tf32_pair(d, dah + o, dbh + o, idesc, (kk > 0 || !first) ? 1u : 0u);
+            mma_tf32_pair(d, dah + o, dbl + o, idesc, 1u);
+            mma_tf32_pair(d, dal + o, dbh + o, idesc, 1u);
+          }
         } else {
 #pragma unroll
           for (int kk = 0; kk < BK / 8; ++kk) {
@@ -607,11 +901,19 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
             if (V == V_BAND || !P.a_exact) mma_tf32(d, dal + o, dbh + o, idesc, 1u);
           }
         }
-        if constexpr (kgroup > 1) mma_commit(&empty[s]);   // the slot back to the producer
-        if (last) mma_commit(&accF[a]);  // the group's sum to the epilogue (kgroup 1: and the slot)
+        if constexpr (pair) {
+          if (last) mma_commit_pair(&accF[a]);   // both CTAs: the sum, and the slot
+        } else {
+          if constexpr (kgroup > 1) mma_commit(&empty[s]);   // the slot back to the producer
+          if (last) mma_commit(&accF[a]);  // the group's sum to the epilogue (kgroup 1: and the slot)
+        }
       }
-      if (nk > 0) mma_commit(accum);  // tracks every MMA issued above
-      else mbar_arrive(accum);
+      if (nk > 0) {  // tracks every MMA issued above
+        if constexpr (pair) mma_commit_pair(accum);
+        else mma_commit(accum);
+      } else {
+        mbar_arrive(accum);
+      }
       // wind-down guard: all issued MMAs complete before anyone frees TMEM
       if (!mbar_wait(accum, 0, drain)) raise_status(P.status, BAKRON_ERR_TIMEOUT);
     }
@@ -624,14 +926,14 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
     float acc[EPI_COLS];
 #pragma unroll
     for (int u = 0; u < EPI_COLS; ++u) acc[u] = 0.f;
-    bool write = true;
+    bool write = blk.own;
     for (int i = 0; i < ngroups; ++i) {
       const int a = i % NACC;
       // one lane waits; the decision is warp-uniform (tcgen05.ld is warp-collective)
       int ok = 1;
       if (lane == 0) {
         ok = mbar_wait(&accF[a], (uint32_t)(i / NACC) & 1u, P.spin_cycles) ? 1 : 0;
-        if (!ok) { raise_status(P.status, BAKRON_ERR_TIMEOUT); *abort_flag = 1; }
+        if (!ok) { raise_status(P.status, BAKRON_ERR_TIMEOUT); abort_all(); }
         if (*abort_flag) ok = 0;
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -649,7 +951,10 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
       }
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       __syncwarp();
-      if (lane == 0) mbar_arrive(&accE[a]);
+      if (lane == 0) {
+        if constexpr (pair) cmbar_arrive(caccE0 + (uint32_t)(a * 8));
+        else mbar_arrive(&accE[a]);
+      }
     }
     if (P.mode == MODE_GRAM) {
       // entry (gi, gj <= gi) and its mirror (gj, gi); for a fixed u the warp's
@@ -714,7 +1019,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // visible to the TMA unit
       }
       asm volatile("bar.sync 2, %0;" ::"n"(EPI_WARPS * 32) : "memory");   // the epilogue warps
-      if (warp == 2 && lane == 0 && !*abort_flag) {
+      if (warp == 2 && lane == 0 && !*abort_flag && blk.own) {
         const int x0 = blk.cb * BN, y0 = blk.rb * BM;
         if (P.mode == MODE_STAGE1) {
 #pragma unroll
@@ -722,7 +1027,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
             tma_store_2d(&mapOh, smem + c * TILE_BYTES, x0 + 32 * c, y0);
             tma_store_2d(&mapOl, smem + (4 + c) * TILE_BYTES, x0 + 32 * c, y0);
           }
-        } else if (nk > 0) {
+        } else if (blk.onk > 0) {
           // X += the block's tiles that lie in S2 (32 x 32 boxes: rows 32 ti
           // .. of box c start 4 KiB apart, whole swizzle periods)
           for (int ti = 0; ti < 4; ++ti) {
@@ -740,12 +1045,21 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
     }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-  __syncthreads();
+  // pairs: neither CTA leaves (nor frees TMEM) while the other may still
+  // signal its barriers or use its shared memory
+  if constexpr (pair) cluster_sync_all();
+  else __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   stamp_end(P.stamp);
   if (warp == 1) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
-                 "r"(TMEM_COLS)
-                 : "memory");
+    if constexpr (pair)
+      asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                   "r"(TMEM_COLS)
+                   : "memory");
+    else
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                   "r"(TMEM_COLS)
+                   : "memory");
   }
 }
 
@@ -828,8 +1142,33 @@ cudaError_t ensure_attr() {
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(k_tc_band<V_GRAM_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              SMEM_BYTES);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_tc_band<V_PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             PAIR_SMEM_BYTES);
   if (e == cudaSuccess) g_attr_done = true;
   return e;
+}
+
+// The paired kernel: clusters of two CTAs along x, with programmatic
+// dependent launch like every other kernel of the solve (pdl = false: a
+// plain launch, for the diagnostic GEMM).
+template <typename... Args>
+cudaError_t launch_pair(dim3 grid, cudaStream_t s, bool pdl, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = PAIR_SMEM_BYTES;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, k_tc_band<V_PAIR>, args...);
 }
 
 // hi/lo split of a dense matrix (diagnostic GEMM only)
@@ -967,6 +1306,8 @@ bool tc_band_maps(TcMaps& maps, const TcOperands& op) {
   ok &= make_map(&maps.Ml, op.ML, op.mp, op.np, op.np, BM);
   ok &= make_map_pair(&maps.M2, op.MH, op.ML, op.mp, op.np, op.np, BM);
   ok &= make_map_pair(&maps.LA2, op.LAH, op.LAL, op.np, op.np, op.np, BN);
+  ok &= make_map_pair(&maps.Et2h, op.EtH, op.EtL, op.np, op.mp, op.mp, BN_HALF);   // pairs' B halves
+  ok &= make_map_pair(&maps.LA2h, op.LAH, op.LAL, op.np, op.np, op.np, BN_HALF);
   ok &= make_map(&maps.X32, op.X, op.mp, op.np, op.np, 32);   // stage-2 reduce target
   return ok;
 }
@@ -978,9 +1319,34 @@ static int raster_rows() {
   return v >= 1 ? v : RASTER_ROWS;
 }
 
+// Band stages on CTA pairs (BAKRON_TC_PAIR=1/0, read per call; default kTcPairDefault).
+constexpr bool kTcPairDefault = false;
+bool tc_pair_on() {
+  const char* e = getenv("BAKRON_TC_PAIR");
+  if (e && *e) return atoi(e) != 0;
+  return kTcPairDefault;
+}
+
+// Pairs: the widest union of column spans over the row-block pairs
+// (rlo + 2p, rlo + 2p + 1) of rows [rlo, rhi].
+static int pair_width(int mode, int k, int h, int l, int Mt, int Nt, int rlo, int rhi) {
+  int width = 0;
+  for (int r0 = rlo; r0 <= rhi; r0 += 2) {
+    int lo = 1 << 30, hi = -1;
+    for (int r = r0; r <= r0 + 1; ++r) {
+      int cl, ch;
+      if (!band_row_span(mode, k, h, l, Mt, Nt, r, cl, ch)) continue;
+      lo = std::min(lo, cl);
+      hi = std::max(hi, ch);
+    }
+    if (hi >= 0) width = std::max(width, hi - lo + 1);
+  }
+  return width;
+}
+
 int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, int h, int l,
                   cudaStream_t s, unsigned long long* stamp) {
-  if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
+  BK_CUDA_OK(ensure_attr());
   TcParams P{};
   P.stamp = stamp;
   P.raster = raster_rows();
@@ -1004,8 +1370,17 @@ int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, in
   }
   if (rlo < 0) return BAKRON_OK;   // nothing to do in this stage
   P.row0 = rlo;
-  dim3 grid(width, rhi - rlo + 1);
   cudaError_t e;
+  if (tc_pair_on()) {
+    const int pairs = (rhi - rlo) / 2 + 1;
+    dim3 pg(2 * pair_width(P.mode, k, h, l, op.Mt, op.Nt, rlo, rhi), pairs);
+    if (stage == 1)
+      e = launch_pair(pg, s, true, maps.LB2, maps.Et2h, maps.Eth, maps.Etl, maps.Mh, maps.Ml, P);
+    else
+      e = launch_pair(pg, s, true, maps.M2, maps.LA2h, maps.Eth, maps.Etl, maps.X32, maps.X32, P);
+    return BK_CUDA_RC(e);
+  }
+  dim3 grid(width, rhi - rlo + 1);
   if (stage == 1)
     e = launch_pdl(k_tc_band<V_BAND>, grid, dim3(THREADS), SMEM_BYTES, s, maps.LB2, maps.Et2,
                    maps.Eth,
@@ -1014,12 +1389,12 @@ int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, in
     e = launch_pdl(k_tc_band<V_BAND>, grid, dim3(THREADS), SMEM_BYTES, s, maps.M2, maps.LA2,
                    maps.Eth,
                    maps.Etl, maps.X32, maps.X32, P);
-  return e == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
+  return BK_CUDA_RC(e);
 }
 
 int tc_cols_stage(const TcMaps& maps, const TcOperands& op, int k, int h, int l, cudaStream_t s,
                   unsigned long long* stamp) {
-  if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
+  BK_CUDA_OK(ensure_attr());
   if (k >= h || h >= l) return BAKRON_OK;
   TcParams P{};
   P.stamp = stamp;
@@ -1034,10 +1409,15 @@ int tc_cols_stage(const TcMaps& maps, const TcOperands& op, int k, int h, int l,
   const int rows = (op.Mt + 3) / 4;              // 128-row blocks holding real tiles
   const int cols = (l - 1) / 4 - h / 4 + 1;      // 128-column blocks covering S2
   P.row0 = 0;
+  if (tc_pair_on()) {
+    const cudaError_t e = launch_pair(dim3(2 * cols, (rows + 1) / 2), s, true, maps.M2,
+                                      maps.LA2h, maps.Eth, maps.Etl, maps.X32, maps.X32, P);
+    return BK_CUDA_RC(e);
+  }
   const cudaError_t e =
       launch_pdl(k_tc_band<V_BAND>, dim3(cols, rows), dim3(THREADS), SMEM_BYTES, s, maps.M2,
                  maps.LA2, maps.Eth, maps.Etl, maps.X32, maps.X32, P);
-  return e == cudaSuccess ? BAKRON_OK : BAKRON_ERR_CUDA;
+  return BK_CUDA_RC(e);
 }
 
 }  // namespace bakron
@@ -1051,7 +1431,7 @@ extern "C" int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C,
   if (M % BM || N % BN || K % BK) return BAKRON_ERR_INVALID_ARG;
   const size_t need = 256 + size_t(2) * (size_t(M) + N) * K * 4;
   if (workspace_bytes < need) return BAKRON_ERR_WORKSPACE;
-  if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
+  BK_CUDA_OK(ensure_attr());
   cudaStream_t s = (cudaStream_t)stream;
   char* ws = (char*)workspace;
   int* status = (int*)ws;
@@ -1075,7 +1455,14 @@ extern "C" int bakron_diag_gemm_tf32x3(const float* A, const float* B, float* C,
   P.status = status;
   P.spin_cycles = spin_cycles_from_env();
   dim3 grid(N / BN, M / BM);
-  k_tc_band<V_BAND><<<grid, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mBh, mBl, mBh, mBl, P);
+  if (tc_pair_on() && M % (2 * BM) == 0) {
+    CUtensorMap mB2h;
+    if (!make_map_pair(&mB2h, Bh, Bl, N, K, K, BN_HALF)) return BAKRON_ERR_CUDA;
+    BK_CUDA_OK(launch_pair(dim3(2 * (N / BN), M / (2 * BM)), s, false, mA2, mB2h, mBh, mBl, mBh,
+                           mBl, P));
+  } else {
+    k_tc_band<V_BAND><<<grid, THREADS, SMEM_BYTES, s>>>(mA2, mB2, mBh, mBl, mBh, mBl, P);
+  }
   BK_CUDA_OK(cudaGetLastError());
   return bakron_read_status(workspace, stream);
 }
@@ -1108,7 +1495,7 @@ extern "C" int bakron_gram(const void* X, int xdtype, int k, int d, int64_t ldx,
   kc = std::min<int64_t>(kc, round_up(k, kq));
   kc = std::min<int64_t>(kc, (int64_t)1 << 30);
   if (kc < kq) return BAKRON_ERR_WORKSPACE;
-  if (ensure_attr() != cudaSuccess) return BAKRON_ERR_CUDA;
+  BK_CUDA_OK(ensure_attr());
   cudaStream_t s = (cudaStream_t)stream;
   char* ws = (char*)workspace;
   int* status = (int*)ws;

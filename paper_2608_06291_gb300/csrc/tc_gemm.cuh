@@ -18,6 +18,7 @@ struct TcOperands {
 // TMA descriptors of every operand plane (built on the host per solve call).
 struct TcMaps {
   CUtensorMap LB2, Et2, M2, LA2;   // hi/lo pairs in one box (32 columns x 128 rows x 2 planes)
+  CUtensorMap Et2h, LA2h;          // the same in 64-row boxes: one half of B for CTA pairs
   CUtensorMap Eth, Etl;            // E^T planes in 32-row boxes (stage-1 sub-tiles at the band's edge)
   CUtensorMap Mh, Ml;              // M planes in 128-row boxes: stage-1 TMA store targets
   CUtensorMap X32;                 // X in 32 x 32 boxes: stage-2 TMA reduce-add target

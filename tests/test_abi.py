@@ -129,6 +129,18 @@ def test_invalid_arguments_rejected_on_host(L):
     assert P.strerror(2) == "damped Gram is not positive definite"
 
 
+@pytest.mark.skipif(torch.cuda.is_available(), reason="needs a machine without a CUDA device")
+def test_cuda_failure_is_recorded_with_its_name_and_place(L):
+    """A CUDA runtime failure surfaces as BAKRON_ERR_CUDA, and the error
+    behind it (here: no device) can be read back with where it happened."""
+    fake = ctypes.c_void_p(4096)
+    assert L.bakron_read_status(fake, None) == 3
+    code, name, where, line = P.bakron_last_cuda_error()
+    assert code != 0 and name.startswith("cuda") and where == "capi.cu" and line > 0
+    with pytest.raises(P.BakronError, match=r"\[cuda\w+ at capi\.cu:\d+\]"):
+        P.bakron.__dict__["_check"](3, "probe")
+
+
 def test_binding_rejects_bad_tensors_before_the_library():
     """The ctypes binding checks device, dtype and shapes itself and raises
     ValueError before calling into the library (no GPU needed)."""
