@@ -71,7 +71,10 @@ constexpr uint32_t TMEM_COLS = NACC * BN;       // all 512 columns: one CTA per 
 // SM and 32-deep K stage that is 48 KiB written into shared memory by TMA and
 // 72 KiB read by the MMAs, against 64 + 96 KiB for one CTA alone: shared
 // memory bandwidth (about 128 B per cycle), not the tensor pipe, bounds the
-// single-CTA kernel.  Four ring slots of 48 KiB.
+// single-CTA kernel.  Four ring slots of 48 KiB.  Measured on GB300 it is
+// slower than one CTA per block (4096^2 band stages 3.07 against 2.12 ms per
+// solve, 28672 x 8192: 101 against 67 ms; the same with CTA-scope waits), so
+// it is off by default (BAKRON_TC_PAIR=1 selects it).
 constexpr int PAIR_STAGES = 4;
 constexpr int BN_HALF = BN / 2;
 constexpr uint32_t PAIR_STAGE_BYTES = 2 * TILE_BYTES + 2 * (TILE_BYTES / 2);
