@@ -158,17 +158,20 @@ def _csrc_hash():
     return h.hexdigest()[:16]
 
 
-def _traffic(family):
-    """DRAM bytes per step of a kernel family from the committed ncu summary,
-    or None when the kernels changed since it was taken."""
+def _traffic(workload, family, launches):
+    """DRAM bytes (read + write) per launch of a kernel family, from the
+    committed ncu summary of this workload (`profiles/traffic.txt`: bytes per
+    solve by family), or None when there is none or the kernel sources
+    changed since it was taken."""
     p = os.path.join(ROOT, "profiles", "traffic.txt")
     try:
         t = json.load(open(p))
     except Exception:
         return None
-    if t.get("csrc_hash") != _csrc_hash():
+    if t.get("csrc_hash") != _csrc_hash() or not launches:
         return None
-    return t.get("dram_bytes_per_step", {}).get(family)
+    per_step = t.get("workloads", {}).get(workload, {}).get(family)
+    return None if per_step is None else per_step / launches
 
 
 class ClockSampler:
@@ -473,6 +476,7 @@ def run_gpu(args):
     timeline_ms = span_ms / max(1, nrep)
 
     peaks = _peaks() or {}
+    wl_key = f"config {args.config}"
     F_alg = f_alg(m, n)
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
     p_eff, p_src = fp32_effective_peak(peaks)
@@ -497,7 +501,7 @@ def run_gpu(args):
                    "bound": "tensor", "achieved": tc_ach, "peak": p_eff, "unit": "TFLOP/s",
                    "frac": tc_ach / p_eff, "peak_source": p_src,
                    "algorithmic_per_step": tc_work, "launches_per_step": tc_n,
-                   "ms_per_step": tc_ms, "traffic": _traffic("tc")}
+                   "ms_per_step": tc_ms, "traffic": _traffic(wl_key, "tc", tc_n)}
     # the leaves against their latency floor: the element anti-diagonals
     # (m + n - 1 dependent rounding steps, Sec. 3.3) at the chain's own
     # measured step time, one tile alone on the GPU
@@ -516,7 +520,7 @@ def run_gpu(args):
                  "floor_ms": floor_ms, "ms_per_step": leaf_ms, "launches_per_step": leaf_n,
                  "schedule_chain_steps": tile_steps,
                  "hbm_gbs": leaf_bytes / (leaf_ms / 1e3) / 1e9 if leaf_ms > 0 else None,
-                 "traffic": _traffic("leaf")}
+                 "traffic": _traffic(wl_key, "leaf", leaf_n)}
     dom = max(groups, key=lambda g: groups[g][0])
     if dom == "tc":
         roof = dict(tc_roof)
@@ -528,7 +532,7 @@ def run_gpu(args):
                 "frac": achieved / fp32_simt_peak,
                 "peak_source": "152 SMs x 128 FP32 lanes x 2 flop x sm_max_mhz (derived)",
                 "algorithmic_per_step": g_work, "launches_per_step": g_n,
-                "traffic": _traffic("simt")}
+                "traffic": _traffic(wl_key, "simt", g_n)}
     else:
         roof = dict(leaf_roof)
     roof["timing"] = ("family times partition the graph-replayed step (timeline stamps, "

@@ -52,3 +52,24 @@ def test_top_left_block_sample_is_exact():
         blk = O.bakron_recursive(W[:k, :k], f.LA[:k, :k], f.LB[:k, :k], g, base=64)
         np.testing.assert_array_equal(blk.codes, full.codes[:k, :k])
         np.testing.assert_allclose(blk.X, full.X[:k, :k], atol=1e-10)
+
+
+def test_traffic_is_per_launch_and_only_for_the_sources_it_was_taken_on(tmp_path, monkeypatch):
+    """roofline.traffic: DRAM bytes per solve of a family from the committed
+    summary, divided by the family's launches per solve; None for another
+    workload, a family without a figure, or changed kernel sources."""
+    import json
+    import os
+    (tmp_path / "profiles").mkdir()
+    (tmp_path / "profiles" / "traffic.txt").write_text(json.dumps(
+        {"csrc_hash": "abc", "workloads": {"config 2": {"leaf": 1000.0, "tc": 620.0}}}))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    monkeypatch.setattr(bench, "_csrc_hash", lambda: "abc")
+    assert bench._traffic("config 2", "leaf", 250) == 4.0
+    assert bench._traffic("config 2", "tc", 62) == 10.0
+    assert bench._traffic("config 3", "tc", 62) is None
+    assert bench._traffic("config 2", "simt", 10) is None
+    assert bench._traffic("config 2", "tc", 0) is None
+    monkeypatch.setattr(bench, "_csrc_hash", lambda: "changed")
+    assert bench._traffic("config 2", "leaf", 250) is None
+    assert os.path.exists(tmp_path / "profiles" / "traffic.txt")
