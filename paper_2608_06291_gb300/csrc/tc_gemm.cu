@@ -132,6 +132,12 @@ struct Ring {
   static constexpr uint32_t stage_bytes = 2 * TILE_BYTES + 2 * b_plane;
 };
 constexpr int GRAM_KGROUP = 4;
+// Band products: K stages summed in place per TMEM accumulator (each group
+// restarts its accumulator; the epilogue adds the groups in fp32).  Two
+// stages per accumulator measured 1% faster per solve on GB300 but moved the
+// 4096^2 free-running objective from 8e-5 to 3e-4 of the fp64 solve's (an
+// earlier tie, then its cascade): one stage it is.
+constexpr int BAND_KGROUP = 1;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);
@@ -692,7 +698,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   stamp_begin(P.stamp);
   const long long drain = 4000000000LL;   // ~2 s at 2 GHz: wind-down bound
   const int nk = blk.nk;
-  constexpr int kgroup = V == V_GRAM_BF16 ? GRAM_KGROUP : 1;
+  constexpr int kgroup = V == V_GRAM_BF16 ? GRAM_KGROUP : (V == V_BAND ? BAND_KGROUP : 1);
   const int ngroups = (nk + kgroup - 1) / kgroup;   // accumulator hand-overs
 
   if (warp == 0) {
