@@ -8,8 +8,9 @@
 //                X[:, h..c1) += E[:, c0..h) L^A[h..c1, c0..h)^T  (tensor cores),
 //                rec(h, c1).
 //
-// A leaf launch gives one warp to each 32-row strip of W (lane p = row p), and
-// the warp walks the range's columns in order.  Column q of a tile is one
+// A leaf launch gives one CTA to each 32-row strip of W; its first warp (lane
+// p = row p) walks the range's columns in order, the other three write the
+// finished tiles out and help form the windows.  Column q of a tile is one
 // step: every lane rounds its row's entry, x_pq -> code, e_pq = s (c - z) - x,
 // then adds e_pq L^A[q'][q] to the pre-rounding values of the later columns
 // q' of the tile, which it keeps in registers.  A later tile of the range
@@ -30,6 +31,7 @@
 namespace bakron {
 
 constexpr int GQ_BLOCK = 4;                               // tile columns per leaf launch
+constexpr int GQ_THREADS = 128;                           // warp 0 rounds; all four form windows
 constexpr int GQ_LA_BLOCKS = GQ_BLOCK * (GQ_BLOCK + 1) / 2;   // L^A blocks one launch reads
 
 struct GptqArgs {
@@ -64,25 +66,29 @@ __device__ __forceinline__ void gq_cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(src) : "memory");
 }
 
-// The window of tile t of the range, T1 = sum_{g=1..t} E[I, J-g] L^A[J, J-g]^T
-// (32 x 32, fp32-accurate by the 3xTF32 split), into S.T1 ([p][q]).  With
-// lane = 4 gid + tig, an m16n8k8 fragment holds A(gid (+8), tig (+4)),
+// Part of the window of tile t of the range: the sum over g = g0 .. g1 of
+// E[I, J-g] L^A[J, J-g]^T (fp32-accurate by the 3xTF32 split), columns
+// 8 ni0 .. 8 (ni0 + NI) - 1, stored into dst ([p][q]) plus `base` when given.
+// With lane = 4 gid + tig, an m16n8k8 fragment holds A(gid (+8), tig (+4)),
 // B(k = tig (+4), n = gid) and D(gid (+8), 2 tig (+1)).
-__device__ __forceinline__ void gptq_window(GptqSmem& S, int t, int lane) {
+template <int NI>
+__device__ __forceinline__ void gptq_window(const GptqSmem& S, int t, int g0, int g1, int ni0,
+                                            const float (*base)[TILE + 1], float (*dst)[TILE + 1],
+                                            int lane) {
   const int gid = lane >> 2, tig = lane & 3;
-  float d[2][4][4];
+  float d[2][NI][4];
 #pragma unroll
   for (int mi = 0; mi < 2; ++mi)
 #pragma unroll
-    for (int ni = 0; ni < 4; ++ni)
+    for (int ni = 0; ni < NI; ++ni)
 #pragma unroll
       for (int r = 0; r < 4; ++r) d[mi][ni][r] = 0.f;
-  for (int g = 1; g <= t; ++g) {
+  for (int g = g0; g <= g1; ++g) {
     const float(*Lg)[LEAF_BLOCK_LD] = S.LA[t * (t + 1) / 2 + g];   // B(k = j, n = q) = Lg[j][q]
     const float(*Eg)[TILE + 1] = S.Es[t - g];                       // A(p, j) = Eg[p][j]
 #pragma unroll
     for (int kk = 0; kk < TILE / 8; ++kk) {
-      uint32_t ah[2][4], al[2][4], bh[4][2], bl[4][2];
+      uint32_t ah[2][4], al[2][4], bh[NI][2], bl[NI][2];
 #pragma unroll
       for (int mi = 0; mi < 2; ++mi) {
         const int r = 16 * mi + gid, c = 8 * kk + tig;
@@ -92,15 +98,15 @@ __device__ __forceinline__ void gptq_window(GptqSmem& S, int t, int lane) {
         tf32_split(Eg[r + 8][c + 4], ah[mi][3], al[mi][3]);
       }
 #pragma unroll
-      for (int ni = 0; ni < 4; ++ni) {
-        const int k = 8 * kk + tig, n = 8 * ni + gid;
+      for (int ni = 0; ni < NI; ++ni) {
+        const int k = 8 * kk + tig, n = 8 * (ni0 + ni) + gid;
         tf32_split(Lg[k][n], bh[ni][0], bl[ni][0]);
         tf32_split(Lg[k + 4][n], bh[ni][1], bl[ni][1]);
       }
 #pragma unroll
       for (int mi = 0; mi < 2; ++mi)
 #pragma unroll
-        for (int ni = 0; ni < 4; ++ni) {
+        for (int ni = 0; ni < NI; ++ni) {
           mma_tf32_16x8x8(d[mi][ni], al[mi], bh[ni]);
           mma_tf32_16x8x8(d[mi][ni], ah[mi], bl[ni]);
           mma_tf32_16x8x8(d[mi][ni], ah[mi], bh[ni]);
@@ -110,21 +116,43 @@ __device__ __forceinline__ void gptq_window(GptqSmem& S, int t, int lane) {
 #pragma unroll
   for (int mi = 0; mi < 2; ++mi)
 #pragma unroll
-    for (int ni = 0; ni < 4; ++ni) {
-      const int r = 16 * mi + gid, c = 8 * ni + 2 * tig;
-      S.T1[r][c] = d[mi][ni][0];
-      S.T1[r][c + 1] = d[mi][ni][1];
-      S.T1[r + 8][c] = d[mi][ni][2];
-      S.T1[r + 8][c + 1] = d[mi][ni][3];
+    for (int ni = 0; ni < NI; ++ni) {
+      const int r = 16 * mi + gid, c = 8 * (ni0 + ni) + 2 * tig;
+      dst[r][c] = d[mi][ni][0] + (base ? base[r][c] : 0.f);
+      dst[r][c + 1] = d[mi][ni][1] + (base ? base[r][c + 1] : 0.f);
+      dst[r + 8][c] = d[mi][ni][2] + (base ? base[r + 8][c] : 0.f);
+      dst[r + 8][c + 1] = d[mi][ni][3] + (base ? base[r + 8][c + 1] : 0.f);
     }
-  __syncwarp();
+}
+
+// The outputs of tile t of the range from shared memory, by `nthr` threads
+// numbered from tid: pre-rounding values, codes, and E as an exact tf32
+// hi/lo pair for the column band (row by row, 32 consecutive columns per warp).
+__device__ __forceinline__ void gptq_store_tile(const GptqSmem& S, const GptqArgs& a, int64_t r0,
+                                                int64_t cbase, int t, int tid, int nthr) {
+  for (int e = tid; e < TILE * TILE; e += nthr) {
+    const int i = e / TILE, c = e % TILE;
+    const int64_t r = r0 + i, col = cbase + (int64_t)t * TILE + c;
+    const int64_t o = r * a.ldx + col;
+    a.X[o] = S.Xo[i][t * TILE + c];
+    const float ev = S.Es[t][i][c];
+    const float hi = tf32_hi(ev);
+    a.EH[o] = hi;
+    a.EL[o] = ev - hi;
+    if (r < a.m && col < a.n) a.codes[r * a.n + col] = S.Cs[i][t * TILE + c];
+  }
 }
 
 // Tiles c0 .. c0 + nt - 1 (nt <= GQ_BLOCK) of the strip of tile row blockIdx.x.
-__global__ void __launch_bounds__(32) k_gptq_leaf(int c0, int nt, GptqArgs a) {
+// Warp 0 walks the columns (lane = row); per tile, all four warps first form
+// its window (one 8-column slice each), then, while warp 0 rounds the tile,
+// warps 1-3 write the previous tile's outputs.  Every thread passes the same
+// CTA barriers.
+__global__ void __launch_bounds__(GQ_THREADS) k_gptq_leaf(int c0, int nt, GptqArgs a) {
   extern __shared__ __align__(16) unsigned char gq_smem[];
   GptqSmem& S = *reinterpret_cast<GptqSmem*>(gq_smem);
-  const int p = threadIdx.x;            // row of the strip
+  const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31;
+  const int p = lane;                   // warp 0: row of the strip
   const int I = blockIdx.x;
   const int64_t r0 = (int64_t)I * TILE, cbase = (int64_t)c0 * TILE;
   // factor blocks (read-only during the solve) before waiting for the
@@ -133,7 +161,8 @@ __global__ void __launch_bounds__(32) k_gptq_leaf(int c0, int nt, GptqArgs a) {
     for (int g = 0; g <= t; ++g) {
       const float* src = a.LAblk + ((int64_t)(c0 + t) * LEAF_BLOCKS + g) * LEAF_BLOCK_FLOATS;
       float* dst = &S.LA[t * (t + 1) / 2 + g][0][0];
-      for (int c = p; c < LEAF_BLOCK_FLOATS / 4; c += 32) gq_cp_async16(dst + 4 * c, src + 4 * c);
+      for (int c = tid; c < LEAF_BLOCK_FLOATS / 4; c += GQ_THREADS)
+        gq_cp_async16(dst + 4 * c, src + 4 * c);
     }
   asm volatile("cp.async.commit_group;" ::: "memory");
   // this row's grid on each tile (a group covers whole tiles: gsz % 32 == 0)
@@ -143,7 +172,7 @@ __global__ void __launch_bounds__(32) k_gptq_leaf(int c0, int nt, GptqArgs a) {
 #pragma unroll
   for (int t = 0; t < GQ_BLOCK; ++t) {
     const int64_t col = cbase + (int64_t)t * TILE;
-    const bool ok = row_real && t < nt && col < a.n;
+    const bool ok = w == 0 && row_real && t < nt && col < a.n;
     const float s = ok ? a.scales[row * a.G + col / a.gsz] : 1.f;
     sv[t] = s;
     iv[t] = 1.f / s;
@@ -154,74 +183,65 @@ __global__ void __launch_bounds__(32) k_gptq_leaf(int c0, int nt, GptqArgs a) {
   stamp_begin(a.stamp);
   // X of the strip's range: all its 16-byte chunks in flight at once
   const int chunks_per_row = nt * TILE / 4;
-  for (int c = p; c < TILE * chunks_per_row; c += 32) {
+  for (int c = tid; c < TILE * chunks_per_row; c += GQ_THREADS) {
     const int i = c / chunks_per_row, k = c % chunks_per_row;
     gq_cp_async16(&S.Xin[i][4 * k], a.X + (r0 + i) * a.ldx + cbase + 4 * k);
   }
   asm volatile("cp.async.commit_group;" ::: "memory");
   asm volatile("cp.async.wait_group 0;" ::: "memory");
-  __syncwarp();
+  __syncthreads();
 
   constexpr float R = 12582912.f;   // 1.5 * 2^23: fl(v + R) - R rounds v to an integer
   const float fq = (float)a.qmax;
   bool bad = false;
   for (int t = 0; t < nt; ++t) {
-    const int64_t col0 = cbase + (int64_t)t * TILE;
-    float acc[TILE];
+    // T1 = the window of tile t, one 8-column slice per warp, every entry
+    // summed over g = 1 .. t in that order
+    if (t >= 1) gptq_window<1>(S, t, 1, t, w, nullptr, S.T1, lane);
+    __syncthreads();   // S.T1 complete
+    if (w == 0) {
+      const int64_t col0 = cbase + (int64_t)t * TILE;
+      float acc[TILE];
 #pragma unroll
-    for (int q4 = 0; q4 < TILE / 4; ++q4) {
-      const float4 v = *reinterpret_cast<const float4*>(&S.Xin[p][t * TILE + 4 * q4]);
-      acc[4 * q4] = v.x;
-      acc[4 * q4 + 1] = v.y;
-      acc[4 * q4 + 2] = v.z;
-      acc[4 * q4 + 3] = v.w;
-    }
-    // the range's earlier tiles: x += sum_g E[I, J-g] L^A[J, J-g]^T
-    if (t > 0) {
-      __syncwarp();                     // this warp's errors of tile t - 1 are in S.Es
-      gptq_window(S, t, p);
-#pragma unroll
-      for (int q = 0; q < TILE; ++q) acc[q] += S.T1[p][q];
-      __syncwarp();                     // S.T1 read before the next tile writes it
-    }
-    // the tile's 32 steps; the unit diagonal of L^A[J, J] is this entry's own
-    const float(*L0)[LEAF_BLOCK_LD] = S.LA[t * (t + 1) / 2];
-    const float s = sv[t], inv = iv[t], mz = -zv[t];
-#pragma unroll
-    for (int q = 0; q < TILE; ++q) {
-      const float x = acc[q];
-      const float tc = fminf(fmaxf(fmaf(x, inv, R), R + mz), R + fq + mz);
-      const float mk = (row_real && col0 + q < a.n) ? 1.f : 0.f;
-      const float e = fmaf(s * mk, tc - R, x * -mk);   // s (c - z) - x, rounded once
-      bad |= !isfinite(x);
-      S.Xo[p][t * TILE + q] = x;
-      S.Es[t][p][q] = e;
-      S.Cs[p][t * TILE + q] = (uint8_t)(int)(tc - (R + mz));
-#pragma unroll
-      for (int q4 = (q + 1) / 4; q4 < TILE / 4; ++q4) {
-        const float4 l = *reinterpret_cast<const float4*>(&L0[q][4 * q4]);
-        if (4 * q4 > q) acc[4 * q4] = fmaf(e, l.x, acc[4 * q4]);
-        if (4 * q4 + 1 > q) acc[4 * q4 + 1] = fmaf(e, l.y, acc[4 * q4 + 1]);
-        if (4 * q4 + 2 > q) acc[4 * q4 + 2] = fmaf(e, l.z, acc[4 * q4 + 2]);
-        if (4 * q4 + 3 > q) acc[4 * q4 + 3] = fmaf(e, l.w, acc[4 * q4 + 3]);
+      for (int q4 = 0; q4 < TILE / 4; ++q4) {
+        const float4 v = *reinterpret_cast<const float4*>(&S.Xin[p][t * TILE + 4 * q4]);
+        acc[4 * q4] = v.x;
+        acc[4 * q4 + 1] = v.y;
+        acc[4 * q4 + 2] = v.z;
+        acc[4 * q4 + 3] = v.w;
       }
+      if (t >= 1) {
+#pragma unroll
+        for (int q = 0; q < TILE; ++q) acc[q] += S.T1[p][q];
+      }
+      // the tile's 32 steps; the unit diagonal of L^A[J, J] is this entry's own
+      const float(*L0)[LEAF_BLOCK_LD] = S.LA[t * (t + 1) / 2];
+      const float s = sv[t], inv = iv[t], mz = -zv[t];
+#pragma unroll
+      for (int q = 0; q < TILE; ++q) {
+        const float x = acc[q];
+        const float tc = fminf(fmaxf(fmaf(x, inv, R), R + mz), R + fq + mz);
+        const float mk = (row_real && col0 + q < a.n) ? 1.f : 0.f;
+        const float e = fmaf(s * mk, tc - R, x * -mk);   // s (c - z) - x, rounded once
+        bad |= !isfinite(x);
+        S.Xo[p][t * TILE + q] = x;
+        S.Es[t][p][q] = e;
+        S.Cs[p][t * TILE + q] = (uint8_t)(int)(tc - (R + mz));
+#pragma unroll
+        for (int q4 = (q + 1) / 4; q4 < TILE / 4; ++q4) {
+          const float4 l = *reinterpret_cast<const float4*>(&L0[q][4 * q4]);
+          if (4 * q4 > q) acc[4 * q4] = fmaf(e, l.x, acc[4 * q4]);
+          if (4 * q4 + 1 > q) acc[4 * q4 + 1] = fmaf(e, l.y, acc[4 * q4 + 1]);
+          if (4 * q4 + 2 > q) acc[4 * q4 + 2] = fmaf(e, l.z, acc[4 * q4 + 2]);
+          if (4 * q4 + 3 > q) acc[4 * q4 + 3] = fmaf(e, l.w, acc[4 * q4 + 3]);
+        }
+      }
+    } else if (t >= 1) {
+      gptq_store_tile(S, a, r0, cbase, t - 1, tid - 32, GQ_THREADS - 32);
     }
+    __syncthreads();   // tile t's values, errors and codes in shared memory
   }
-  __syncwarp();
-  // outputs, coalesced (lane = column): pre-rounding values, codes, and E as
-  // an exact tf32 hi/lo pair for the column band
-  for (int i = 0; i < TILE; ++i) {
-    const int64_t r = r0 + i;
-    for (int c = p; c < nt * TILE; c += 32) {
-      const int64_t o = r * a.ldx + cbase + c;
-      a.X[o] = S.Xo[i][c];
-      const float e = S.Es[c / TILE][i][c % TILE];
-      const float hi = tf32_hi(e);
-      a.EH[o] = hi;
-      a.EL[o] = e - hi;
-      if (r < a.m && cbase + c < a.n) a.codes[r * a.n + cbase + c] = S.Cs[i][c];
-    }
-  }
+  gptq_store_tile(S, a, r0, cbase, nt - 1, tid, GQ_THREADS);
   if (bad) raise_status(a.status, BAKRON_ERR_NONFINITE);
   stamp_end(a.stamp);
 }
@@ -239,9 +259,9 @@ void gq_leaf(GqRun& r, int c0, int c1) {
   LaunchScope ls(kFamLeaf, r.s, 2.0 * TILE * TILE * TILE * r.la.Mt * (c1 - c0) * (c1 - c0 + 1) / 2);
   GptqArgs la = r.la;
   la.stamp = ls.stamp();
-  if (launch_pdl(k_gptq_leaf, dim3(r.la.Mt), dim3(32), sizeof(GptqSmem), r.s, c0, c1 - c0, la) !=
-      cudaSuccess)
-    r.rc = BAKRON_ERR_CUDA;
+  const cudaError_t e = launch_pdl(k_gptq_leaf, dim3(r.la.Mt), dim3(GQ_THREADS), sizeof(GptqSmem),
+                                   r.s, c0, c1 - c0, la);
+  if (e != cudaSuccess) r.rc = cuda_fail(e, __FILE__, __LINE__);
 }
 
 void gq_rec(GqRun& r, int c0, int c1) {
