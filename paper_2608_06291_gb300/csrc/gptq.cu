@@ -214,27 +214,42 @@ __global__ void __launch_bounds__(GQ_THREADS) k_gptq_leaf(int c0, int nt, GptqAr
 #pragma unroll
         for (int q = 0; q < TILE; ++q) acc[q] += S.T1[p][q];
       }
-      // the tile's 32 steps; the unit diagonal of L^A[J, J] is this entry's own
+      // the tile's 32 steps; the unit diagonal of L^A[J, J] is this entry's own.
+      // Row q + 1 of L^A[J, J] is read into registers during step q, before
+      // that step's shared-memory stores, so its loads are never waited for.
       const float(*L0)[LEAF_BLOCK_LD] = S.LA[t * (t + 1) / 2];
       const float s = sv[t], inv = iv[t], mz = -zv[t];
+      float4 Lc[TILE / 4], Ln[TILE / 4];
+#pragma unroll
+      for (int q4 = 0; q4 < TILE / 4; ++q4) {
+        Lc[q4] = *reinterpret_cast<const float4*>(&L0[0][4 * q4]);
+        Ln[q4] = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
 #pragma unroll
       for (int q = 0; q < TILE; ++q) {
+        if (q + 1 < TILE) {
+#pragma unroll
+          for (int q4 = (q + 2) / 4; q4 < TILE / 4; ++q4)
+            Ln[q4] = *reinterpret_cast<const float4*>(&L0[q + 1][4 * q4]);
+        }
         const float x = acc[q];
         const float tc = fminf(fmaxf(fmaf(x, inv, R), R + mz), R + fq + mz);
         const float mk = (row_real && col0 + q < a.n) ? 1.f : 0.f;
         const float e = fmaf(s * mk, tc - R, x * -mk);   // s (c - z) - x, rounded once
-        bad |= !isfinite(x);
-        S.Xo[p][t * TILE + q] = x;
-        S.Es[t][p][q] = e;
-        S.Cs[p][t * TILE + q] = (uint8_t)(int)(tc - (R + mz));
 #pragma unroll
         for (int q4 = (q + 1) / 4; q4 < TILE / 4; ++q4) {
-          const float4 l = *reinterpret_cast<const float4*>(&L0[q][4 * q4]);
+          const float4 l = Lc[q4];
           if (4 * q4 > q) acc[4 * q4] = fmaf(e, l.x, acc[4 * q4]);
           if (4 * q4 + 1 > q) acc[4 * q4 + 1] = fmaf(e, l.y, acc[4 * q4 + 1]);
           if (4 * q4 + 2 > q) acc[4 * q4 + 2] = fmaf(e, l.z, acc[4 * q4 + 2]);
           if (4 * q4 + 3 > q) acc[4 * q4 + 3] = fmaf(e, l.w, acc[4 * q4 + 3]);
         }
+        bad |= !isfinite(x);
+        S.Xo[p][t * TILE + q] = x;
+        S.Es[t][p][q] = e;
+        S.Cs[p][t * TILE + q] = (uint8_t)(int)(tc - (R + mz));
+#pragma unroll
+        for (int q4 = 0; q4 < TILE / 4; ++q4) Lc[q4] = Ln[q4];
       }
     } else if (t >= 1) {
       gptq_store_tile(S, a, r0, cbase, t - 1, tid - 32, GQ_THREADS - 32);
