@@ -256,7 +256,9 @@ def _block_note(m, n, k):
 
 
 def _timed(fn):
-    """Wall time of fn() and the host threads it kept busy on average."""
+    """Wall time of fn() and the host threads it kept busy on average (CPU
+    time / wall time, at least 1): the `cores` of a cpu_baseline; the host's
+    logical CPUs and BLAS threads are reported beside it (`host_info`)."""
     c0 = os.times()
     t0 = time.perf_counter()
     fn()
@@ -281,13 +283,14 @@ def extra_cpu_baseline(workload, data):
         wall, cores = _timed(lambda: O.gram(X, alpha=1.0 / k_s))
         return {"value": d * (d + 1) * k_s / wall, "unit": "flop/s", "cores": cores,
                 "kind": "oracle",
-                "sample": f"first {k_s} of the rows ({k_s} x {d}), float64 Gram, {wall:.2f} s wall"}
+                "sample": f"first {k_s} of the rows ({k_s} x {d}), float64 Gram, {wall:.2f} s wall",
+                "host": host_info()}
     if workload == "symgrid":
         W = data["W"]
         wall, cores = _timed(lambda: O.symmetric_grid(W.astype(np.float32), 3, 0, 50))
         return {"value": W.size / wall, "unit": "entries/s", "cores": cores, "kind": "oracle",
                 "sample": f"first {W.shape[0]} rows ({W.shape[0]} x {W.shape[1]}), l = 3, "
-                          f"50 shrink steps, {wall:.2f} s wall"}
+                          f"50 shrink steps, {wall:.2f} s wall", "host": host_info()}
     W, LA, LB, bits = data["W"], data["LA"], data["LB"], data["bits"]
     # the per-row grid of the full rows (data["rows"]), which the block's
     # columns share: the block is then an exact part of the full solve
