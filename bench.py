@@ -633,7 +633,7 @@ def run_extra(args):
                weights (one bakron_grid_symmetric call per step);
       batched  the 4096 x 4096 weights as 32 heads of 128 rows, each with its
                own 128 x 128 output-side Gram and the layer's input-side one,
-               one bakron_solve_batched call over 16 lanes per step (CUDA graph
+               one bakron_solve_batched call over 32 lanes per step (CUDA graph
                replay; the same call on one lane is timed for context);
       gptq     the 4096 x 4096 solve with B = I (GPTQ, the method's special
                case) under the layer's input-side factor, bakron_solve_gptq,
@@ -717,7 +717,7 @@ def run_extra(args):
         cfg2 = WL.CONFIGS[2]
         W, A, _ = WL.make(cfg2, device=dev)
         Hh, mh, n = 32, 128, cfg2.n
-        lanes = 16
+        lanes = int(os.environ.get("BAKRON_BENCH_LANES", "32"))   # one per head
         Ws = [W[h * mh:(h + 1) * mh] for h in range(Hh)]
         # the shared input-side factor once; each head's output-side factor
         # from a small prepare of its own Gram; assembled per head
@@ -764,7 +764,7 @@ def run_extra(args):
         mma = None
         unit = "entries/s"
         metric = ("per-head BaKron solves: 32 heads of 128x4096 (bf16, 4-bit), "
-                  "16 lanes, entries/s")
+                  f"{lanes} lanes, entries/s")
         per_launch = launches_per
         F_alg = Hh * f_alg(mh, n)
         p_eff, roof_src = fp32_effective_peak(peaks)
