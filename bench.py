@@ -742,8 +742,8 @@ def run_extra(args):
                                        sync=False, out=outs)
             return gr, wsb
         g1, _ = graph_of(1)
-        launches_per = P.bakron_last_launches()
         gS, wsS = graph_of(lanes)
+        launches_per = P.bakron_last_launches()   # the timed call's (captured last)
 
         def one_lane():
             g1.replay()

@@ -8,7 +8,10 @@
 // at each step of its wavefront, so the problems run side by side: problem h
 // is enqueued on lane h mod S of S library-owned streams, which fork from the
 // caller's stream through an event and join back into it through one event
-// per lane.  Each lane owns one slice of the workspace and runs its problems
+// per lane.  With one lane per problem (S = H), the leaves of all problems
+// share one launch per tile anti-diagonal on the caller's stream and only the
+// band products run on the lanes (solve_heads_impl), joined before and
+// forked after every block of leaves.  Each lane owns one slice of the workspace and runs its problems
 // one after another; a problem's kernels are those of bakron_solve (same
 // schedule table, same programmatic dependent launch within its lane).  The
 // fork/join is made of event records and waits only, so the whole call can
@@ -106,7 +109,23 @@ int bakron_solve_batched(int H, const void* const* W, int wdtype, int m, int n, 
     BK_CUDA_OK(cudaMemsetAsync(ws + (size_t)l * slice, 0, 256, L->stream[l]));
   }
   int launches = 0;
-  for (int h = 0; h < H && rc == BAKRON_OK; ++h) {
+  bool done = false;
+  if (S == H && H >= 2) {
+    // one lane per problem: the leaves of all problems share one launch per
+    // tile anti-diagonal on the caller's stream, the band products run per
+    // problem on the lanes (unless the shape's schedule needs dataflow leaves
+    // or persistent subtrees: then nothing was enqueued, and the lanes run
+    // the problems one by one below)
+    rc = solve_heads_impl(H, W, wdtype, m, n, ldw, factors, (1 << bits) - 1, group_size, codes,
+                          scales, zeros, ws, slice, s, L->stream, L->fork, L->done);
+    if (rc == BAKRON_ERR_INVALID_ARG) {
+      rc = BAKRON_OK;
+    } else {
+      done = true;
+      launches = launch_count();
+    }
+  }
+  for (int h = 0; h < H && rc == BAKRON_OK && !done; ++h) {
     const int l = h % S;
     rc = solve_impl(W[h], wdtype, m, n, ldw, factors[h], (1 << bits) - 1, group_size, codes[h],
                     scales[h], zeros[h], nullptr, ws + (size_t)l * slice, L->stream[l], nullptr,

@@ -863,6 +863,42 @@ __global__ void __launch_bounds__(LEAF_THREADS) k_leaf(int K, LeafArgs a) {
   leaf_tile<LEAF_PDL, P>(a, I, K - I, S);
 }
 
+// The leaves of anti-diagonal K of H problems of one shape in one launch
+// (blockIdx.y = problem): problem h's workspace is `slice` bytes after problem
+// h - 1's, its factor buffer and outputs are its own.
+constexpr int MAX_HEADS = 32;
+struct LeafHeads {
+  LeafArgs base;       // problem 0
+  int64_t slice;       // bytes between consecutive problems' workspaces
+  const float* LBblk[MAX_HEADS];
+  const float* LAblk[MAX_HEADS];
+  uint8_t* codes[MAX_HEADS];
+  const float* scales[MAX_HEADS];
+  const float* zeros[MAX_HEADS];
+};
+
+template <int P>
+__global__ void __launch_bounds__(LEAF_THREADS) k_leaf_heads(int K, const __grid_constant__ LeafHeads L) {
+  extern __shared__ __align__(16) unsigned char leaf_smem[];
+  LeafSmem& S = *reinterpret_cast<LeafSmem*>(leaf_smem);
+  const int h = blockIdx.y;
+  const int64_t ds = (int64_t)h * L.slice;
+  LeafArgs a = L.base;
+  a.X = (float*)((char*)a.X + ds);
+  a.EtH = (float*)((char*)a.EtH + ds);
+  a.EtL = (float*)((char*)a.EtL + ds);
+  a.EtF = (float*)((char*)a.EtF + ds);
+  a.Gout = (float*)((char*)a.Gout + ds);
+  a.status = (int*)((char*)a.status + ds);
+  a.LBblk = L.LBblk[h];
+  a.LAblk = L.LAblk[h];
+  a.codes = L.codes[h];
+  a.scales = L.scales[h];
+  a.zeros = L.zeros[h];
+  const int I = max(0, K - (a.Nt - 1)) + blockIdx.x;
+  leaf_tile<LEAF_PDL, P>(a, I, K - I, S);
+}
+
 // A whole block of leaves [k, l) in one launch (LEAF_FLOW).  The block's
 // tiles are numbered by anti-diagonal, then row; CTAs take them in that order
 // from a counter, and a tile waits only for tiles numbered before it, which
@@ -1336,10 +1372,21 @@ static cudaError_t launch_leaf_window(int window, dim3 grid, dim3 block, size_t 
   return launch_leaf_window<0>(window, grid, block, sm, s, K, la);
 }
 
-// dynamic shared memory of k_leaf<P> .. k_leaf<LEAF_WINDOW>
+template <int P>
+static cudaError_t launch_heads_window(int window, dim3 grid, dim3 block, size_t sm,
+                                       cudaStream_t s, int K, const LeafHeads& lh) {
+  if (window == P || P == LEAF_WINDOW) return launch_pdl(k_leaf_heads<P>, grid, block, sm, s, K, lh);
+  if constexpr (P < LEAF_WINDOW)
+    return launch_heads_window<P + 1>(window, grid, block, sm, s, K, lh);
+  return cudaErrorInvalidValue;
+}
+
+// dynamic shared memory of k_leaf<P>, k_leaf_heads<P> .. (P up to LEAF_WINDOW)
 template <int P>
 static cudaError_t set_leaf_smem(int bytes) {
   cudaError_t e = cudaFuncSetAttribute(k_leaf<P>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_leaf_heads<P>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
   if constexpr (P < LEAF_WINDOW)
     if (e == cudaSuccess) e = set_leaf_smem<P + 1>(bytes);
   return e;
@@ -1558,15 +1605,15 @@ long long* g_diag_leaf_clk = nullptr;
 // `keep_status`: leave the status word as it is (a batch of solves sharing the
 // workspace keeps the first error of any of them); the grid-barrier words
 // after it are cleared either way.
-int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
-               int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
-               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
-               bool keep_status) {
+// The arguments of one solve of W (m x n) in `workspace` on stream s, with
+// schedule tu; the tensor maps of the band stages built when they are used.
+static int init_solve_args(SolveArgs& a, int m, int n, const void* factors, int qmax,
+                           int group_size, uint8_t* codes, float* scales, float* zeros,
+                           void* workspace, cudaStream_t s, const Tuning& tu) {
   FactorLayout fl(m, n);
   SolveLayout sl(m, n);
   char* ws = (char*)workspace;
   const char* f = (const char*)factors;
-  SolveArgs a;
   a.m = m; a.n = n;
   a.Mt = ceil_div(m, TILE); a.Nt = ceil_div(n, TILE);
   a.gsz = group_size == 0 ? n : group_size;
@@ -1594,37 +1641,50 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
   a.ba = BandArgs{a.LBH, a.LBL, a.mp, a.EtH, a.EtL, a.mp, a.LAH, a.LAL, a.np,
                   a.MH, a.ML, a.np, a.X, a.np, nullptr};
   a.profiling = profiling_on();
+  BK_CUDA_OK(ensure_leaf_attrs());
+  a.tc_min_band = tu.tc_min_band;         // 0 or less: tensor cores off
+  a.fused_max_band = tu.fused_max_band;
+  a.subtree_max = tu.subtree_max;         // 0 or 1: no persistent subtrees
+  a.leaf_block = std::min(std::max(tu.leaf_block, 1), LEAF_WINDOW + 1);
+  if (a.subtree_max > MAX_SUBTREE) a.subtree_max = MAX_SUBTREE;
+  a.subtree_grid = 0;
+  if (a.subtree_max >= 2) {
+    const int cap = subtree_capacity();
+    if (cap < 0) return BAKRON_ERR_CUDA;
+    a.subtree_grid = cap;
+  }
+  a.spin_cycles = spin_cycles_from_env();
+  a.leaf_flow = tu.leaf_flow != 0;
+  a.flow_grid = 0;
+  a.flow_claim = (unsigned*)(ws + sl.off_flow);
+  a.flow_done = a.flow_claim + FLOW_COUNTERS;
+  a.ntp = (int)(sl.np / TILE);
+  if (a.leaf_flow) {
+    a.flow_grid = flow_capacity();
+    if (a.flow_grid <= 0) return BAKRON_ERR_CUDA;
+  }
+  a.tc_ready = false;
+  if (a.tc_min_band > 0) {
+    a.tco = TcOperands{a.mp, a.np, a.Mt, a.Nt, a.LBH, a.LBL, a.LAH, a.LAL,
+                       a.EtH, a.EtL, a.MH, a.ML, a.X, a.status};
+    a.tc_ready = tc_band_maps(a.tcm, a.tco);
+    if (!a.tc_ready) return BAKRON_ERR_CUDA;
+  }
+  return BAKRON_OK;
+}
+
+int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* factors, int qmax,
+               int group_size, uint8_t* codes, float* scales, float* zeros, float* prerounding,
+               void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
+               bool keep_status) {
+  SolveLayout sl(m, n);
+  char* ws = (char*)workspace;
+  SolveArgs a;
   {
-    BK_CUDA_OK(ensure_leaf_attrs());
     const Tuning tu = force ? *force : tuning_for(m, n);
-    a.tc_min_band = tu.tc_min_band;         // 0 or less: tensor cores off
-    a.fused_max_band = tu.fused_max_band;
-    a.subtree_max = tu.subtree_max;         // 0 or 1: no persistent subtrees
-    a.leaf_block = std::min(std::max(tu.leaf_block, 1), LEAF_WINDOW + 1);
-    if (a.subtree_max > MAX_SUBTREE) a.subtree_max = MAX_SUBTREE;
-    a.subtree_grid = 0;
-    if (a.subtree_max >= 2) {
-      const int cap = subtree_capacity();
-      if (cap < 0) return BAKRON_ERR_CUDA;
-      a.subtree_grid = cap;
-    }
-    a.spin_cycles = spin_cycles_from_env();
-    a.leaf_flow = tu.leaf_flow != 0;
-    a.flow_grid = 0;
-    a.flow_claim = (unsigned*)(ws + sl.off_flow);
-    a.flow_done = a.flow_claim + FLOW_COUNTERS;
-    a.ntp = (int)(sl.np / TILE);
-    if (a.leaf_flow) {
-      a.flow_grid = flow_capacity();
-      if (a.flow_grid <= 0) return BAKRON_ERR_CUDA;
-    }
-    a.tc_ready = false;
-    if (a.tc_min_band > 0) {
-      a.tco = TcOperands{a.mp, a.np, a.Mt, a.Nt, a.LBH, a.LBL, a.LAH, a.LAL,
-                         a.EtH, a.EtL, a.MH, a.ML, a.X, a.status};
-      a.tc_ready = tc_band_maps(a.tcm, a.tco);
-      if (!a.tc_ready) return BAKRON_ERR_CUDA;
-    }
+    const int rc = init_solve_args(a, m, n, factors, qmax, group_size, codes, scales, zeros,
+                                   workspace, s, tu);
+    if (rc != BAKRON_OK) return rc;
   }
   reset_launch_count();
   if (keep_status)
@@ -1644,6 +1704,115 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
   }
   BK_CUDA_OK(cudaGetLastError());
   return a.rc;
+}
+
+// ------------------------------------------------- problems side by side
+namespace {
+struct HeadsRun {
+  int H;
+  SolveArgs* a;               // per problem, each on its own lane
+  cudaStream_t main;
+  const cudaStream_t* lanes;
+  cudaEvent_t fork;
+  const cudaEvent_t* done;
+  LeafHeads lh;
+  bool on_main;               // the lanes have joined into main since the last fork
+  int rc;
+};
+
+void heads_join(HeadsRun& r) {
+  if (r.on_main) return;
+  for (int h = 0; h < r.H; ++h) {
+    if (cudaEventRecord(r.done[h], r.lanes[h]) != cudaSuccess ||
+        cudaStreamWaitEvent(r.main, r.done[h], 0) != cudaSuccess)
+      r.rc = BAKRON_ERR_CUDA;
+  }
+  r.on_main = true;
+}
+
+void heads_fork(HeadsRun& r) {
+  if (!r.on_main) return;
+  if (cudaEventRecord(r.fork, r.main) != cudaSuccess) r.rc = BAKRON_ERR_CUDA;
+  for (int h = 0; h < r.H; ++h)
+    if (cudaStreamWaitEvent(r.lanes[h], r.fork, 0) != cudaSuccess) r.rc = BAKRON_ERR_CUDA;
+  r.on_main = false;
+}
+
+void heads_rec(HeadsRun& r, int k, int l) {
+  const SolveArgs& a0 = r.a[0];
+  if (l - k <= a0.leaf_block) {
+    heads_join(r);
+    for (int K = k; K < l; ++K) {
+      const int ilo = max(0, K - (a0.Nt - 1)), ihi = min(K, a0.Mt - 1);
+      LaunchScope ls(kFamLeaf, r.main, 2.0 * TILE * TILE * TILE * (1 + window_products(K - k)) *
+                                           (ihi - ilo + 1) * r.H);
+      LeafHeads lh = r.lh;
+      lh.base.stamp = ls.stamp();
+      const cudaError_t e = launch_heads_window<0>(K - k, dim3(ihi - ilo + 1, r.H),
+                                                   dim3(LEAF_THREADS), sizeof(LeafSmem), r.main,
+                                                   K, lh);
+      if (e != cudaSuccess) r.rc = cuda_fail(e, __FILE__, __LINE__);
+    }
+    return;
+  }
+  const int h = (k + l) / 2;
+  heads_rec(r, k, h);
+  heads_fork(r);
+  for (int p = 0; p < r.H; ++p) {
+    band(r.a[p], k, h, l);
+    if (r.a[p].rc != BAKRON_OK) r.rc = r.a[p].rc;
+  }
+  heads_rec(r, h, l);
+}
+}  // namespace
+
+int solve_heads_impl(int H, const void* const* W, int wdt, int m, int n, int64_t ldw,
+                     const void* const* factors, int qmax, int group_size,
+                     uint8_t* const* codes, float* const* scales, float* const* zeros,
+                     char* workspace, size_t slice, cudaStream_t main,
+                     const cudaStream_t* lanes, cudaEvent_t fork, const cudaEvent_t* done) {
+  if (H < 1 || H > MAX_HEADS) return BAKRON_ERR_INVALID_ARG;
+  const Tuning tu = tuning_for(m, n);
+  if (tu.leaf_flow || tu.subtree_max >= 2) return BAKRON_ERR_INVALID_ARG;   // not in this schedule
+  SolveLayout sl(m, n);
+  SolveArgs a[MAX_HEADS];
+  for (int h = 0; h < H; ++h) {
+    const int rc = init_solve_args(a[h], m, n, factors[h], qmax, group_size, codes[h], scales[h],
+                                   zeros[h], workspace + (size_t)h * slice, lanes[h], tu);
+    if (rc != BAKRON_OK) return rc;
+  }
+  HeadsRun r;
+  r.H = H;
+  r.a = a;
+  r.main = main;
+  r.lanes = lanes;
+  r.fork = fork;
+  r.done = done;
+  r.on_main = false;          // the caller forked the lanes from main
+  r.rc = BAKRON_OK;
+  r.lh.base = a[0].la;
+  r.lh.slice = (int64_t)slice;
+  for (int h = 0; h < H; ++h) {
+    r.lh.LBblk[h] = a[h].la.LBblk;
+    r.lh.LAblk[h] = a[h].la.LAblk;
+    r.lh.codes[h] = codes[h];
+    r.lh.scales[h] = scales[h];
+    r.lh.zeros[h] = zeros[h];
+  }
+  reset_launch_count();
+  // per problem on its lane: the grid-barrier words (the caller cleared the
+  // status word), the grid, X from W
+  for (int h = 0; h < H; ++h) {
+    char* ws = workspace + (size_t)h * slice;
+    BK_CUDA_OK(cudaMemsetAsync(ws + sl.off_status + 64, 0, 256 - 64, lanes[h]));
+    launch_grid(W[h], wdt, m, n, ldw, a[h].gsz, a[h].G, a[h].qmax, scales[h], zeros[h], lanes[h]);
+    const int rc = launch_init(W[h], wdt, m, n, ldw, a[h].X, a[h].mp, a[h].np, lanes[h]);
+    if (rc != BAKRON_OK) r.rc = rc;
+  }
+  heads_rec(r, 0, a[0].Mt + a[0].Nt - 1);
+  heads_fork(r);              // the caller joins the lanes into main at the end
+  BK_CUDA_OK(cudaGetLastError());
+  return r.rc;
 }
 
 // The first kernels of a solve: the min-max grid (k_grid) and X from W (k_init).

@@ -20,6 +20,21 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
                void* workspace, cudaStream_t s, const Tuning* force, bool grid_given,
                bool keep_status);
 
+// H <= 32 problems of one shape solved side by side, problem h in the
+// workspace slice `slice` bytes after problem h - 1's: each tile anti-diagonal's
+// leaves of all problems in one launch on `main`, each node's band products
+// per problem on lanes[h]; the lanes must have been forked from `main` (an
+// event recorded on main and waited on by every lane), and the caller joins
+// them back afterwards; status words are cleared by the caller.  Returns
+// BAKRON_ERR_INVALID_ARG, enqueueing nothing, when the shape's schedule uses
+// dataflow leaves or persistent subtrees (the caller then runs the problems
+// one by one on the lanes).
+int solve_heads_impl(int H, const void* const* W, int wdt, int m, int n, int64_t ldw,
+                     const void* const* factors, int qmax, int group_size,
+                     uint8_t* const* codes, float* const* scales, float* const* zeros,
+                     char* workspace, size_t slice, cudaStream_t main,
+                     const cudaStream_t* lanes, cudaEvent_t fork, const cudaEvent_t* done);
+
 // The B = I (GPTQ) solve (gptq.cu): grid, X from W, then the column
 // recursion.  Workspace and factor buffer as the general solve (only L^A's
 // planes and leaf blocks are read; the M planes hold E row-major).  Requires

@@ -1,7 +1,10 @@
 """GPU tests of bakron_solve_batched: H independent problems of one shape on
 several lane streams give, problem by problem, the codes of bakron_solve
 (bit for bit: the same kernels in the same order per problem) and agree with
-the float64 oracle; the call can be captured into a CUDA graph.
+the float64 oracle; the call can be captured into a CUDA graph.  With one
+lane per problem the leaves of all problems share one launch per tile
+anti-diagonal (the per-problem arithmetic is the same, so the codes are
+still bit for bit those of bakron_solve).
 
 The per-head setting (Sec. 4, local attention Hessians; BoA): W_Q of one
 layer split into heads of 64 rows, a shared input-side A and one small
@@ -36,8 +39,12 @@ def _heads(H, mh, n, seed):
     return W, A, Bs
 
 
-@pytest.mark.parametrize("streams", [1, 3, 8])
-def test_batched_equals_single_solves(streams):
+@pytest.mark.parametrize("streams,tc", [(1, False), (3, False), (8, False), (6, True), (2, True)])
+def test_batched_equals_single_solves(streams, tc, monkeypatch):
+    if tc:   # small leaf blocks and tensor cores on every node: band stages on each lane
+        monkeypatch.setenv("BAKRON_LEAF_BLOCK", "4")
+        monkeypatch.setenv("BAKRON_TC_MIN_BAND", "2")
+        monkeypatch.setenv("BAKRON_SUBTREE_MAX", "0")
     H, mh, n = 6, 64, 200
     W, A, Bs = _heads(H, mh, n, 31)
     Wd = W.cuda().to(torch.bfloat16)
@@ -78,15 +85,15 @@ def test_batched_matches_oracle_with_groups():
             np.testing.assert_array_equal(c, ref.codes)
 
 
-def test_batched_graph_capture():
+@pytest.mark.parametrize("S", [3, 5])
+def test_batched_graph_capture(S):
     """Captured once (after a first eager call created the lanes), replayed
-    on new inputs: the results follow the inputs."""
+    on new inputs: the results follow the inputs (S = 5: one lane per problem)."""
     H, mh, n = 5, 64, 256
     W, A, Bs = _heads(H, mh, n, 77)
     fs = [P.bakron_prepare(A.cuda(), Bs[h].cuda(), 0.01) for h in range(H)]
     Wd = W.cuda()
     Ws = [Wd[h * mh:(h + 1) * mh] for h in range(H)]
-    S = 3
     ws = torch.empty(P.bakron_batched_workspace_bytes(mh, n, S), dtype=torch.uint8, device="cuda")
     outs = P.bakron_solve_batched(Ws, fs, 4, 0, streams=S, workspace=ws)
     torch.cuda.synchronize()
@@ -107,8 +114,8 @@ def test_batched_graph_capture():
 
 def test_batched_bench_workload_certificate():
     """The bench's workload: the 4096 x 4096 layer as 32 heads of 128 x 4096
-    over 16 lanes, each head certified (teacher-forced, every entry) against
-    fp64 factors of its own damped Grams."""
+    over 32 lanes (one per head), each head certified (teacher-forced, every
+    entry) against fp64 factors of its own damped Grams."""
     cfg = WL.CONFIGS[2]
     W, A, _ = WL.make(cfg, device="cuda")
     Hh, mh, n = 32, 128, cfg.n
@@ -120,7 +127,7 @@ def test_batched_bench_workload_certificate():
         LBh, _, rBh, _ = P.bakron_get_factors(P.bakron_prepare(Bs[h], Bs[h], cfg.damp))
         fs.append(P.bakron_set_factors(LA, LBh, rA, rBh))
     Ws = [W[h * mh:(h + 1) * mh] for h in range(Hh)]
-    outs = P.bakron_solve_batched(Ws, fs, cfg.bits, 0, streams=16)
+    outs = P.bakron_solve_batched(Ws, fs, cfg.bits, 0, streams=32)
     torch.cuda.synchronize()
     RA = O.rev_cholesky(O.damped(to_np(A), cfg.damp))
     W64 = to_np(W.float())
