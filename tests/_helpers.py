@@ -4,7 +4,7 @@ import torch
 
 import oracle as O
 
-TIE_BAND = 1e-4   # grid units: |x/s - (k + 1/2)| below this is a tie (spec bar)
+TIE_BAND = 1e-4   # grid units: |x/s - (k + 1/2)| below this is a tie (the parity bar's tie rule)
 
 
 def to_np(t):

@@ -9,7 +9,7 @@ import oracle as O
 import workloads as WL
 
 
-def test_f_alg_matches_the_survey_table():
+def test_f_alg_matches_the_tabulated_values():
     # 2 x the multiply-adds with structurally nonzero factor operands of Alg. 4
     # down to single entries (cheaper order, strictly-lower triangular parts)
     assert bench.f_alg(128, 128) == pytest.approx(7.168e6, rel=1e-3)

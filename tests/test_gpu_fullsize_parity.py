@@ -12,7 +12,7 @@ fp32 and fp64 arithmetic decide it differently, or an entry up-left of it
 already differs and the error feedback carries that difference along.  A
 *root* mismatch is one with no mismatch anywhere up-left of it; every root
 must lie within 1e-4 grid units of a boundary in the oracle's pre-rounding
-values (the north-star's tie band).  The cascades below the roots are
+values (the parity bar's tie band).  The cascades below the roots are
 reported, not asserted: their size measures how chaotic the feedback is, not
 the kernels.  The match rate, the objectives and their relative difference
 are printed (run pytest with -s to see them).

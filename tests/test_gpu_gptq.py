@@ -9,7 +9,7 @@ tensor-core column bands, bit widths 2-8 and column groups.  At 4096 x 4096
 (the attention-projection workload's W and input-side Gram) the GPU solve with
 its own device prepare is compared free-running with the oracle's own fp64
 solve: with B = I a near-tie decided differently can only disturb the rest of
-its own row, so the spec bar (>= 99.9% identical codes, every first
+its own row, so the parity bar (>= 99.9% identical codes, every first
 difference a tie, objective within 1e-4) applies as stated.
 """
 import numpy as np
