@@ -9,9 +9,10 @@
 // is enqueued on lane h mod S of S library-owned streams, which fork from the
 // caller's stream through an event and join back into it through one event
 // per lane.  With one lane per problem (S = H), the leaves of all problems
-// share one launch per tile anti-diagonal on the caller's stream and only the
-// band products run on the lanes (solve_heads_impl), joined before and
-// forked after every block of leaves.  Each lane owns one slice of the workspace and runs its problems
+// share one launch per tile anti-diagonal on the caller's stream, and so do
+// the tensor-core band stages (one launch per stage, blockIdx.z = problem);
+// only CUDA-core band products of narrow nodes run per problem on the lanes
+// (solve_heads_impl).  Each lane owns one slice of the workspace and runs its problems
 // one after another; a problem's kernels are those of bakron_solve (same
 // schedule table, same programmatic dependent launch within its lane).  The
 // fork/join is made of event records and waits only, so the whole call can

@@ -1757,10 +1757,30 @@ void heads_rec(HeadsRun& r, int k, int l) {
   }
   const int h = (k + l) / 2;
   heads_rec(r, k, h);
-  heads_fork(r);
-  for (int p = 0; p < r.H; ++p) {
-    band(r.a[p], k, h, l);
-    if (r.a[p].rc != BAKRON_OK) r.rc = r.a[p].rc;
+  if (a0.tc_ready && l - k >= a0.tc_min_band) {
+    // both stages for every problem in one tensor-core launch each, on main
+    heads_join(r);
+    const TcMaps* maps[MAX_HEADS];
+    int* status[MAX_HEADS];
+    for (int p = 0; p < r.H; ++p) {
+      maps[p] = &r.a[p].tcm;
+      status[p] = r.a[p].status;
+    }
+    double p1 = 0.0, p2 = 0.0;
+    if (a0.profiling) band_tile_products(a0, k, h, l, p1, p2);
+    const double f = 2.0 * TILE * TILE * TILE * r.H;
+    for (int stage = 1; stage <= 2; ++stage) {
+      LaunchScope ls(stage == 1 ? kFamTc1 : kFamTc2, r.main, f * (stage == 1 ? p1 : p2));
+      const int rc = tc_band_stage_heads(stage, r.H, maps, status, a0.tco, k, h, l, r.main,
+                                         ls.stamp());
+      if (rc != BAKRON_OK) r.rc = rc;
+    }
+  } else {
+    heads_fork(r);
+    for (int p = 0; p < r.H; ++p) {
+      band(r.a[p], k, h, l);
+      if (r.a[p].rc != BAKRON_OK) r.rc = r.a[p].rc;
+    }
   }
   heads_rec(r, h, l);
 }

@@ -22,10 +22,12 @@ int solve_impl(const void* W, int wdt, int m, int n, int64_t ldw, const void* fa
 
 // H <= 32 problems of one shape solved side by side, problem h in the
 // workspace slice `slice` bytes after problem h - 1's: each tile anti-diagonal's
-// leaves of all problems in one launch on `main`, each node's band products
-// per problem on lanes[h]; the lanes must have been forked from `main` (an
-// event recorded on main and waited on by every lane), and the caller joins
-// them back afterwards; status words are cleared by the caller.  Returns
+// leaves of all problems in one launch on `main`, each node's tensor-core band
+// stages of all problems in one launch each on `main`, a narrower node's
+// CUDA-core band products per problem on lanes[h]; the lanes must have been
+// forked from `main` (an event recorded on main and waited on by every
+// lane), and the caller joins them back afterwards; status words are cleared
+// by the caller.  Returns
 // BAKRON_ERR_INVALID_ARG, enqueueing nothing, when the shape's schedule uses
 // dataflow leaves or persistent subtrees (the caller then runs the problems
 // one by one on the lanes).

@@ -564,12 +564,13 @@ __device__ __forceinline__ bool block_of_pair(const TcParams& P, int rank, Block
   return true;
 }
 
+// The kernel body, for the tensor maps of one problem (kernel parameters, so
+// their addresses are those of the parameters) and its status word.
 template <int V>
-__global__ void __launch_bounds__(THREADS, 1)
-k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUtensorMap mapB2,
-          const __grid_constant__ CUtensorMap mapBh, const __grid_constant__ CUtensorMap mapBl,
-          const __grid_constant__ CUtensorMap mapOh, const __grid_constant__ CUtensorMap mapOl,
-          const TcParams P) {
+__device__ __forceinline__ void tc_body(const CUtensorMap& mapA2, const CUtensorMap& mapB2,
+                                        const CUtensorMap& mapBh, const CUtensorMap& mapBl,
+                                        const CUtensorMap& mapOh, const CUtensorMap& mapOl,
+                                        const TcParams& P, int* status) {
   using RG = Ring<V>;
   constexpr bool pair = RG::pair;
   constexpr int NST = RG::stages;
@@ -720,7 +721,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
       }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok || *abort_flag) {
-        if (lane == 0 && !ok) { raise_status(P.status, BAKRON_ERR_TIMEOUT); abort_all(); }
+        if (lane == 0 && !ok) { raise_status(status, BAKRON_ERR_TIMEOUT); abort_all(); }
         // slots loaded in part before the wait: arrive, so that their phase
         // completes once those copies land (the drain below waits for them)
         if (lane == 0) {
@@ -841,7 +842,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
         const int first = last > NST ? last - NST : 0;
         for (int i = first; i < last; ++i) {
           if (!mbar_wait(&full[i % NST], (uint32_t)(i / NST) & 1u, drain))
-            raise_status(P.status, BAKRON_ERR_TIMEOUT);
+            raise_status(status, BAKRON_ERR_TIMEOUT);
         }
       }
     }
@@ -856,7 +857,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
       // the peer: the leader's MMAs write this CTA's TMEM and read its shared
       // memory; its last commit arrives here too once they have completed
       if (nk == 0) mbar_arrive(accum);
-      if (!mbar_wait(accum, 0, drain)) raise_status(P.status, BAKRON_ERR_TIMEOUT);
+      if (!mbar_wait(accum, 0, drain)) raise_status(status, BAKRON_ERR_TIMEOUT);
     } else if (lane == 0) {
       const uint32_t idesc = idesc_tf32(pair ? 2 * BM : BM, BN), idesc_b = idesc_bf16(BM, BN);
       const uint64_t desc0 = smem_desc(smem_u32(smem));   // stage 0, A hi, K step 0
@@ -878,7 +879,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
                (!first || g < NACC ||
                 mbar_wait(&accE[a], (uint32_t)(g / NACC - 1) & 1u, P.spin_cycles));
         if (!ok) {
-          raise_status(P.status, BAKRON_ERR_TIMEOUT);
+          raise_status(status, BAKRON_ERR_TIMEOUT);
           abort_all();
           break;
         }
@@ -924,7 +925,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
         mbar_arrive(accum);
       }
       // wind-down guard: all issued MMAs complete before anyone frees TMEM
-      if (!mbar_wait(accum, 0, drain)) raise_status(P.status, BAKRON_ERR_TIMEOUT);
+      if (!mbar_wait(accum, 0, drain)) raise_status(status, BAKRON_ERR_TIMEOUT);
     }
     __syncwarp();
   } else {
@@ -942,7 +943,7 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
       int ok = 1;
       if (lane == 0) {
         ok = mbar_wait(&accF[a], (uint32_t)(i / NACC) & 1u, P.spin_cycles) ? 1 : 0;
-        if (!ok) { raise_status(P.status, BAKRON_ERR_TIMEOUT); abort_all(); }
+        if (!ok) { raise_status(status, BAKRON_ERR_TIMEOUT); abort_all(); }
         if (*abort_flag) ok = 0;
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -1072,6 +1073,30 @@ k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUt
   }
 }
 
+template <int V>
+__global__ void __launch_bounds__(THREADS, 1)
+k_tc_band(const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUtensorMap mapB2,
+          const __grid_constant__ CUtensorMap mapBh, const __grid_constant__ CUtensorMap mapBl,
+          const __grid_constant__ CUtensorMap mapOh, const __grid_constant__ CUtensorMap mapOl,
+          const TcParams P) {
+  tc_body<V>(mapA2, mapB2, mapBh, mapBl, mapOh, mapOl, P, P.status);
+}
+
+// One band stage of up to TC_MAX_HEADS problems of one shape in one launch
+// (blockIdx.z = problem): each problem's six tensor maps and status word
+// (about 25 KB of kernel parameters in all, within the 32 KB limit).
+constexpr int TC_MAX_HEADS = 32;
+struct TcHeads {
+  CUtensorMap maps[TC_MAX_HEADS][6];   // A2, B2, Bh, Bl, Oh, Ol per problem
+  int* status[TC_MAX_HEADS];
+  TcParams P;
+};
+
+__global__ void __launch_bounds__(THREADS, 1) k_tc_heads(const __grid_constant__ TcHeads T) {
+  const CUtensorMap* m = T.maps[blockIdx.z];
+  tc_body<V_BAND>(m[0], m[1], m[2], m[3], m[4], m[5], T.P, T.status[blockIdx.z]);
+}
+
 // ------------------------------------------------------------- host side
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
@@ -1154,6 +1179,8 @@ cudaError_t ensure_attr() {
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(k_tc_band<V_PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              PAIR_SMEM_BYTES);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_tc_heads, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   if (e == cudaSuccess) g_attr_done = true;
   return e;
 }
@@ -1399,6 +1426,46 @@ int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, in
                    maps.Eth,
                    maps.Etl, maps.X32, maps.X32, P);
   return BK_CUDA_RC(e);
+}
+
+int tc_band_stage_heads(int stage, int H, const TcMaps* const* maps, int* const* status,
+                        const TcOperands& op, int k, int h, int l, cudaStream_t s,
+                        unsigned long long* stamp) {
+  if (H < 1 || H > TC_MAX_HEADS) return BAKRON_ERR_INVALID_ARG;
+  BK_CUDA_OK(ensure_attr());
+  static thread_local TcHeads T;   // 25 KB: kept off the stack
+  TcParams& P = T.P;
+  P = TcParams{};
+  P.stamp = stamp;
+  P.raster = raster_rows();
+  P.mode = stage == 1 ? MODE_STAGE1 : MODE_STAGE2;
+  P.k = k; P.h = h; P.l = l;
+  P.Mt = op.Mt; P.Nt = op.Nt;
+  P.ldo = op.np;
+  P.spin_cycles = spin_cycles_from_env();
+  int rlo = -1, rhi = -1, width = 0;
+  const int nb_rows = (int)(op.mp / BM);
+  for (int rb = 0; rb < nb_rows; ++rb) {
+    int cl, ch;
+    if (!band_row_span(P.mode, k, h, l, op.Mt, op.Nt, rb, cl, ch)) continue;
+    if (rlo < 0) rlo = rb;
+    rhi = rb;
+    width = std::max(width, ch - cl + 1);
+  }
+  if (rlo < 0) return BAKRON_OK;
+  P.row0 = rlo;
+  for (int p = 0; p < H; ++p) {
+    const TcMaps& m = *maps[p];
+    CUtensorMap* d = T.maps[p];
+    if (stage == 1) {
+      d[0] = m.LB2; d[1] = m.Et2; d[2] = m.Eth; d[3] = m.Etl; d[4] = m.Mh; d[5] = m.Ml;
+    } else {
+      d[0] = m.M2; d[1] = m.LA2; d[2] = m.Eth; d[3] = m.Etl; d[4] = m.X32; d[5] = m.X32;
+    }
+    T.status[p] = status[p];
+  }
+  return BK_CUDA_RC(launch_pdl(k_tc_heads, dim3(width, rhi - rlo + 1, H), dim3(THREADS),
+                               SMEM_BYTES, s, T));
 }
 
 int tc_cols_stage(const TcMaps& maps, const TcOperands& op, int k, int h, int l, cudaStream_t s,

@@ -36,6 +36,12 @@ long long spin_cycles_from_env();
 int tc_band_stage(int stage, const TcMaps& maps, const TcOperands& op, int k, int h, int l,
                   cudaStream_t s, unsigned long long* stamp = nullptr);
 
+// Stage `stage` of node (k, h, l) for H <= 32 problems of one shape (op gives
+// the shape; maps[p] and status[p] are problem p's) in one launch.
+int tc_band_stage_heads(int stage, int H, const TcMaps* const* maps, int* const* status,
+                        const TcOperands& op, int k, int h, int l, cudaStream_t s,
+                        unsigned long long* stamp = nullptr);
+
 // The column-band update of the B = I (GPTQ) schedule over 128 x 128 output
 // blocks: X[:, S2] += E[:, S1] L^A[S2, S1]^T, S1 = tile columns [k, h), S2 =
 // [h, l), with E in the M planes (row-major hi/lo).
