@@ -174,6 +174,12 @@ def _traffic(workload, family, launches):
     return None if per_step is None else per_step / launches
 
 
+def _traffic_warm(workload, family, launches):
+    """The same per launch from the launch list taken without ncu's L2 flush
+    between launches (`<family>_warm_l2`), or None."""
+    return _traffic(workload, family + "_warm_l2", launches)
+
+
 class ClockSampler:
     """nvidia-smi sampling of SM clocks and throttle reasons (read only)."""
     FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -504,7 +510,8 @@ def run_gpu(args):
                    "bound": "tensor", "achieved": tc_ach, "peak": p_eff, "unit": "TFLOP/s",
                    "frac": tc_ach / p_eff, "peak_source": p_src,
                    "algorithmic_per_step": tc_work, "launches_per_step": tc_n,
-                   "ms_per_step": tc_ms, "traffic": _traffic(wl_key, "tc", tc_n)}
+                   "ms_per_step": tc_ms, "traffic": _traffic(wl_key, "tc", tc_n),
+                   "traffic_warm_l2": _traffic_warm(wl_key, "tc", tc_n)}
     # the leaves against their latency floor: the element anti-diagonals
     # (m + n - 1 dependent rounding steps, Sec. 3.3) at the chain's own
     # measured step time, one tile alone on the GPU
@@ -523,7 +530,8 @@ def run_gpu(args):
                  "floor_ms": floor_ms, "ms_per_step": leaf_ms, "launches_per_step": leaf_n,
                  "schedule_chain_steps": tile_steps,
                  "hbm_gbs": leaf_bytes / (leaf_ms / 1e3) / 1e9 if leaf_ms > 0 else None,
-                 "traffic": _traffic(wl_key, "leaf", leaf_n)}
+                 "traffic": _traffic(wl_key, "leaf", leaf_n),
+                 "traffic_warm_l2": _traffic_warm(wl_key, "leaf", leaf_n)}
     dom = max(groups, key=lambda g: groups[g][0])
     if dom == "tc":
         roof = dict(tc_roof)
