@@ -109,15 +109,19 @@ __global__ void k_potrf_block(RT* C, int64_t ldc, int k0, int b, RT* Dinv, int* 
 }
 
 // ------------------------------------------------------------ SIMT GEMM
-// C[M x N] = beta*C + alpha * A[M x K] * op(B),  op(B) = B (K x N) or B^T
-// (B given N x K).  64 x 64 output tiles, 256 threads, 4 x 4 per thread.
+// C[M x N] = beta*C + alpha * op(A) * op(B):  op(A) = A (M x K) or A^T (A
+// given K x M), op(B) = B (K x N) or B^T (B given N x K).  64 x 64 output
+// tiles, 256 threads, 4 x 4 per thread; each operand is staged with the
+// thread index running along its contiguous dimension.
 // mode bit 1: only tiles with tile_row >= tile_col (lower part, for SYRK).
-// mode bit 2: B is lower triangular (K x N): skip k < tile_col * 64.
+// mode bit 2: op(B) is lower triangular: skip k < tile_col * 64.
+// mode bit 4: op(A) is upper triangular: skip k < tile_row * 64.
+// mode bit 8: op(A) is lower triangular: skip k >= (tile_row + 1) * 64.
 // Each CTA reads all of its A rows before writing, so C may alias A when
 // N <= 64 (the panel solve uses this).
-enum { GM_LOWER_C = 1, GM_TRI_B = 2 };
+enum { GM_LOWER_C = 1, GM_TRI_B = 2, GM_UPPER_A = 4, GM_LOWER_A = 8 };
 
-template <typename RT, bool TRANS_B>
+template <typename RT, bool TRANS_A, bool TRANS_B>
 __global__ void __launch_bounds__(256) k_gemm(int M, int N, int K, RT alpha,
                                               const RT* A, int64_t lda,
                                               const RT* B, int64_t ldb, RT beta,
@@ -129,16 +133,24 @@ __global__ void __launch_bounds__(256) k_gemm(int M, int N, int K, RT alpha,
   const int t = threadIdx.x;
   const int ty = t / 16, tx = t % 16;
   RT acc[4][4] = {};
-  int kbeg = (mode & GM_TRI_B) ? tc * GT : 0;
-  for (int k0 = kbeg; k0 < K; k0 += GK) {
+  int kbeg = 0, kend = K;
+  if (mode & GM_TRI_B) kbeg = max(kbeg, tc * GT);
+  if (mode & GM_UPPER_A) kbeg = max(kbeg, tr * GT);
+  if (mode & GM_LOWER_A) kend = min(kend, (tr + 1) * GT);
+  for (int k0 = kbeg; k0 < kend; k0 += GK) {
     for (int e = t; e < GK * GT; e += 256) {
-      int kk = e % GK, r = e / GK;
-      int gr = tr * GT + r, gk = k0 + kk;
-      As[kk][r] = (gr < M && gk < K) ? A[(int64_t)gr * lda + gk] : RT(0);
-      int c = r, gc = tc * GT + c;
-      RT bv = 0;
-      if (gc < N && gk < K) bv = TRANS_B ? B[(int64_t)gc * ldb + gk] : B[(int64_t)gk * ldb + gc];
-      Bs[kk][c] = bv;
+      const int kk = TRANS_A ? e / GT : e % GK, r = TRANS_A ? e % GT : e / GK;
+      const int gr = tr * GT + r, gk = k0 + kk;
+      As[kk][r] = (gr < M && gk < K) ? (TRANS_A ? A[(int64_t)gk * lda + gr]
+                                                : A[(int64_t)gr * lda + gk])
+                                     : RT(0);
+    }
+    for (int e = t; e < GK * GT; e += 256) {
+      const int kk = TRANS_B ? e % GK : e / GT, c = TRANS_B ? e / GK : e % GT;
+      const int gc = tc * GT + c, gk = k0 + kk;
+      Bs[kk][c] = (gc < N && gk < K) ? (TRANS_B ? B[(int64_t)gc * ldb + gk]
+                                                : B[(int64_t)gk * ldb + gc])
+                                     : RT(0);
     }
     __syncthreads();
 #pragma unroll
@@ -170,13 +182,18 @@ __global__ void __launch_bounds__(256) k_gemm(int M, int N, int K, RT alpha,
 
 template <typename RT>
 static void gemm(cudaStream_t s, int M, int N, int K, RT alpha, const RT* A, int64_t lda,
-                 const RT* B, int64_t ldb, bool transB, RT beta, RT* C, int64_t ldc, int mode) {
+                 bool transA, const RT* B, int64_t ldb, bool transB, RT beta, RT* C, int64_t ldc,
+                 int mode) {
   if (M <= 0 || N <= 0) return;
   dim3 grid(ceil_div(N, GT), ceil_div(M, GT));
-  if (transB)
-    k_gemm<RT, true><<<grid, 256, 0, s>>>(M, N, K, alpha, A, lda, B, ldb, beta, C, ldc, mode);
+  if (transA && transB)
+    k_gemm<RT, true, true><<<grid, 256, 0, s>>>(M, N, K, alpha, A, lda, B, ldb, beta, C, ldc, mode);
+  else if (transB)
+    k_gemm<RT, false, true><<<grid, 256, 0, s>>>(M, N, K, alpha, A, lda, B, ldb, beta, C, ldc, mode);
+  else if (transA)
+    k_gemm<RT, true, false><<<grid, 256, 0, s>>>(M, N, K, alpha, A, lda, B, ldb, beta, C, ldc, mode);
   else
-    k_gemm<RT, false><<<grid, 256, 0, s>>>(M, N, K, alpha, A, lda, B, ldb, beta, C, ldc, mode);
+    k_gemm<RT, false, false><<<grid, 256, 0, s>>>(M, N, K, alpha, A, lda, B, ldb, beta, C, ldc, mode);
 }
 
 // Copy a b x b block of Dinv into X's diagonal block (lower part only).
@@ -222,6 +239,36 @@ __global__ void k_assemble(const RT* C, const RT* Xinv, int64_t dp, int d, float
   }
 }
 
+// X[i0 .. i0 + n) x [i0 .. i0 + n) = inverse of the lower triangle of C's
+// diagonal block there, by recursive halving at a multiple of NB: with
+// C = [[C11, 0], [C21, C22]], X11 = C11^-1 and X22 = C22^-1 (recursively; a
+// block of at most NB is the inverse the panel factorisation left in Dinv),
+// X21 = -X22 (C21 X11).  The product C21 X11 is kept transposed in C's upper
+// triangle above the node's diagonal block (C11's rows, C22's columns),
+// which the lower Cholesky factor leaves unused; X above the diagonal stays
+// as zeroed.  Every level is two GEMMs over whole halves, so the work runs
+// on the whole GPU (a block-row recurrence gives each step at most i0 / 64
+// output tiles).
+template <typename RT>
+static void inv_lower(cudaStream_t s, RT* C, RT* X, int64_t dp, const RT* Dinv, int i0, int n) {
+  if (n <= NB) {
+    k_put_diag<RT><<<n, NB, 0, s>>>(Dinv + (int64_t)(i0 / NB) * NB * NB, n, X, dp, i0);
+    return;
+  }
+  const int n1 = (ceil_div(n, NB) / 2) * NB, n2 = n - n1;
+  inv_lower<RT>(s, C, X, dp, Dinv, i0, n1);
+  inv_lower<RT>(s, C, X, dp, Dinv, i0 + n1, n2);
+  RT* R = C + (int64_t)i0 * dp + (i0 + n1);                    // n1 x n2, above the diagonal
+  const RT* C21 = C + (int64_t)(i0 + n1) * dp + i0;            // n2 x n1
+  const RT* X11 = X + (int64_t)i0 * dp + i0;                   // n1 x n1, lower
+  const RT* X22 = X + (int64_t)(i0 + n1) * dp + (i0 + n1);     // n2 x n2, lower
+  RT* X21 = X + (int64_t)(i0 + n1) * dp + i0;                  // n2 x n1
+  // R = (C21 X11)^T = X11^T C21^T  (X11^T upper triangular)
+  gemm<RT>(s, n1, n2, n1, RT(1), X11, dp, true, C21, dp, true, RT(0), R, dp, GM_UPPER_A);
+  // X21 = -X22 R^T  (X22 lower triangular)
+  gemm<RT>(s, n2, n1, n2, RT(-1), X22, dp, false, R, dp, true, RT(0), X21, dp, GM_LOWER_A);
+}
+
 // One Gram -> one unit-lower factor (fp32, Lp x Lp) and its RevCholesky diagonal.
 template <typename RT>
 static int factor_one(const float* H, int d, float damp, float* L, float* Llo, int64_t Lp,
@@ -253,26 +300,14 @@ static int factor_one(const float* H, int d, float damp, float* L, float* Llo, i
     if (rest > 0) {
       RT* P = C + (int64_t)(k0 + b) * dp + k0;
       // panel solve P <- P L_kk^-T  (in place: one CTA per 64 whole rows, N = b <= 64)
-      gemm<RT>(s, rest, b, b, RT(1), P, dp, Dk, NB, true, RT(0), P, dp, 0);
+      gemm<RT>(s, rest, b, b, RT(1), P, dp, false, Dk, NB, true, RT(0), P, dp, 0);
       // trailing update C22 -= P P^T on the lower tiles
       RT* C22 = C + (int64_t)(k0 + b) * dp + (k0 + b);
-      gemm<RT>(s, rest, rest, b, RT(-1), P, dp, P, dp, true, RT(1), C22, dp, GM_LOWER_C);
+      gemm<RT>(s, rest, rest, b, RT(-1), P, dp, false, P, dp, true, RT(1), C22, dp, GM_LOWER_C);
     }
   }
-  // blocked inverse X = C^-1 by block rows:
-  //   X_ii = L_ii^-1,  X[i, 0:i] = -L_ii^-1 (C[i, 0:i] X[0:i, 0:i])
-  for (int i0 = 0; i0 < d; i0 += NB) {
-    const int b = d - i0 < NB ? d - i0 : NB;
-    const RT* Di = Dinv + (int64_t)(i0 / NB) * NB * NB;
-    RT* Xrow = X + (int64_t)i0 * dp;
-    if (i0 > 0) {
-      const RT* Crow = C + (int64_t)i0 * dp;
-      gemm<RT>(s, b, i0, i0, RT(1), Crow, dp, X, dp, false, RT(0), Xrow, dp, GM_TRI_B);
-      // in place: M = b <= 64, so each CTA reads its whole column block first
-      gemm<RT>(s, b, i0, b, RT(-1), Di, NB, Xrow, dp, false, RT(0), Xrow, dp, 0);
-    }
-    k_put_diag<RT><<<b, NB, 0, s>>>(Di, b, X, dp, i0);
-  }
+  // X = C^-1 by recursive halving (inv_lower)
+  inv_lower<RT>(s, C, X, dp, Dinv, 0, d);
   {
     dim3 blk(32, 8), grid((unsigned)(Lp / 32), (unsigned)(Lp / 32));
     k_assemble<RT><<<grid, blk, 0, s>>>(C, X, dp, d, L, Llo, Lp, Lp, rdiag);
