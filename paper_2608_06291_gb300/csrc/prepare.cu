@@ -92,15 +92,25 @@ __global__ void k_potrf_block(RT* C, int64_t ldc, int k0, int b, RT* Dinv, int* 
     }
     __syncthreads();
   }
-  // inverse of the lower-triangular block: column c solved by one thread
-  for (int c = t; c < NB; c += nt) {
-    for (int r = 0; r < NB; ++r) {
-      RT acc = (r == c) ? RT(1) : RT(0);
-      for (int k = c; k < r; ++k) acc -= s[r][k] * inv[k][c];
-      inv[r][c] = (r >= c) ? acc / s[r][r] : RT(0);
-    }
+  // inverse of the lower-triangular block, right-looking: row k of the
+  // inverse is final once divided by the pivot, then every later row r drops
+  // s[r][k] times it (independent updates spread over the whole CTA instead
+  // of one dependent chain per column)
+  for (int e = t; e < NB * NB; e += nt) {
+    const int r = e / NB, c = e % NB;
+    inv[r][c] = (r == c) ? RT(1) : RT(0);
   }
   __syncthreads();
+  for (int k = 0; k < NB; ++k) {
+    for (int c = t; c <= k; c += nt) inv[k][c] /= s[k][k];
+    __syncthreads();
+    const int w = k + 1, rows = NB - 1 - k;
+    for (int e = t; e < rows * w; e += nt) {
+      const int r = k + 1 + e / w, c = e % w;
+      inv[r][c] -= s[r][k] * inv[k][c];
+    }
+    __syncthreads();
+  }
   for (int e = t; e < NB * NB; e += nt) {
     int r = e / NB, c = e % NB;
     if (r < b && c <= r) C[(int64_t)(k0 + r) * ldc + k0 + c] = s[r][c];
