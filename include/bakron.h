@@ -246,15 +246,19 @@ int bakron_sample_sqnorms(const void* Y, int ydtype, int k, int d, int64_t ldy,
  * call: the per-head problems of attention layers whose output-side factor
  * is block diagonal (one B per head, a shared input-side A; the local
  * attention Hessians of Sec. 4 and the BoA setting).  Problem h rounds W[h]
- * under factors[h] exactly as bakron_solve would (same kernels, same
- * schedule table, same codes bit for bit).
+ * under factors[h] exactly as bakron_solve would (the same arithmetic and
+ * schedule table, the same codes bit for bit).
  *   W, factors, codes, scales, zeros  HOST arrays of H device pointers (the
  *            buffers of problem h; factors[h] may repeat); the device
  *            buffers are those of bakron_solve for one m x n problem
  *   streams  S, 1..32: problems run side by side on S library-owned CUDA
  *            streams, problem h on lane h mod S, each lane in order; the
  *            lanes fork from `stream` and join back into it through events,
- *            so later work on `stream` sees every result
+ *            so later work on `stream` sees every result.  With S = H >= 2
+ *            (one lane per problem) the leaves of all problems share one
+ *            launch per tile anti-diagonal and each tensor-core band stage
+ *            one launch, on `stream` itself (unless the shape's schedule
+ *            uses dataflow leaves or persistent subtrees)
  *   workspace device, >= bakron_batched_workspace_bytes(m, n, min(S, H))
  *            bytes: lane l uses slice l (bakron_workspace_bytes(m, n) rounded
  *            up to 256 bytes, at offset l times that)
